@@ -1,0 +1,256 @@
+"""fp64 CPU oracle for PACE's condense-and-extract hot path.
+
+TEST INFRASTRUCTURE ONLY.  Only the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may import this module.  The product path (the
+CUDA library and its binding) never reads it, and it shares no code with them.
+
+Every function is a plain, slow statement of one step of the method, written
+from the paper (arxiv 2608.27206, "PACE: A Unified Condense-and-Extract
+Paradigm for Fast VLM Inference"), in float64, with numpy library primitives
+(matmul, sort, exp) as the only building blocks.  Citations name the paper's
+sections and equations.
+
+Readings taken where the paper is silent or cannot be followed literally
+(each is listed again, with its reason, in the design notes):
+  R1  APC preview feature: the paper's T_v is the output of ViT block 1
+      (Sec. 3.2, "Shallow Feature Preview").  No ViT weights are used here, so
+      the token of patch i is the stand-in T_i = [x_i / 255 ; 1], x_i the
+      14x14x3 patch in (row, column, channel) order, patches in raster order.
+  R2  "top 10 %" of d_i: k_tail = max(1, floor(tail_frac * N + 0.5)).
+  R3  r = min(max(rho, r_min), r_max); r_max is the hard budget cap of
+      Sec. 3.2 "Adaptive Condensation" (default 1, i.e. no cap), r_min = 0.
+  R4  target size: both sides scaled by sqrt(r) (App. B.3) and snapped to the
+      28-pixel merge unit: H' = min(H, max(28, 28 * floor(H sqrt(r) / 28 + 0.5))).
+  R5  bicubic resize: separable cubic convolution (a = -0.5), centre-aligned
+      sampling, support widened by the downscale factor (antialias), window
+      clipped at the border, weights renormalised; round half to even.
+  R6  S_vis: the attention each patch receives in the final ViT block, summed
+      over heads and query rows (softmax over all patches of the image, no
+      mask), then summed over the 4 patches of each 2x2 merge unit.
+  R7  S_llm: text queries over the visual keys only (no mask), GQA head
+      h -> KV head h // (Hq / Hkv), summed over heads and queries.
+  R8  min-max of a constant map gives 0; sigma is the population deviation.
+  R9  top-K ties: the lower index wins; the kept indices are returned in
+      ascending order.  K = floor(p * N_vis + 0.5) clamped to [0, N_vis].
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict, List, Sequence
+
+import numpy as np
+
+PATCH = 14
+MERGE_UNIT = 28
+
+# Hyper-parameters the paper fixes (Sec. 4.1 "Implementation Details", App. B.3).
+ALPHA = 0.6      # global/local balance of Eq. 6
+GAMMA = 1.5      # local contrast scaling of Eq. 5
+TAIL_FRAC = 0.10  # "top 10 %" tail of d_i (Sec. 3.2; App. tail-percentile study)
+TAU = 0.5        # fusion temperature of Eq. 7
+
+
+# ==============================================================================================
+# Condense: Adaptive Pixel Compressor (Sec. 3.2)
+# ==============================================================================================
+def patch_tokens(img: np.ndarray) -> np.ndarray:
+    """Reading R1: stand-in preview tokens T [N, 589] of a uint8 HxWx3 image."""
+    H, W, _ = img.shape
+    gh, gw = H // PATCH, W // PATCH
+    x = img[: gh * PATCH, : gw * PATCH].astype(np.float64) / 255.0
+    x = x.reshape(gh, PATCH, gw, PATCH, 3).transpose(0, 2, 1, 3, 4).reshape(gh * gw, PATCH * PATCH * 3)
+    return np.concatenate([x, np.ones((gh * gw, 1))], axis=1)
+
+
+def global_redundancy(T: np.ndarray, rows_per_block: int = 512) -> float:
+    """Eq. 1: phi = (1/N^2) sum_i sum_j cos(T_i, T_j), summed literally over all N^2 pairs."""
+    Tn = T / np.linalg.norm(T, axis=1, keepdims=True)
+    N = Tn.shape[0]
+    total = 0.0
+    for i0 in range(0, N, rows_per_block):
+        total += float((Tn[i0:i0 + rows_per_block] @ Tn.T).sum())
+    return total / (N * N)
+
+
+def apc_density_tokens(T: np.ndarray, alpha: float = ALPHA, gamma: float = GAMMA,
+                       tail_frac: float = TAIL_FRAC) -> Dict[str, object]:
+    """Eq. 1-6 on preview tokens T [N, D] (any N >= 1, any D)."""
+    N = T.shape[0]
+    Tn = T / np.linalg.norm(T, axis=1, keepdims=True)          # l2-normalised tokens
+    phi = global_redundancy(T)                                  # Eq. 1
+    rho_g = 1.0 - phi                                           # Eq. 2
+    c = Tn.mean(axis=0)                                         # Eq. 3
+    c_hat = c / np.linalg.norm(c)
+    d = np.linalg.norm(Tn - c_hat[None, :], axis=1)             # Eq. 4
+    k_tail = max(1, int(math.floor(tail_frac * N + 0.5)))       # reading R2
+    d_top = float(np.sort(d)[::-1][:k_tail].mean())
+    rho_d = min(d_top / gamma, 1.0)                             # Eq. 5
+    rho = alpha * rho_g + (1.0 - alpha) * rho_d                 # Eq. 6
+    return dict(N=N, phi=phi, rho_g=rho_g, c=c, c_hat=c_hat, d=d, k_tail=k_tail,
+                d_top=d_top, rho_d=rho_d, rho=rho)
+
+
+def retention_ratio(rho: float, r_min: float = 0.0, r_max: float = 1.0) -> float:
+    """Sec. 3.2 'Adaptive Condensation': r = rho, capped by the budget's maximum ratio (R3)."""
+    return min(max(rho, r_min), r_max)
+
+
+def target_size(H: int, W: int, r: float):
+    """App. B.3: width and height scaled by sqrt(r), snapped to 28 px (reading R4)."""
+    s = math.sqrt(max(r, 0.0))
+
+    def side(n):
+        return min(n, max(MERGE_UNIT, MERGE_UNIT * int(math.floor(n * s / MERGE_UNIT + 0.5))))
+    return side(H), side(W)
+
+
+def apc_density(img: np.ndarray, alpha: float = ALPHA, gamma: float = GAMMA,
+                tail_frac: float = TAIL_FRAC, r_min: float = 0.0, r_max: float = 1.0):
+    """Full APC decision for one image: density statistics, r and the target size."""
+    st = apc_density_tokens(patch_tokens(img), alpha, gamma, tail_frac)
+    st["r"] = retention_ratio(st["rho"], r_min, r_max)
+    st["H_out"], st["W_out"] = target_size(img.shape[0], img.shape[1], st["r"])
+    return st
+
+
+def cubic(t: np.ndarray, a: float = -0.5) -> np.ndarray:
+    """Keys' cubic convolution kernel with a = -0.5 (the bicubic of App. B.3)."""
+    t = np.abs(t)
+    w = np.zeros_like(t)
+    m1 = t < 1.0
+    m2 = (t >= 1.0) & (t < 2.0)
+    w[m1] = ((a + 2.0) * t[m1] - (a + 3.0)) * t[m1] ** 2 + 1.0
+    w[m2] = ((a * t[m2] - 5.0 * a) * t[m2] + 8.0 * a) * t[m2] - 4.0 * a
+    return w
+
+
+def resample_matrix(n_in: int, n_out: int) -> np.ndarray:
+    """Reading R5: dense [n_out, n_in] matrix of the 1-D antialiased cubic resample."""
+    scale = n_in / n_out
+    fs = max(scale, 1.0)
+    centre = (np.arange(n_out, dtype=np.float64) + 0.5) * scale
+    x = np.arange(n_in, dtype=np.float64) + 0.5
+    Wm = cubic((x[None, :] - centre[:, None]) / fs)
+    return Wm / Wm.sum(axis=1, keepdims=True)
+
+
+def resample_float(img: np.ndarray, H_out: int, W_out: int) -> np.ndarray:
+    """Separable resample of a uint8 HxWx3 image to H_out x W_out, fp64, before rounding."""
+    H, W, C = img.shape
+    Wy = resample_matrix(H, H_out)
+    Wx = resample_matrix(W, W_out)
+    x = img.astype(np.float64)
+    return np.stack([Wy @ x[:, :, ch] @ Wx.T for ch in range(C)], axis=2)
+
+
+def apc_resample(img: np.ndarray, H_out: int, W_out: int) -> np.ndarray:
+    """App. B.3 bicubic resize to the target size; uint8 out, round half to even."""
+    return np.clip(np.rint(resample_float(img, H_out, W_out)), 0, 255).astype(np.uint8)
+
+
+# ==============================================================================================
+# Extract: Dynamic Dual-Attention Extractor (Sec. 3.3)
+# ==============================================================================================
+def received_attention(q: np.ndarray, k: np.ndarray, scale: float, rows_per_block: int = 512) -> np.ndarray:
+    """Column sums of the row-softmax attention matrix of one head.
+
+    q [Nq, d], k [Nk, d] -> a [Nk], a_j = sum_i softmax_j(scale * q_i . k_j).
+    Rows are independent, so they are taken a block at a time.
+    """
+    a = np.zeros(k.shape[0])
+    for i0 in range(0, q.shape[0], rows_per_block):
+        s = (q[i0:i0 + rows_per_block] @ k.T) * scale
+        s -= s.max(axis=1, keepdims=True)
+        p = np.exp(s)
+        p /= p.sum(axis=1, keepdims=True)
+        a += p.sum(axis=0)
+    return a
+
+
+def vit_attn_importance(Q: np.ndarray, K: np.ndarray, cu_seqlens: Sequence[int], scale: float,
+                        merge: int = 4) -> np.ndarray:
+    """Reading R6 of S_vis (Sec. 3.3; App. B.3: the final ViT block).
+
+    Q, K float64 [sum N, H, d]; images are the row ranges of cu_seqlens.
+    Returns S_vis_raw [sum N / merge].
+    """
+    out: List[np.ndarray] = []
+    for b in range(len(cu_seqlens) - 1):
+        s0, s1 = int(cu_seqlens[b]), int(cu_seqlens[b + 1])
+        a = np.zeros(s1 - s0)
+        for h in range(Q.shape[1]):
+            a += received_attention(Q[s0:s1, h], K[s0:s1, h], scale)
+        out.append(a.reshape(-1, merge).sum(axis=1))
+    return np.concatenate(out) if out else np.zeros(0)
+
+
+def llm_text_visual_importance(Q: np.ndarray, K: np.ndarray, cu_q: Sequence[int], cu_k: Sequence[int],
+                               scale: float) -> np.ndarray:
+    """Reading R7 of S_llm (Sec. 3.3; App. B.3: layer L_ext = 2).
+
+    Q float64 [sum Tq, Hq, d], K float64 [sum Nv, Hkv, d].  Returns S_llm_raw [sum Nv].
+    """
+    Hq, Hkv = Q.shape[1], K.shape[1]
+    group = Hq // Hkv
+    out: List[np.ndarray] = []
+    for b in range(len(cu_q) - 1):
+        q0, q1 = int(cu_q[b]), int(cu_q[b + 1])
+        k0, k1 = int(cu_k[b]), int(cu_k[b + 1])
+        u = np.zeros(k1 - k0)
+        for h in range(Hq):
+            u += received_attention(Q[q0:q1, h], K[k0:k1, h // group], scale)
+        out.append(u)
+    return np.concatenate(out) if out else np.zeros(0)
+
+
+def min_max(x: np.ndarray) -> np.ndarray:
+    """Sec. 3.3: min-max normalisation to [0, 1]; a constant map becomes 0 (R8)."""
+    lo, hi = float(x.min()), float(x.max())
+    if hi == lo:
+        return np.zeros_like(x, dtype=np.float64)
+    return (x - lo) / (hi - lo)
+
+
+def ddae_fuse(s_llm_raw: np.ndarray, s_vis_raw: np.ndarray, tau: float = TAU) -> Dict[str, object]:
+    """Eq. 7 and S_final = alpha_w * S_llm + beta_w * S_vis for one image."""
+    S_llm = min_max(np.asarray(s_llm_raw, dtype=np.float64))
+    S_vis = min_max(np.asarray(s_vis_raw, dtype=np.float64))
+    sigma_llm = float(S_llm.std())      # population deviation (R8)
+    sigma_vis = float(S_vis.std())
+    z = np.array([sigma_llm, sigma_vis]) / tau
+    e = np.exp(z - z.max())
+    w = e / e.sum()
+    S_final = w[0] * S_llm + w[1] * S_vis
+    return dict(S_llm=S_llm, S_vis=S_vis, sigma_llm=sigma_llm, sigma_vis=sigma_vis,
+                alpha_w=float(w[0]), beta_w=float(w[1]), S_final=S_final)
+
+
+def budget(n_vis: int, frac: float) -> int:
+    """Reading R9: K = floor(frac * N_vis + 0.5) clamped to [0, N_vis]."""
+    return int(min(max(math.floor(frac * n_vis + 0.5), 0), n_vis))
+
+
+def top_k_ascending(S_final: np.ndarray, K: int) -> np.ndarray:
+    """Sec. 3.3: indices of the K highest S_final (ties: lower index), in ascending order."""
+    n = len(S_final)
+    order = np.lexsort((np.arange(n), -np.asarray(S_final, dtype=np.float64)))
+    return np.sort(order[:K]).astype(np.int64)
+
+
+def ddae_select(s_llm_raw: np.ndarray, s_vis_raw: np.ndarray, cu_v: Sequence[int],
+                keep: Sequence[int], tau: float = TAU) -> Dict[str, np.ndarray]:
+    """Per image: fuse, then keep the top K_b tokens.  Kept rows are global (cu_v-offset) indices."""
+    S_final, weights, kept = [], [], []
+    for b in range(len(cu_v) - 1):
+        v0, v1 = int(cu_v[b]), int(cu_v[b + 1])
+        f = ddae_fuse(s_llm_raw[v0:v1], s_vis_raw[v0:v1], tau)
+        S_final.append(f["S_final"])
+        weights.append([f["alpha_w"], f["beta_w"]])
+        kept.append(top_k_ascending(f["S_final"], int(keep[b])) + v0)
+    return dict(S_final=np.concatenate(S_final), weights=np.asarray(weights),
+                kept=np.concatenate(kept) if kept else np.zeros(0, dtype=np.int64))
+
+
+def gather_rows(E: np.ndarray, idx: np.ndarray) -> np.ndarray:
+    """Sec. 3.3: the kept visual rows form the pruned LLM context."""
+    return E[np.asarray(idx, dtype=np.int64)]
