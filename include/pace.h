@@ -1,0 +1,237 @@
+/*
+ * libpace — C ABI of the GB300 (sm_103a) condense-and-extract hot path of PACE
+ * (arxiv 2608.27206, "PACE: A Unified Condense-and-Extract Paradigm for Fast
+ * VLM Inference").
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every call returns a pace_status_t.  Arguments are checked on the host
+ *    before anything is launched; a rejected call launches nothing.
+ *  - "device" pointers are caller-owned device memory on the current CUDA
+ *    device; "host" arrays are read during the call only (they are copied into
+ *    kernel parameters), so they may be freed or reused as soon as it returns.
+ *  - Nothing is allocated or freed inside a call.  Scratch memory comes from the
+ *    caller as (ws, ws_bytes), sized by the matching *_workspace_size query;
+ *    a too-small workspace returns PACE_ERR_WORKSPACE.
+ *  - All work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream) and runs asynchronously.  Launch failures return PACE_ERR_CUDA
+ *    and the CUDA error code is kept for pace_last_cuda_error().
+ *  - Device-side waits are bounded.  A kernel whose wait runs out records
+ *    PACE_ERR_TIMEOUT in the device status word (pace_device_status) and
+ *    returns early; its outputs are then undefined.
+ *  - The library runs only on sm_103 devices (GB300); elsewhere every compute
+ *    call returns PACE_ERR_UNSUPPORTED_ARCH.  There is no CPU fallback.
+ *  - bf16 tensors are passed as `const void*` holding IEEE bfloat16 values.
+ */
+#ifndef PACE_H_
+#define PACE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define PACE_API __attribute__((visibility("default")))
+#else
+#define PACE_API
+#endif
+
+typedef struct CUstream_st* pace_stream_t; /* same type as cudaStream_t */
+
+typedef enum pace_status_t {
+  PACE_OK = 0,
+  PACE_ERR_INVALID_ARG = 1,      /* a size, pointer or parameter is out of range */
+  PACE_ERR_UNSUPPORTED_ARCH = 2, /* the current device is not an sm_103 GPU */
+  PACE_ERR_WORKSPACE = 3,        /* ws_bytes smaller than the size query returned */
+  PACE_ERR_CUDA = 4,             /* a CUDA runtime call or launch failed */
+  PACE_ERR_TIMEOUT = 5           /* a bounded device-side wait ran out (device status word) */
+} pace_status_t;
+
+/* Human-readable name of a status code (static string). */
+PACE_API const char* pace_status_string(pace_status_t status);
+
+/* CUDA error code (cudaError_t) of the last PACE_ERR_CUDA on the calling thread. */
+PACE_API int pace_last_cuda_error(void);
+
+/* Checks that `device` is an sm_103 GPU and prepares per-device state (device
+ * status word).  Optional: every entry point does the same check lazily. */
+PACE_API pace_status_t pace_init(int device);
+
+/* Reads the device status word of the current device (synchronises the device).
+ * *code = PACE_OK or PACE_ERR_TIMEOUT; *where = the kernel that recorded it
+ * (0 if none).  With clear != 0 the word is reset to PACE_OK afterwards. */
+PACE_API pace_status_t pace_device_status(int* code, int* where, int clear);
+
+/* ==============================================================================
+ * Condense — Adaptive Pixel Compressor (APC), Sec. 3.2, Eq. 1-6; App. B.3.
+ * ============================================================================== */
+
+typedef struct pace_apc_params {
+  float alpha;     /* weight of rho_g in rho = alpha rho_g + (1-alpha) rho_d (Eq. 6); 0.6 */
+  float gamma;     /* local contrast scale of rho_d = min(d_top / gamma, 1) (Eq. 5); 1.5  */
+  float tail_frac; /* fraction of tokens averaged into d_top; 0.10                         */
+  float r_min;     /* lower clamp of the retention ratio r; 0                             */
+  float r_max;     /* hard budget cap of r (Sec. 3.2, Adaptive Condensation); 1           */
+  int32_t align;   /* output sides are multiples of this (merge unit); 28                 */
+} pace_apc_params;
+
+/* Per-image result of pace_apc_density (written on the device). */
+typedef struct pace_apc_stats {
+  float phi;         /* mean pairwise cosine of the preview tokens (Eq. 1) */
+  float rho_g;       /* 1 - phi (Eq. 2) */
+  float d_top;       /* mean of the k_tail largest d_i */
+  float rho_d;       /* min(d_top / gamma, 1) (Eq. 5) */
+  float rho;         /* alpha rho_g + (1 - alpha) rho_d (Eq. 6) */
+  float r;           /* min(max(rho, r_min), r_max): retained area ratio */
+  int32_t n_patches; /* N = (H/14) (W/14) */
+  int32_t k_tail;    /* max(1, floor(tail_frac N + 0.5)) */
+  int32_t h_out;     /* min(H, max(align, align * floor(H sqrt(r) / align + 0.5))) */
+  int32_t w_out;     /* same for W */
+} pace_apc_stats;
+
+/* Fills the paper's defaults: alpha 0.6, gamma 1.5, tail 10 %, r in [0, 1], align 28. */
+PACE_API void pace_apc_params_default(pace_apc_params* params);
+
+/* Scratch bytes needed by pace_apc_density for these images (host arrays H, W). */
+PACE_API size_t pace_apc_density_workspace_size(int B, const int32_t* H, const int32_t* W);
+
+/*
+ * APC information density of B images (Sec. 3.2, Eq. 1-6, "per-region density on
+ * raw pixels").  The preview token of 14x14 patch i is the stand-in
+ * T_i = [x_i / 255 ; 1] (x_i = the patch's 588 bytes in row, column, channel
+ * order); t_i = T_i / |T_i|; c = mean t_i; phi = |c|^2 (equal to Eq. 1's double
+ * sum); c_hat = c / |c|; d_i = |t_i - c_hat| (Eq. 4).
+ *
+ *  img      device  uint8 HWC images; image b starts at byte img_off[b], 16-byte aligned
+ *  img_off  host    int64 [B]
+ *  H, W     host    int32 [B]; multiples of 14, >= 14
+ *  params   host    NULL for the defaults
+ *  d_out    device  float [sum N_b]: d_i of every patch, images in order, patches in
+ *                   raster order (may be NULL)
+ *  stats    device  pace_apc_stats [B]
+ *  ws       device  >= pace_apc_density_workspace_size(B, H, W) bytes, 16-byte aligned
+ */
+PACE_API pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img_off, const int32_t* H, const int32_t* W,
+                               int B, const pace_apc_params* params, float* d_out, pace_apc_stats* stats,
+                               void* ws, size_t ws_bytes, pace_stream_t stream);
+
+/*
+ * APC resize (Sec. 3.2 "Adaptive Condensation"; App. B.3: width and height scaled by
+ * sqrt(r), bicubic).  Separable cubic convolution (a = -0.5) with centre-aligned
+ * sampling, support widened by the downscale factor (antialias), the window clipped
+ * at the border and renormalised; fp32 weights, round half to even, clamp to [0,255].
+ * The target size (h_out, w_out) of image b is read from stats[b] on the device, so no
+ * host synchronisation is needed between density and resize.
+ *
+ *  src, src_off, H, W  as for pace_apc_density
+ *  stats    device  pace_apc_stats [B] from pace_apc_density (h_out <= H, w_out <= W)
+ *  dst      device  uint8; image b is written as h_out x w_out x 3 at byte dst_off[b];
+ *                   the caller reserves H*W*3 bytes there (the largest possible size)
+ *  dst_off  host    int64 [B]
+ */
+PACE_API pace_status_t pace_apc_resample(const uint8_t* src, const int64_t* src_off, const int32_t* H, const int32_t* W,
+                                const pace_apc_stats* stats, uint8_t* dst, const int64_t* dst_off, int B,
+                                pace_stream_t stream);
+
+/* Same resize to explicit host-given sizes H_out[b] x W_out[b] (1 <= H_out <= H, 1 <= W_out <= W). */
+PACE_API pace_status_t pace_apc_resample_to(const uint8_t* src, const int64_t* src_off, const int32_t* H, const int32_t* W,
+                                   const int32_t* H_out, const int32_t* W_out, uint8_t* dst,
+                                   const int64_t* dst_off, int B, pace_stream_t stream);
+
+/* ==============================================================================
+ * Extract — Dynamic Dual-Attention Extractor (DDAE), Sec. 3.3, Eq. 7; App. B.3.
+ * ============================================================================== */
+
+/* Scratch bytes for pace_vit_attn_importance (host cu_seqlens [B+1]). */
+PACE_API size_t pace_vit_attn_importance_workspace_size(int B, const int32_t* cu_seqlens, int n_heads);
+
+/*
+ * S_vis: attention each patch receives in a full-attention ViT layer (Sec. 3.3; App. B.3,
+ * final ViT block).  For image b (rows cu_seqlens[b] .. cu_seqlens[b+1]) and head h:
+ * a_j = sum_h sum_i softmax_j(scale q_ih . k_jh), softmax over all patches of the image,
+ * then s_vis_raw[m] = sum of a_j over the `merge` consecutive patches of merged token m.
+ * Computed flash-style in two passes (row log-sum-exp, then column sums of
+ * exp(s - lse)) on tcgen05 tensor cores; the N x N matrix is never stored.
+ *
+ *  Q, K        device  bf16 [total, n_heads, head_dim], row-major (head_dim contiguous)
+ *  cu_seqlens  host    int32 [B+1], cu_seqlens[0] = 0, nondecreasing; every image
+ *                      non-empty with a length and start divisible by `merge`
+ *  head_dim    64, 80 or 128;  merge 1, 2 or 4
+ *  s_vis_raw   device  float [total / merge]
+ *  ws          device  >= pace_vit_attn_importance_workspace_size(...) bytes, 16-B aligned
+ */
+PACE_API pace_status_t pace_vit_attn_importance(const void* Q, const void* K, const int32_t* cu_seqlens, int B,
+                                       int n_heads, int head_dim, float scale, int merge, float* s_vis_raw,
+                                       void* ws, size_t ws_bytes, pace_stream_t stream);
+
+/* Scratch bytes for pace_llm_text_visual_importance (host cu_q, cu_k [B+1]). */
+PACE_API size_t pace_llm_text_visual_importance_workspace_size(int B, const int32_t* cu_q, const int32_t* cu_k,
+                                                      int n_q_heads, int n_kv_heads);
+
+/*
+ * S_llm: attention from text query tokens to visual tokens in an LLM prefill layer with
+ * grouped-query attention (Sec. 3.3; App. B.3, layer L_ext = 2).  For image b, query head
+ * h and its KV head g = h / (n_q_heads / n_kv_heads):
+ * u_j = sum_h sum_t softmax_j(scale q_th . k_jg), softmax over the image's visual keys.
+ *
+ *  Q           device  bf16 [sum Tq, n_q_heads, head_dim]
+ *  K           device  bf16 [sum Nv, n_kv_heads, head_dim]
+ *  cu_q, cu_k  host    int32 [B+1] prefix sums of Tq_b >= 1 and Nv_b >= 1
+ *  n_q_heads % n_kv_heads == 0;  head_dim 64, 80 or 128
+ *  s_llm_raw   device  float [sum Nv]
+ */
+PACE_API pace_status_t pace_llm_text_visual_importance(const void* Q, const void* K, const int32_t* cu_q,
+                                              const int32_t* cu_k, int B, int n_q_heads, int n_kv_heads,
+                                              int head_dim, float scale, float* s_llm_raw, void* ws,
+                                              size_t ws_bytes, pace_stream_t stream);
+
+typedef struct pace_ddae_params {
+  float tau; /* temperature of Eq. 7; 0.5 */
+} pace_ddae_params;
+
+/* Fills the paper's default tau = 0.5. */
+PACE_API void pace_ddae_params_default(pace_ddae_params* params);
+
+/* Token budget K = floor(frac * n_vis + 0.5), clamped to [0, n_vis]. */
+PACE_API int32_t pace_budget(int32_t n_vis, double frac);
+
+/* Largest visual-token count per image accepted by pace_ddae_select. */
+#define PACE_DDAE_MAX_TOKENS 24576
+
+/*
+ * DDAE fusion and top-K (Sec. 3.3, Eq. 7).  Per image b: S_llm, S_vis = min-max
+ * normalised maps (a constant map becomes 0); sigma = population standard deviation;
+ * [alpha_w, beta_w] = softmax([sigma_llm, sigma_vis] / tau);
+ * S_final = alpha_w S_llm + beta_w S_vis; keep the K_b = cu_keep[b+1] - cu_keep[b]
+ * highest S_final (ties: lower index first), written in ascending index order.
+ *
+ *  s_llm_raw, s_vis_raw  device  float [sum Nv]
+ *  cu_v      host    int32 [B+1]; 1 <= Nv_b <= PACE_DDAE_MAX_TOKENS
+ *  cu_keep   host    int32 [B+1]; 0 <= K_b <= Nv_b
+ *  params    host    NULL for tau = 0.5
+ *  s_final   device  float [sum Nv] (may be NULL)
+ *  weights   device  float [B, 2] = (alpha_w, beta_w) (may be NULL)
+ *  kept      device  int32 [sum K]: global rows cu_v[b] + i of the kept tokens
+ */
+PACE_API pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s_vis_raw, const int32_t* cu_v,
+                               const int32_t* cu_keep, int B, const pace_ddae_params* params, float* s_final,
+                               float* weights, int32_t* kept, pace_stream_t stream);
+
+/*
+ * Gather of the kept rows, the pruned LLM context (Sec. 3.3; App. C): dst[r] = src[idx[r]],
+ * row_bytes bytes per row, byte-exact.  An index outside [0, n_src_rows) writes a zero row
+ * and records PACE_ERR_INVALID_ARG in the device status word.
+ *
+ *  src  device  [n_src_rows, row_bytes];  idx device int32 [n_idx];  dst device [n_idx, row_bytes]
+ */
+PACE_API pace_status_t pace_gather(const void* src, int64_t n_src_rows, int64_t row_bytes, const int32_t* idx,
+                          int64_t n_idx, void* dst, pace_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PACE_H_ */

@@ -1,0 +1,560 @@
+// Condense: Adaptive Pixel Compressor (Sec. 3.2, Eq. 1-6) and the bicubic resize (App. B.3).
+//
+// Density, three kernels on the caller's stream:
+//   apc_pass1  one CTA per strip of up to 32 patches of one patch row.  The strip's
+//              14 image rows are staged in shared memory with coalesced 2- or 4-byte
+//              loads; each warp reduces |x|^2 of its patches (exact integers) to the
+//              inverse token norm 1/|T_i|; the strip's weighted column sums
+//              sum_i x_ik / (255 |T_i|) (and sum_i 1/|T_i| for the constant coordinate)
+//              are added to a per-image 589-vector as 2^-32 fixed-point integers, so the
+//              reduction is exact and independent of the CTA order.
+//   apc_pass2  same strips: c = sums / N, phi = |c|^2, c_hat = c / |c| (recomputed per
+//              CTA from the 589 integers), then d_i = |t_i - c_hat| computed directly from
+//              the staged pixels (no 2 - 2cos cancellation).
+//   apc_tail   one CTA per image: radix select of the k_tail-th largest d_i (fp32 bits),
+//              tail mean, rho_d, rho, r and the target size.
+// Resize: apc_resample, one CTA per 8 x 32 output tile; input rows are filtered
+// horizontally 8 at a time into shared memory and accumulated vertically in registers.
+#include <cfloat>
+#include <cmath>
+
+#include "pace_common.cuh"
+
+namespace pace {
+namespace {
+
+constexpr int kPatch = 14;
+constexpr int kPatchBytes = kPatch * kPatch * 3;     // 588
+constexpr int kTokDim = kPatchBytes + 1;             // 589: pixels + constant coordinate
+constexpr int kStrip = 32;                           // patches per strip
+constexpr int kStripRowBytes = kStrip * kPatch * 3;  // 1344 bytes of one image row per strip
+constexpr int kApcThreads = 256;
+constexpr int kApcMaxB = 64;
+constexpr double kFix = 4294967296.0;                // 2^32 fixed-point scale
+
+struct ApcTable {
+  int64_t off[kApcMaxB];    // byte offset of image b
+  int H[kApcMaxB];
+  int W[kApcMaxB];
+  int gw[kApcMaxB];         // patches per row
+  int chunks[kApcMaxB];     // strips per patch row
+  int patch0[kApcMaxB];     // first global patch of image b
+  int ktail[kApcMaxB];
+  int unit_prefix[kApcMaxB + 1];
+  int nb;
+  int b_base;               // global index of image 0 of this table
+};
+
+__device__ __forceinline__ int find_image(const ApcTable& t, int unit) {
+  int b = 0;
+  while (b + 1 < t.nb && t.unit_prefix[b + 1] <= unit) ++b;
+  return b;
+}
+
+// Stages the 14 rows x (np * 42) bytes of one strip into s (row pitch kStripRowBytes).
+template <bool WIDE>
+__device__ __forceinline__ void load_strip(const uint8_t* __restrict__ img, int W, int py, int px0, int np,
+                                           uint8_t* s) {
+  const int seg = np * kPatch * 3;  // bytes per row (even; a multiple of 4 when WIDE)
+  const int64_t pitch = static_cast<int64_t>(W) * 3;
+  const uint8_t* base = img + static_cast<int64_t>(py) * kPatch * pitch + static_cast<int64_t>(px0) * kPatch * 3;
+  if (WIDE) {
+    const int words = seg >> 2;
+    for (int i = threadIdx.x; i < kPatch * words; i += kApcThreads) {
+      const int y = i / words, w = i - y * words;
+      const uint32_t v = __ldg(reinterpret_cast<const uint32_t*>(base + y * pitch) + w);
+      *reinterpret_cast<uint32_t*>(s + y * kStripRowBytes + 4 * w) = v;
+    }
+  } else {
+    const int halves = seg >> 1;
+    for (int i = threadIdx.x; i < kPatch * halves; i += kApcThreads) {
+      const int y = i / halves, w = i - y * halves;
+      const uint16_t v = __ldg(reinterpret_cast<const uint16_t*>(base + y * pitch) + w);
+      *reinterpret_cast<uint16_t*>(s + y * kStripRowBytes + 2 * w) = v;
+    }
+  }
+}
+
+__device__ __forceinline__ int warp_sum_int(int v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+template <bool WIDE>
+__global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restrict__ img,
+                                                         const __grid_constant__ ApcTable t,
+                                                         float* __restrict__ inv_norm,
+                                                         unsigned long long* __restrict__ sums) {
+  __shared__ __align__(16) uint8_t s[kPatch * kStripRowBytes];
+  __shared__ float inv[kStrip];
+  const int unit = blockIdx.x;
+  const int b = find_image(t, unit);
+  const int u = unit - t.unit_prefix[b];
+  const int py = u / t.chunks[b], cx = u - py * t.chunks[b];
+  const int px0 = cx * kStrip;
+  const int np = min(kStrip, t.gw[b] - px0);
+  load_strip<WIDE>(img + t.off[b], t.W[b], py, px0, np, s);
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int p = warp; p < np; p += kApcThreads / 32) {
+    int ss = 0;
+    for (int i = lane; i < kPatchBytes; i += 32) {
+      const int y = i / 42, k = i - y * 42;
+      const int v = s[y * kStripRowBytes + p * 42 + k];
+      ss += v * v;
+    }
+    ss = warp_sum_int(ss);
+    if (lane == 0) {
+      const float n2 = static_cast<float>(ss) * (1.0f / 65025.0f) + 1.0f;
+      const float iv = 1.0f / sqrtf(n2);
+      inv[p] = iv;
+      inv_norm[t.patch0[b] + py * t.gw[b] + px0 + p] = iv;
+    }
+  }
+  __syncthreads();
+  unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * kTokDim;
+  for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) {
+    float acc = 0.f;
+    if (k < kPatchBytes) {
+      const int y = k / 42, kk = k - y * 42;
+      const uint8_t* col = s + y * kStripRowBytes + kk;
+      for (int p = 0; p < np; ++p) acc = fmaf(inv[p], static_cast<float>(col[p * 42]), acc);
+      acc *= (1.0f / 255.0f);
+    } else {
+      for (int p = 0; p < np; ++p) acc += inv[p];
+    }
+    const unsigned long long q = static_cast<unsigned long long>(llrint(static_cast<double>(acc) * kFix));
+    atomicAdd(sb + k, q);
+  }
+}
+
+template <bool WIDE>
+__global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restrict__ img,
+                                                         const __grid_constant__ ApcTable t,
+                                                         const float* __restrict__ inv_norm,
+                                                         const unsigned long long* __restrict__ sums,
+                                                         float* __restrict__ d_out,
+                                                         pace_apc_stats* __restrict__ stats) {
+  __shared__ __align__(16) uint8_t s[kPatch * kStripRowBytes];
+  __shared__ float chat[kTokDim + 3];
+  __shared__ float red[kApcThreads / 32];
+  const int unit = blockIdx.x;
+  const int b = find_image(t, unit);
+  const int u = unit - t.unit_prefix[b];
+  const int py = u / t.chunks[b], cx = u - py * t.chunks[b];
+  const int px0 = cx * kStrip;
+  const int np = min(kStrip, t.gw[b] - px0);
+  const int N = (t.H[b] / kPatch) * t.gw[b];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  // c = sums / N, |c|^2 (fixed summation order)
+  const unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * kTokDim;
+  float part = 0.f;
+  for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) {
+    const float c = static_cast<float>(static_cast<double>(sb[k]) * (1.0 / kFix) / N);
+    chat[k] = c;
+    part = fmaf(c, c, part);
+  }
+  part = warp_sum_f(part);
+  if (lane == 0) red[warp] = part;
+  load_strip<WIDE>(img + t.off[b], t.W[b], py, px0, np, s);
+  __syncthreads();
+  float phi = 0.f;
+#pragma unroll
+  for (int w = 0; w < kApcThreads / 32; ++w) phi += red[w];
+  const float inv_c = 1.0f / sqrtf(phi);
+  for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) chat[k] *= inv_c;
+  if (u == 0 && threadIdx.x == 0) {
+    stats[t.b_base + b].phi = phi;
+    stats[t.b_base + b].rho_g = 1.0f - phi;
+    stats[t.b_base + b].n_patches = N;
+    stats[t.b_base + b].k_tail = t.ktail[b];
+  }
+  __syncthreads();
+  const float* pinv = inv_norm + t.patch0[b] + py * t.gw[b] + px0;
+  for (int p = warp; p < np; p += kApcThreads / 32) {
+    const float iv = pinv[p];
+    const float sc = iv * (1.0f / 255.0f);
+    float acc = 0.f;
+    for (int i = lane; i < kPatchBytes; i += 32) {
+      const int y = i / 42, k = i - y * 42;
+      const float v = fmaf(static_cast<float>(s[y * kStripRowBytes + p * 42 + k]), sc, -chat[i]);
+      acc = fmaf(v, v, acc);
+    }
+    acc = warp_sum_f(acc);
+    if (lane == 0) {
+      const float v = iv - chat[kPatchBytes];
+      d_out[t.patch0[b] + py * t.gw[b] + px0 + p] = sqrtf(fmaf(v, v, acc));
+    }
+  }
+}
+
+struct TailParams {
+  float alpha, gamma, r_min, r_max;
+  int align;
+};
+
+__global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTable t, const float* __restrict__ d,
+                                                 TailParams prm, pace_apc_stats* __restrict__ stats) {
+  __shared__ unsigned hist[256];
+  __shared__ unsigned sel[2];
+  __shared__ float red[32];
+  __shared__ unsigned cred[32];
+  const int b = blockIdx.x;
+  const int N = (t.H[b] / kPatch) * t.gw[b];
+  const float* db = d + t.patch0[b];
+  const unsigned k = static_cast<unsigned>(t.ktail[b]);
+  unsigned prefix = 0u, mask = 0u, remaining = k;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0u;
+    __syncthreads();
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+      const unsigned key = __float_as_uint(db[i]);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned above = 0u;
+      int dg = 255;
+      for (; dg > 0; --dg) {
+        if (above + hist[dg] >= remaining) break;
+        above += hist[dg];
+      }
+      sel[0] = static_cast<unsigned>(dg);
+      sel[1] = above;
+    }
+    __syncthreads();
+    prefix |= sel[0] << shift;
+    mask |= 255u << shift;
+    remaining -= sel[1];
+    __syncthreads();
+  }
+  const float T = __uint_as_float(prefix);   // k-th largest d
+  float s = 0.f;
+  unsigned cnt = 0u;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    const float v = db[i];
+    if (__float_as_uint(v) > prefix) {
+      s += v;
+      ++cnt;
+    }
+  }
+  s = warp_sum_f(s);
+  for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    red[warp] = s;
+    cred[warp] = cnt;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float tot = 0.f;
+    unsigned c = 0u;
+    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) {
+      tot += red[w];
+      c += cred[w];
+    }
+    tot += static_cast<float>(k - c) * T;  // the remaining entries all equal T
+    const float d_top = tot / static_cast<float>(k);
+    const float rho_g = stats[t.b_base + b].rho_g;
+    const float rho_d = fminf(d_top / prm.gamma, 1.0f);
+    const float rho = prm.alpha * rho_g + (1.0f - prm.alpha) * rho_d;
+    const float r = fminf(fmaxf(rho, prm.r_min), prm.r_max);
+    const float sr = sqrtf(fmaxf(r, 0.0f));
+    const int al = prm.align;
+    const int H = t.H[b], W = t.W[b];
+    int ho = al * static_cast<int>(floorf(static_cast<float>(H) * sr / al + 0.5f));
+    int wo = al * static_cast<int>(floorf(static_cast<float>(W) * sr / al + 0.5f));
+    ho = min(H, max(al, ho));
+    wo = min(W, max(al, wo));
+    pace_apc_stats& st = stats[t.b_base + b];
+    st.d_top = d_top;
+    st.rho_d = rho_d;
+    st.rho = rho;
+    st.r = r;
+    st.h_out = ho;
+    st.w_out = wo;
+  }
+}
+
+// ------------------------------------------------------------------------------------------------
+// resample
+// ------------------------------------------------------------------------------------------------
+constexpr int kRsTH = 8;    // output rows per CTA
+constexpr int kRsTW = 32;   // output columns per CTA
+constexpr int kRsChunk = 8; // input rows filtered per step
+
+struct ResampleTable {
+  int64_t src_off[kApcMaxB];
+  int64_t dst_off[kApcMaxB];
+  int H[kApcMaxB];
+  int W[kApcMaxB];
+  int Ho[kApcMaxB];  // used when stats == nullptr
+  int Wo[kApcMaxB];
+  int nb;
+  int b_base;
+};
+
+__device__ __forceinline__ float cubic_w(float t) {
+  // Keys' cubic convolution, a = -0.5
+  t = fabsf(t);
+  if (t < 1.0f) return (1.5f * t - 2.5f) * t * t + 1.0f;
+  if (t < 2.0f) return ((-0.5f * t + 2.5f) * t - 4.0f) * t + 2.0f;
+  return 0.0f;
+}
+
+// Window [lo, lo + n) of taps for output index o, the tap offset of lo, 1/fs, 1/sum(weights).
+__device__ __forceinline__ void window_1d(int o, int n_in, int n_out, int& lo, int& n, float& off0, float& ifs,
+                                          float& inorm) {
+  const double scale = static_cast<double>(n_in) / n_out;
+  const double fs = scale > 1.0 ? scale : 1.0;
+  const double support = 2.0 * fs;
+  const double centre = (o + 0.5) * scale;
+  int a = static_cast<int>(floor(centre - support));
+  int e = static_cast<int>(ceil(centre + support));
+  if (a < 0) a = 0;
+  if (e > n_in) e = n_in;
+  lo = a;
+  n = e - a;
+  off0 = static_cast<float>((a + 0.5 - centre) / fs);
+  ifs = static_cast<float>(1.0 / fs);
+  float s = 0.f;
+  for (int i = 0; i < n; ++i) s += cubic_w(fmaf(static_cast<float>(i), ifs, off0));
+  inorm = 1.0f / s;
+}
+
+__global__ void __launch_bounds__(256) apc_resample(const uint8_t* __restrict__ src,
+                                                    const __grid_constant__ ResampleTable t,
+                                                    const pace_apc_stats* __restrict__ stats,
+                                                    uint8_t* __restrict__ dst) {
+  __shared__ int xlo[kRsTW], xn[kRsTW];
+  __shared__ float xoff[kRsTW], xifs[kRsTW], xnorm[kRsTW];
+  __shared__ int ylo[kRsTH], yn[kRsTH];
+  __shared__ float yoff[kRsTH], yifs[kRsTH], ynorm[kRsTH];
+  __shared__ float hbuf[kRsChunk][kRsTW][3];
+  const int b = blockIdx.z;
+  const int H = t.H[b], W = t.W[b];
+  const int Ho = stats ? stats[t.b_base + b].h_out : t.Ho[b];
+  const int Wo = stats ? stats[t.b_base + b].w_out : t.Wo[b];
+  const int ox0 = blockIdx.x * kRsTW, oy0 = blockIdx.y * kRsTH;
+  if (ox0 >= Wo || oy0 >= Ho || Ho < 1 || Wo < 1 || Ho > H || Wo > W) return;
+  const int tid = threadIdx.x;
+  if (tid < kRsTW) {
+    const int ox = min(ox0 + tid, Wo - 1);
+    window_1d(ox, W, Wo, xlo[tid], xn[tid], xoff[tid], xifs[tid], xnorm[tid]);
+  } else if (tid >= 32 && tid < 32 + kRsTH) {
+    const int i = tid - 32;
+    const int oy = min(oy0 + i, Ho - 1);
+    window_1d(oy, H, Ho, ylo[i], yn[i], yoff[i], yifs[i], ynorm[i]);
+  }
+  __syncthreads();
+  const int nrows = min(kRsTH, Ho - oy0);
+  const int iy_lo = ylo[0];
+  const int iy_hi = ylo[nrows - 1] + yn[nrows - 1];  // exclusive
+  const uint8_t* img = src + t.src_off[b];
+  const int64_t pitch = static_cast<int64_t>(W) * 3;
+  // this thread's output pixel
+  const int my_r = tid / kRsTW, my_c = tid % kRsTW;
+  float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f;
+  for (int r0 = iy_lo; r0 < iy_hi; r0 += kRsChunk) {
+    // horizontal pass: kRsChunk rows x 32 columns x 3 channels
+    for (int v = tid; v < kRsChunk * kRsTW * 3; v += 256) {
+      const int rr = v / (kRsTW * 3), rem = v - rr * (kRsTW * 3);
+      const int cc = rem / 3, ch = rem - cc * 3;
+      const int iy = r0 + rr;
+      float h = 0.f;
+      if (iy < iy_hi) {
+        const uint8_t* row = img + iy * pitch + ch;
+        const int lo = xlo[cc], n = xn[cc];
+        const float off = xoff[cc], ifs = xifs[cc];
+        for (int i = 0; i < n; ++i) h = fmaf(cubic_w(fmaf(static_cast<float>(i), ifs, off)),
+                                             static_cast<float>(__ldg(row + 3 * (lo + i))), h);
+        h *= xnorm[cc];
+      }
+      hbuf[rr][cc][ch] = h;
+    }
+    __syncthreads();
+    if (my_r < nrows) {
+      const int lo = ylo[my_r], n = yn[my_r];
+      const float off = yoff[my_r], ifs = yifs[my_r];
+      for (int rr = 0; rr < kRsChunk; ++rr) {
+        const int i = r0 + rr - lo;
+        if (i >= 0 && i < n) {
+          const float w = cubic_w(fmaf(static_cast<float>(i), ifs, off));
+          acc0 = fmaf(w, hbuf[rr][my_c][0], acc0);
+          acc1 = fmaf(w, hbuf[rr][my_c][1], acc1);
+          acc2 = fmaf(w, hbuf[rr][my_c][2], acc2);
+        }
+      }
+    }
+    __syncthreads();
+  }
+  const int oy = oy0 + my_r, ox = ox0 + my_c;
+  if (my_r < nrows && ox < Wo) {
+    const float nrm = ynorm[my_r];
+    uint8_t* o = dst + t.dst_off[b] + (static_cast<int64_t>(oy) * Wo + ox) * 3;
+    o[0] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc0 * nrm))));
+    o[1] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc1 * nrm))));
+    o[2] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc2 * nrm))));
+  }
+}
+
+// ------------------------------------------------------------------------------------------------
+// host side
+// ------------------------------------------------------------------------------------------------
+struct DensityLayout {
+  size_t sums_off, inv_off, d_off, total;
+  int64_t n_total;
+};
+
+DensityLayout density_layout(int B, const int32_t* H, const int32_t* W) {
+  DensityLayout L{};
+  int64_t n = 0;
+  for (int b = 0; b < B; ++b) n += static_cast<int64_t>(H[b] / kPatch) * (W[b] / kPatch);
+  L.n_total = n;
+  L.sums_off = 0;
+  L.inv_off = align_up(static_cast<size_t>(B) * kTokDim * sizeof(unsigned long long), 256);
+  L.d_off = L.inv_off + align_up(static_cast<size_t>(n) * sizeof(float), 256);
+  L.total = L.d_off + align_up(static_cast<size_t>(n) * sizeof(float), 256);
+  return L;
+}
+
+pace_status_t check_images(const uint8_t* img, const int64_t* off, const int32_t* H, const int32_t* W, int B) {
+  if (B < 0) return PACE_ERR_INVALID_ARG;
+  if (B == 0) return PACE_OK;
+  if (img == nullptr || off == nullptr || H == nullptr || W == nullptr) return PACE_ERR_INVALID_ARG;
+  for (int b = 0; b < B; ++b) {
+    if (H[b] < kPatch || W[b] < kPatch || H[b] % kPatch || W[b] % kPatch) return PACE_ERR_INVALID_ARG;
+    if (off[b] < 0 || (reinterpret_cast<uintptr_t>(img) + off[b]) % 16) return PACE_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(H[b]) * W[b] > (int64_t{1} << 30)) return PACE_ERR_INVALID_ARG;
+  }
+  return PACE_OK;
+}
+
+}  // namespace
+}  // namespace pace
+
+using namespace pace;
+
+extern "C" size_t pace_apc_density_workspace_size(int B, const int32_t* H, const int32_t* W) {
+  if (B <= 0 || H == nullptr || W == nullptr) return 0;
+  for (int b = 0; b < B; ++b)
+    if (H[b] < kPatch || W[b] < kPatch) return 0;
+  return density_layout(B, H, W).total;
+}
+
+extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img_off, const int32_t* H,
+                                          const int32_t* W, int B, const pace_apc_params* params, float* d_out,
+                                          pace_apc_stats* stats, void* ws, size_t ws_bytes,
+                                          pace_stream_t stream) {
+  PACE_CHECK(check_images(img, img_off, H, W, B));
+  if (B == 0) return PACE_OK;
+  if (stats == nullptr) return PACE_ERR_INVALID_ARG;
+  pace_apc_params p;
+  if (params) p = *params; else pace_apc_params_default(&p);
+  if (!(p.tail_frac > 0.f && p.tail_frac <= 1.f) || !(p.gamma > 0.f) || !(p.alpha >= 0.f && p.alpha <= 1.f) ||
+      !(p.r_min <= p.r_max) || p.align < 1)
+    return PACE_ERR_INVALID_ARG;
+  const DensityLayout L = density_layout(B, H, W);
+  if (ws == nullptr || ws_bytes < L.total || reinterpret_cast<uintptr_t>(ws) % 16) return PACE_ERR_WORKSPACE;
+  PACE_CHECK(check_device());
+  uint8_t* w8 = static_cast<uint8_t*>(ws);
+  auto* sums = reinterpret_cast<unsigned long long*>(w8 + L.sums_off);
+  auto* inv = reinterpret_cast<float*>(w8 + L.inv_off);
+  float* d = d_out ? d_out : reinterpret_cast<float*>(w8 + L.d_off);
+  PACE_CUDA(cudaMemsetAsync(sums, 0, static_cast<size_t>(B) * kTokDim * sizeof(unsigned long long), stream));
+  int patch0 = 0;
+  for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
+    const int nb = (B - c0) < kApcMaxB ? (B - c0) : kApcMaxB;
+    ApcTable t{};
+    t.nb = nb;
+    t.b_base = c0;
+    t.unit_prefix[0] = 0;
+    bool wide = true;
+    for (int i = 0; i < nb; ++i) {
+      const int b = c0 + i;
+      t.off[i] = img_off[b];
+      t.H[i] = H[b];
+      t.W[i] = W[b];
+      t.gw[i] = W[b] / kPatch;
+      t.chunks[i] = (t.gw[i] + kStrip - 1) / kStrip;
+      t.patch0[i] = patch0;
+      const int N = (H[b] / kPatch) * t.gw[i];
+      double kt = std::floor(static_cast<double>(p.tail_frac) * N + 0.5);
+      if (kt < 1) kt = 1;
+      if (kt > N) kt = N;
+      t.ktail[i] = static_cast<int>(kt);
+      patch0 += N;
+      t.unit_prefix[i + 1] = t.unit_prefix[i] + (H[b] / kPatch) * t.chunks[i];
+      if ((static_cast<int64_t>(W[b]) * 3) % 4 != 0 || (t.gw[i] % 2) != 0 || (img_off[b] % 4) != 0) wide = false;
+    }
+    const int units = t.unit_prefix[nb];
+    if (wide) apc_pass1<true><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums);
+    else apc_pass1<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums);
+    PACE_CHECK(check_launch());
+    if (wide) apc_pass2<true><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d, stats);
+    else apc_pass2<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d, stats);
+    PACE_CHECK(check_launch());
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
+    apc_tail<<<nb, 1024, 0, stream>>>(t, d, tp, stats);
+    PACE_CHECK(check_launch());
+  }
+  return PACE_OK;
+}
+
+static pace_status_t resample_impl(const uint8_t* src, const int64_t* src_off, const int32_t* H, const int32_t* W,
+                                   const int32_t* Ho, const int32_t* Wo, const pace_apc_stats* stats,
+                                   uint8_t* dst, const int64_t* dst_off, int B, pace_stream_t stream) {
+  PACE_CHECK(check_images(src, src_off, H, W, B));
+  if (B == 0) return PACE_OK;
+  if (dst == nullptr || dst_off == nullptr) return PACE_ERR_INVALID_ARG;
+  if (stats == nullptr) {
+    if (Ho == nullptr || Wo == nullptr) return PACE_ERR_INVALID_ARG;
+    for (int b = 0; b < B; ++b)
+      if (Ho[b] < 1 || Wo[b] < 1 || Ho[b] > H[b] || Wo[b] > W[b]) return PACE_ERR_INVALID_ARG;
+  }
+  for (int b = 0; b < B; ++b)
+    if (dst_off[b] < 0) return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(check_device());
+  for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
+    const int nb = (B - c0) < kApcMaxB ? (B - c0) : kApcMaxB;
+    ResampleTable t{};
+    t.nb = nb;
+    t.b_base = c0;
+    int hmax = 1, wmax = 1;
+    for (int i = 0; i < nb; ++i) {
+      const int b = c0 + i;
+      t.src_off[i] = src_off[b];
+      t.dst_off[i] = dst_off[b];
+      t.H[i] = H[b];
+      t.W[i] = W[b];
+      t.Ho[i] = stats ? H[b] : Ho[b];
+      t.Wo[i] = stats ? W[b] : Wo[b];
+      if (t.Ho[i] > hmax) hmax = t.Ho[i];
+      if (t.Wo[i] > wmax) wmax = t.Wo[i];
+    }
+    dim3 grid((wmax + kRsTW - 1) / kRsTW, (hmax + kRsTH - 1) / kRsTH, nb);
+    apc_resample<<<grid, 256, 0, stream>>>(src, t, stats, dst);
+    PACE_CHECK(check_launch());
+  }
+  return PACE_OK;
+}
+
+extern "C" pace_status_t pace_apc_resample(const uint8_t* src, const int64_t* src_off, const int32_t* H,
+                                           const int32_t* W, const pace_apc_stats* stats, uint8_t* dst,
+                                           const int64_t* dst_off, int B, pace_stream_t stream) {
+  if (B > 0 && stats == nullptr) return PACE_ERR_INVALID_ARG;
+  return resample_impl(src, src_off, H, W, nullptr, nullptr, stats, dst, dst_off, B, stream);
+}
+
+extern "C" pace_status_t pace_apc_resample_to(const uint8_t* src, const int64_t* src_off, const int32_t* H,
+                                              const int32_t* W, const int32_t* H_out, const int32_t* W_out,
+                                              uint8_t* dst, const int64_t* dst_off, int B, pace_stream_t stream) {
+  return resample_impl(src, src_off, H, W, H_out, W_out, nullptr, dst, dst_off, B, stream);
+}

@@ -1,0 +1,327 @@
+// DDAE fusion + top-K selection (Sec. 3.3, Eq. 7) and the gather of kept rows.
+//
+// pace_ddae_select: one CTA of 1024 threads per image.  Both raw maps are staged in
+// shared memory; min/max, mean and the population variance are block reductions in a
+// fixed order (bit-stable run to run); the K-th largest S_final is found by an MSB-first
+// 8-bit radix select on the fp32 bit patterns (S_final >= 0, so integer order equals
+// float order), and the kept set is compacted in ascending index order with warp
+// ballots, the lower index winning among equal scores.
+//
+// pace_gather: one warp per kept row, 16-byte vector loads and stores.
+#include <cfloat>
+#include <cmath>
+
+#include "pace_common.cuh"
+
+namespace pace {
+namespace {
+
+constexpr int kSelThreads = 1024;
+constexpr int kSelMaxB = 256;
+
+struct SelectTable {
+  int v0[kSelMaxB];  // first global row of image b
+  int nv[kSelMaxB];  // visual tokens of image b
+  int k0[kSelMaxB];  // first output slot of image b
+  int nk[kSelMaxB];  // tokens kept for image b
+};
+
+__device__ __forceinline__ float warp_min(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Block-wide reduction of two values; every thread gets the result.  `red` holds 2*32 floats.
+template <int OP>  // 0 = sum, 1 = min, 2 = max
+__device__ __forceinline__ float2 block_reduce2(float a, float b, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (OP == 0) { a = warp_sum(a); b = warp_sum(b); }
+  if (OP == 1) { a = warp_min(a); b = warp_min(b); }
+  if (OP == 2) { a = warp_max(a); b = warp_max(b); }
+  __syncthreads();
+  if (lane == 0) { red[warp] = a; red[32 + warp] = b; }
+  __syncthreads();
+  if (warp == 0) {
+    a = red[lane];
+    b = red[32 + lane];
+    if (OP == 0) { a = warp_sum(a); b = warp_sum(b); }
+    if (OP == 1) { a = warp_min(a); b = warp_min(b); }
+    if (OP == 2) { a = warp_max(a); b = warp_max(b); }
+    if (lane == 0) { red[0] = a; red[32] = b; }
+  }
+  __syncthreads();
+  return make_float2(red[0], red[32]);
+}
+
+// Exclusive prefix count of `flag` over the block in thread order; returns (prefix, total).
+__device__ __forceinline__ int2 block_scan_flag(bool flag, int* wsum) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const unsigned bal = __ballot_sync(0xffffffffu, flag);
+  const int in_warp = __popc(bal & ((1u << lane) - 1u));
+  __syncthreads();
+  if (lane == 0) wsum[warp] = __popc(bal);
+  __syncthreads();
+  if (warp == 0) {
+    int v = wsum[lane];
+    int incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    wsum[lane] = incl - v;       // exclusive prefix of warp totals
+    if (lane == 31) wsum[32] = incl;
+  }
+  __syncthreads();
+  return make_int2(wsum[warp] + in_warp, wsum[32]);
+}
+
+__global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* __restrict__ s_llm,
+                                                                  const float* __restrict__ s_vis,
+                                                                  const __grid_constant__ SelectTable tab,
+                                                                  float tau, float* __restrict__ s_final,
+                                                                  float* __restrict__ weights,
+                                                                  int32_t* __restrict__ kept, int b_base) {
+  extern __shared__ float sm[];
+  __shared__ float red[64];
+  __shared__ int wsum[33];
+  __shared__ unsigned hist[256];
+  __shared__ unsigned sel[2];
+  const int b = blockIdx.x;
+  const int nv = tab.nv[b], v0 = tab.v0[b];
+  float* A = sm;        // S_llm raw -> normalised -> S_final
+  float* V = sm + nv;   // S_vis raw -> normalised
+  const int tid = threadIdx.x;
+
+  // 1. stage both maps, min / max
+  float amin = FLT_MAX, amax = -FLT_MAX, vmin = FLT_MAX, vmax = -FLT_MAX;
+  for (int i = tid; i < nv; i += kSelThreads) {
+    const float a = s_llm[v0 + i], v = s_vis[v0 + i];
+    A[i] = a;
+    V[i] = v;
+    amin = fminf(amin, a); amax = fmaxf(amax, a);
+    vmin = fminf(vmin, v); vmax = fmaxf(vmax, v);
+  }
+  const float2 mn = block_reduce2<1>(amin, vmin, red);
+  const float2 mx = block_reduce2<2>(amax, vmax, red);
+  const float ar = mx.x - mn.x, vr = mx.y - mn.y;
+
+  // 2. min-max normalisation (a constant map becomes 0) and the means
+  float sa = 0.f, sv = 0.f;
+  for (int i = tid; i < nv; i += kSelThreads) {
+    const float a = ar > 0.f ? __fdiv_rn(A[i] - mn.x, ar) : 0.f;
+    const float v = vr > 0.f ? __fdiv_rn(V[i] - mn.y, vr) : 0.f;
+    A[i] = a;
+    V[i] = v;
+    sa += a;
+    sv += v;
+  }
+  const float2 sums = block_reduce2<0>(sa, sv, red);
+  const float ma = sums.x / nv, mv = sums.y / nv;
+  float qa = 0.f, qv = 0.f;
+  for (int i = tid; i < nv; i += kSelThreads) {
+    const float da = A[i] - ma, dv = V[i] - mv;
+    qa = fmaf(da, da, qa);
+    qv = fmaf(dv, dv, qv);
+  }
+  const float2 sq = block_reduce2<0>(qa, qv, red);
+  const float sig_a = sqrtf(sq.x / nv), sig_v = sqrtf(sq.y / nv);
+
+  // 3. Eq. 7: confidence-weighted softmax fusion
+  const float za = sig_a / tau, zv = sig_v / tau, zm = fmaxf(za, zv);
+  const float ea = expf(za - zm), ev = expf(zv - zm);
+  const float wa = ea / (ea + ev), wv = ev / (ea + ev);
+  if (tid == 0 && weights != nullptr) {
+    weights[2 * (b_base + b)] = wa;
+    weights[2 * (b_base + b) + 1] = wv;
+  }
+  for (int i = tid; i < nv; i += kSelThreads) {
+    const float f = fmaf(wa, A[i], wv * V[i]);
+    A[i] = f;
+    if (s_final != nullptr) s_final[v0 + i] = f;
+  }
+  __syncthreads();
+
+  // 4. top-K threshold by radix select on the fp32 bits
+  const int K = tab.nk[b], k0 = tab.k0[b];
+  if (K <= 0) return;
+  if (K >= nv) {
+    for (int i = tid; i < nv; i += kSelThreads) kept[k0 + i] = v0 + i;
+    return;
+  }
+  unsigned prefix = 0u, mask = 0u;
+  unsigned remaining = static_cast<unsigned>(K);
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
+    __syncthreads();
+    for (int i = tid; i < nv; i += kSelThreads) {
+      const unsigned key = __float_as_uint(A[i]);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      unsigned above = 0u;
+      int d = 255;
+      for (; d > 0; --d) {
+        if (above + hist[d] >= remaining) break;
+        above += hist[d];
+      }
+      sel[0] = static_cast<unsigned>(d);
+      sel[1] = above;
+    }
+    __syncthreads();
+    prefix |= sel[0] << shift;
+    mask |= 255u << shift;
+    remaining -= sel[1];
+    __syncthreads();
+  }
+  const unsigned T = prefix;  // bit pattern of the K-th largest S_final
+  // `remaining` = how many keys equal to T are kept (lowest indices first)
+
+  // 5. ascending compaction
+  int eq_before = 0, taken_before = 0;
+  for (int base = 0; base < nv; base += kSelThreads) {
+    const int i = base + tid;
+    const unsigned key = i < nv ? __float_as_uint(A[i]) : 0u;
+    const bool gt = i < nv && key > T;
+    const bool eq = i < nv && key == T;
+    const int2 er = block_scan_flag(eq, wsum);
+    const bool take = gt || (eq && static_cast<unsigned>(eq_before + er.x) < remaining);
+    const int2 tr = block_scan_flag(take, wsum);
+    if (take) kept[k0 + taken_before + tr.x] = v0 + i;
+    eq_before += er.y;
+    taken_before += tr.y;
+  }
+}
+
+// One warp per row; 16-byte vectors.
+__global__ void __launch_bounds__(256) gather_rows_v16(const uint4* __restrict__ src, int64_t n_src,
+                                                       int64_t row_vec, const int32_t* __restrict__ idx,
+                                                       int64_t n_idx, uint4* __restrict__ dst, int* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  constexpr int U = 8;
+  for (int64_t r = warp0; r < n_idx; r += nwarps) {
+    const int64_t s = idx[r];
+    uint4* dp = dst + r * row_vec;
+    if (s < 0 || s >= n_src) {
+      for (int64_t c = lane; c < row_vec; c += 32) dp[c] = make_uint4(0u, 0u, 0u, 0u);
+      if (lane == 0) record_error(status, PACE_ERR_INVALID_ARG, K_GATHER);
+      continue;
+    }
+    const uint4* sp = src + s * row_vec;
+    for (int64_t c0 = 0; c0 < row_vec; c0 += 32 * U) {
+      uint4 v[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int64_t c = c0 + u * 32 + lane;
+        if (c < row_vec) v[u] = __ldcs(sp + c);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int64_t c = c0 + u * 32 + lane;
+        if (c < row_vec) __stcs(dp + c, v[u]);
+      }
+    }
+  }
+}
+
+// Byte-granular fallback for rows that are not 16-byte multiples or not 16-byte aligned.
+__global__ void __launch_bounds__(256) gather_rows_bytes(const uint8_t* __restrict__ src, int64_t n_src,
+                                                         int64_t row_bytes, const int32_t* __restrict__ idx,
+                                                         int64_t n_idx, uint8_t* __restrict__ dst, int* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  for (int64_t r = warp0; r < n_idx; r += nwarps) {
+    const int64_t s = idx[r];
+    uint8_t* dp = dst + r * row_bytes;
+    if (s < 0 || s >= n_src) {
+      for (int64_t c = lane; c < row_bytes; c += 32) dp[c] = 0;
+      if (lane == 0) record_error(status, PACE_ERR_INVALID_ARG, K_GATHER);
+      continue;
+    }
+    const uint8_t* sp = src + s * row_bytes;
+    for (int64_t c = lane; c < row_bytes; c += 32) dp[c] = sp[c];
+  }
+}
+
+}  // namespace
+}  // namespace pace
+
+using namespace pace;
+
+extern "C" pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s_vis_raw, const int32_t* cu_v,
+                                          const int32_t* cu_keep, int B, const pace_ddae_params* params,
+                                          float* s_final, float* weights, int32_t* kept, pace_stream_t stream) {
+  if (B < 0 || (B > 0 && (cu_v == nullptr || cu_keep == nullptr))) return PACE_ERR_INVALID_ARG;
+  if (B == 0) return PACE_OK;
+  if (s_llm_raw == nullptr || s_vis_raw == nullptr) return PACE_ERR_INVALID_ARG;
+  if (cu_v[0] != 0 || cu_keep[0] != 0) return PACE_ERR_INVALID_ARG;
+  int max_nv = 0;
+  for (int b = 0; b < B; ++b) {
+    const int nv = cu_v[b + 1] - cu_v[b], nk = cu_keep[b + 1] - cu_keep[b];
+    if (nv < 1 || nv > PACE_DDAE_MAX_TOKENS || nk < 0 || nk > nv) return PACE_ERR_INVALID_ARG;
+    if (nv > max_nv) max_nv = nv;
+  }
+  if (cu_keep[B] > 0 && kept == nullptr) return PACE_ERR_INVALID_ARG;
+  const float tau = params ? params->tau : 0.5f;
+  if (!(tau > 0.f) || !std::isfinite(tau)) return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(check_device());
+  const size_t smem = static_cast<size_t>(2 * max_nv) * sizeof(float);
+  PACE_CUDA(cudaFuncSetAttribute(ddae_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(smem)));
+  for (int c0 = 0; c0 < B; c0 += kSelMaxB) {
+    const int nb = (B - c0) < kSelMaxB ? (B - c0) : kSelMaxB;
+    SelectTable t;
+    for (int i = 0; i < nb; ++i) {
+      const int b = c0 + i;
+      t.v0[i] = cu_v[b];
+      t.nv[i] = cu_v[b + 1] - cu_v[b];
+      t.k0[i] = cu_keep[b];
+      t.nk[i] = cu_keep[b + 1] - cu_keep[b];
+    }
+    ddae_select_kernel<<<nb, kSelThreads, smem, stream>>>(s_llm_raw, s_vis_raw, t, tau, s_final, weights, kept,
+                                                           c0);
+    PACE_CHECK(check_launch());
+  }
+  return PACE_OK;
+}
+
+extern "C" pace_status_t pace_gather(const void* src, int64_t n_src_rows, int64_t row_bytes, const int32_t* idx,
+                                     int64_t n_idx, void* dst, pace_stream_t stream) {
+  if (n_idx < 0 || row_bytes <= 0 || n_src_rows < 0) return PACE_ERR_INVALID_ARG;
+  if (n_idx == 0) return PACE_OK;
+  if (src == nullptr || idx == nullptr || dst == nullptr) return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(check_device());
+  int* status = device_status_word();
+  int sms = 152;
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t warps_per_block = 8;
+  int64_t blocks = (n_idx + warps_per_block - 1) / warps_per_block;
+  const int64_t cap = static_cast<int64_t>(sms) * 16;
+  if (blocks > cap) blocks = cap;
+  const bool vec = (row_bytes % 16 == 0) && (reinterpret_cast<uintptr_t>(src) % 16 == 0) &&
+                   (reinterpret_cast<uintptr_t>(dst) % 16 == 0);
+  if (vec) {
+    gather_rows_v16<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
+        static_cast<const uint4*>(src), n_src_rows, row_bytes / 16, idx, n_idx, static_cast<uint4*>(dst), status);
+  } else {
+    gather_rows_bytes<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
+        static_cast<const uint8_t*>(src), n_src_rows, row_bytes, idx, n_idx, static_cast<uint8_t*>(dst), status);
+  }
+  return check_launch();
+}

@@ -1,0 +1,129 @@
+// libpace host API: status strings, per-device initialisation (sm_103 check and
+// device status word), budget helper and parameter defaults.
+#include <cmath>
+#include <mutex>
+
+#include "pace_common.cuh"
+
+namespace pace {
+
+namespace {
+constexpr int kMaxDevices = 64;
+thread_local int t_last_cuda_error = 0;
+std::mutex g_mutex;
+bool g_checked[kMaxDevices] = {};
+bool g_ok[kMaxDevices] = {};
+int* g_status[kMaxDevices] = {};
+
+// Status word of every device that loads the library: [code, kernel id].
+__device__ int g_status_word[2];
+}  // namespace
+
+pace_status_t set_cuda_error(cudaError_t e) {
+  t_last_cuda_error = static_cast<int>(e);
+  return PACE_ERR_CUDA;
+}
+
+static pace_status_t init_device_locked(int dev) {
+  if (dev < 0 || dev >= kMaxDevices) return PACE_ERR_INVALID_ARG;
+  if (g_checked[dev]) return g_ok[dev] ? PACE_OK : PACE_ERR_UNSUPPORTED_ARCH;
+  int major = 0, minor = 0;
+  PACE_CUDA(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev));
+  PACE_CUDA(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev));
+  g_checked[dev] = true;
+  g_ok[dev] = (major == 10 && minor == 3);
+  if (!g_ok[dev]) return PACE_ERR_UNSUPPORTED_ARCH;
+  int prev = -1;
+  PACE_CUDA(cudaGetDevice(&prev));
+  if (prev != dev) PACE_CUDA(cudaSetDevice(dev));
+  void* p = nullptr;
+  cudaError_t e = cudaGetSymbolAddress(&p, g_status_word);
+  if (e == cudaSuccess) e = cudaMemset(p, 0, 2 * sizeof(int));
+  if (prev != dev) cudaSetDevice(prev);
+  if (e != cudaSuccess) {
+    g_checked[dev] = false;
+    return set_cuda_error(e);
+  }
+  g_status[dev] = static_cast<int*>(p);
+  return PACE_OK;
+}
+
+pace_status_t check_device() {
+  int dev = -1;
+  PACE_CUDA(cudaGetDevice(&dev));
+  if (dev >= 0 && dev < kMaxDevices && g_checked[dev]) return g_ok[dev] ? PACE_OK : PACE_ERR_UNSUPPORTED_ARCH;
+  std::lock_guard<std::mutex> lk(g_mutex);
+  return init_device_locked(dev);
+}
+
+int* device_status_word() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  return g_status[dev];
+}
+
+pace_status_t check_launch() {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return set_cuda_error(e);
+  return PACE_OK;
+}
+
+}  // namespace pace
+
+extern "C" {
+
+const char* pace_status_string(pace_status_t s) {
+  switch (s) {
+    case PACE_OK: return "PACE_OK";
+    case PACE_ERR_INVALID_ARG: return "PACE_ERR_INVALID_ARG";
+    case PACE_ERR_UNSUPPORTED_ARCH: return "PACE_ERR_UNSUPPORTED_ARCH";
+    case PACE_ERR_WORKSPACE: return "PACE_ERR_WORKSPACE";
+    case PACE_ERR_CUDA: return "PACE_ERR_CUDA";
+    case PACE_ERR_TIMEOUT: return "PACE_ERR_TIMEOUT";
+  }
+  return "PACE_ERR_UNKNOWN";
+}
+
+int pace_last_cuda_error(void) { return pace::t_last_cuda_error; }
+
+pace_status_t pace_init(int device) {
+  std::lock_guard<std::mutex> lk(pace::g_mutex);
+  return pace::init_device_locked(device);
+}
+
+pace_status_t pace_device_status(int* code, int* where, int clear) {
+  PACE_CHECK(pace::check_device());
+  int* w = pace::device_status_word();
+  if (w == nullptr) return PACE_ERR_INVALID_ARG;
+  int h[2] = {0, 0};
+  PACE_CUDA(cudaDeviceSynchronize());
+  PACE_CUDA(cudaMemcpy(h, w, sizeof(h), cudaMemcpyDeviceToHost));
+  if (code) *code = h[0];
+  if (where) *where = h[1];
+  if (clear) PACE_CUDA(cudaMemset(w, 0, sizeof(h)));
+  return PACE_OK;
+}
+
+int32_t pace_budget(int32_t n_vis, double frac) {
+  if (n_vis <= 0 || !(frac > 0.0)) return 0;
+  double k = std::floor(frac * static_cast<double>(n_vis) + 0.5);
+  if (k > n_vis) k = n_vis;
+  return static_cast<int32_t>(k);
+}
+
+void pace_apc_params_default(pace_apc_params* p) {
+  if (!p) return;
+  p->alpha = 0.6f;
+  p->gamma = 1.5f;
+  p->tail_frac = 0.10f;
+  p->r_min = 0.0f;
+  p->r_max = 1.0f;
+  p->align = 28;
+}
+
+void pace_ddae_params_default(pace_ddae_params* p) {
+  if (!p) return;
+  p->tau = 0.5f;
+}
+
+}  // extern "C"

@@ -1,0 +1,328 @@
+"""GPU parity of every libpace entry point against the fp64 oracle on small seeded inputs.
+
+Sizes span several 128-row tiles with ragged tails, multi-image batches, and the
+degenerate cases (one patch, one token, K = 0 or N, constant maps, ties).
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import pace_oracle as O
+from paper_2608_27206_gb300 import synth
+from tests.helpers import assert_kept_matches, assert_scores_close, bf16_tensor, f64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def pace():
+    from paper_2608_27206_gb300 import build
+    build.build()
+    from paper_2608_27206_gb300 import pace as P
+    P.pace_init(0)
+    P.pace_device_status(clear=True)
+    return P
+
+
+def _no_device_error(P):
+    code, where = P.pace_device_status(clear=True)
+    assert code == 0, (code, where)
+
+
+# ----------------------------------------------------------------------------------------------
+# gather
+# ----------------------------------------------------------------------------------------------
+@pytest.mark.parametrize("n_rows,row_elems,n_idx", [(300, 3584, 50), (1, 3584, 3), (97, 8, 200), (64, 5, 7)])
+def test_gather_bit_exact(pace, n_rows, row_elems, n_idx):
+    rng = np.random.default_rng(n_rows + n_idx)
+    E = rng.integers(-32768, 32767, size=(n_rows, row_elems), dtype=np.int16)
+    idx = rng.integers(0, n_rows, size=n_idx).astype(np.int32)
+    out = pace.pace_gather(torch.from_numpy(E).cuda(), torch.from_numpy(idx).cuda()).cpu().numpy()
+    np.testing.assert_array_equal(out, O.gather_rows(E, idx))
+    _no_device_error(pace)
+
+
+def test_gather_empty_and_bad_index(pace):
+    E = torch.arange(64 * 16, dtype=torch.int16, device="cuda").view(64, 16)
+    assert pace.pace_gather(E, torch.zeros(0, dtype=torch.int32, device="cuda")).numel() == 0
+    idx = torch.tensor([3, 64, -1, 5], dtype=torch.int32, device="cuda")   # two out of range
+    out = pace.pace_gather(E, idx).cpu().numpy()
+    ref = E.cpu().numpy()
+    np.testing.assert_array_equal(out[0], ref[3])
+    np.testing.assert_array_equal(out[3], ref[5])
+    assert not out[1].any() and not out[2].any()
+    code, where = pace.pace_device_status(clear=True)
+    assert code == pace.PACE_ERR_INVALID_ARG and where == 10
+
+
+# ----------------------------------------------------------------------------------------------
+# APC density + resample
+# ----------------------------------------------------------------------------------------------
+def _density(pace, images, params=None, **kw):
+    buf, off = synth.pack_images(images)
+    H = [im.shape[0] for im in images]
+    W = [im.shape[1] for im in images]
+    d, st = pace.pace_apc_density(torch.from_numpy(buf).cuda(), off, H, W, params=params)
+    return d.cpu().numpy(), pace.stats_dict(st)
+
+
+def _check_density(d, st, images, alpha=0.6, gamma=1.5, tail=0.1, r_min=0.0, r_max=1.0):
+    p0 = 0
+    for im, s in zip(images, st):
+        ref = O.apc_density(im, alpha, gamma, tail, r_min, r_max)
+        n = ref["N"]
+        assert s["n_patches"] == n and s["k_tail"] == ref["k_tail"]
+        # d_i are distances between unit vectors (O(1)); 1e-5 absolute covers fp32 rounding
+        # where the exact distance is 0 (identical tokens)
+        assert_scores_close(d[p0:p0 + n], ref["d"], atol_frac=2e-3, atol=1e-5, what="d_i")
+        for k in ("phi", "d_top", "rho_d", "r"):
+            assert abs(s[k] - ref[k]) <= 2e-3 * max(abs(ref[k]), 1e-3), (k, s[k], ref[k])
+        assert abs(s["rho_g"] - ref["rho_g"]) <= 2e-3 * max(abs(ref["rho_g"]), 1e-3) + 2e-6
+        assert abs(s["rho"] - ref["rho"]) <= 2e-3 * max(abs(ref["rho"]), 1e-3) + 2e-6
+        # target size: an integer decided in floating point; equal unless the oracle's value
+        # sits within the score tolerance of a rounding boundary
+        for side, key in ((im.shape[0], "h_out"), (im.shape[1], "w_out")):
+            x = side * math.sqrt(max(ref["r"], 0.0)) / 28 + 0.5
+            near = abs(x - round(x)) < 2e-3 * x
+            exp = ref["H_out"] if key == "h_out" else ref["W_out"]
+            assert s[key] == exp or (near and abs(s[key] - exp) == 28), (key, s[key], exp)
+        p0 += n
+
+
+@pytest.mark.parametrize("shape,tiles,hf", [((28, 28), (1, 1), 1.0), ((14, 14), (1, 1), 1.0),
+                                             ((112, 154), (2, 2), 0.5), ((448, 448), (4, 4), 0.5),
+                                             ((70, 462), (3, 1), 0.3), ((322, 98), (2, 5), 0.6)])
+def test_density_single(pace, shape, tiles, hf):
+    rng = np.random.default_rng(shape[0] * 7 + shape[1])
+    img = synth.make_image(rng, shape[0], shape[1], tiles[0], tiles[1], hf)
+    d, st = _density(pace, [img])
+    _check_density(d, st, [img])
+    _no_device_error(pace)
+
+
+def test_density_batch_and_params(pace):
+    rng = np.random.default_rng(3)
+    imgs = [synth.make_image(rng, h, w, 3, 2, f) for h, w, f in
+            [(224, 448, 0.2), (56, 56, 0.9), (616, 532, 0.4), (1008, 28, 0.1), (42, 70, 0.5)]]
+    d, st = _density(pace, imgs)
+    _check_density(d, st, imgs)
+    p = pace.apc_params(alpha=0.3, gamma=0.8, tail_frac=0.05, r_min=0.1, r_max=0.4)
+    d, st = _density(pace, imgs, params=p)
+    _check_density(d, st, imgs, alpha=0.3, gamma=0.8, tail=0.05, r_min=0.1, r_max=0.4)
+    _no_device_error(pace)
+
+
+def test_density_constant_images(pace):
+    imgs = [np.full((112, 168, 3), v, dtype=np.uint8) for v in (0, 77, 255)]
+    d, st = _density(pace, imgs)
+    assert np.abs(d).max() < 2e-3
+    for s in st:
+        assert abs(s["phi"] - 1.0) < 1e-5 and abs(s["rho"]) < 2e-3
+        assert (s["h_out"], s["w_out"]) == (28, 28)
+
+
+def test_density_rejects_bad_sizes(pace):
+    img = np.zeros((30, 28, 3), dtype=np.uint8)
+    with pytest.raises(pace.PaceError) as e:
+        _density(pace, [img])
+    assert e.value.status == pace.PACE_ERR_INVALID_ARG
+
+
+def _resample_gpu(pace, images, sizes):
+    buf, off = synth.pack_images(images)
+    H = [im.shape[0] for im in images]
+    W = [im.shape[1] for im in images]
+    dst_off = np.concatenate([[0], np.cumsum([h * w * 3 for h, w in zip(H, W)])])[:-1]
+    dst = torch.zeros(int(sum(h * w * 3 for h, w in zip(H, W))), dtype=torch.uint8, device="cuda")
+    pace.pace_apc_resample_to(torch.from_numpy(buf).cuda(), off, H, W, [s[0] for s in sizes],
+                              [s[1] for s in sizes], dst, dst_off)
+    out = dst.cpu().numpy()
+    return [out[o:o + ho * wo * 3].reshape(ho, wo, 3) for o, (ho, wo) in zip(dst_off, sizes)]
+
+
+@pytest.mark.parametrize("shape,size", [((56, 84), (28, 28)), ((98, 70), (42, 56)), ((140, 140), (28, 70)),
+                                        ((84, 56), (37, 19)), ((448, 448), (308, 308)), ((56, 84), (56, 84)),
+                                        ((616, 1232), (28, 28)), ((2156, 392), (1092, 196))])
+def test_resample_within_one_lsb(pace, shape, size):
+    rng = np.random.default_rng(shape[0] + size[1])
+    img = synth.make_image(rng, shape[0], shape[1], 3, 3, 0.5)
+    out = _resample_gpu(pace, [img], [size])[0]
+    ref = O.apc_resample(img, *size)
+    diff = np.abs(out.astype(np.int32) - ref.astype(np.int32))
+    assert diff.max() <= 1, diff.max()
+    if size == shape:
+        np.testing.assert_array_equal(out, img)
+    _no_device_error(pace)
+
+
+def test_resample_constant_bit_exact_and_batch(pace):
+    imgs = [np.full((112, 168, 3), v, dtype=np.uint8) for v in (0, 201, 255)]
+    sizes = [(28, 28), (56, 84), (84, 112)]
+    for o, v in zip(_resample_gpu(pace, imgs, sizes), (0, 201, 255)):
+        assert np.all(o == v)
+    rng = np.random.default_rng(5)
+    imgs = [synth.make_image(rng, h, w, 2, 2, 0.5) for h, w in [(224, 448), (56, 56), (616, 532)]]
+    sizes = [(112, 308), (28, 28), (420, 364)]
+    for o, im, sz in zip(_resample_gpu(pace, imgs, sizes), imgs, sizes):
+        assert np.abs(o.astype(int) - O.apc_resample(im, *sz).astype(int)).max() <= 1
+
+
+def test_resample_from_device_stats(pace):
+    """pace_apc_resample reads (h_out, w_out) on the device; same pixels as the explicit call."""
+    rng = np.random.default_rng(6)
+    imgs = [synth.make_image(rng, h, w, 4, 4, f) for h, w, f in [(448, 448, 0.5), (280, 560, 0.1)]]
+    buf, off = synth.pack_images(imgs)
+    H, W = [448, 280], [448, 560]
+    src = torch.from_numpy(buf).cuda()
+    _, st = pace.pace_apc_density(src, off, H, W)
+    sd = pace.stats_dict(st)
+    dst_off = [0, 448 * 448 * 3]
+    dst = torch.zeros(448 * 448 * 3 + 280 * 560 * 3, dtype=torch.uint8, device="cuda")
+    pace.pace_apc_resample(src, off, H, W, st, dst, dst_off)
+    dst2 = torch.zeros_like(dst)
+    pace.pace_apc_resample_to(src, off, H, W, [s["h_out"] for s in sd], [s["w_out"] for s in sd], dst2, dst_off)
+    for b, s in enumerate(sd):
+        n = s["h_out"] * s["w_out"] * 3
+        assert torch.equal(dst[dst_off[b]:dst_off[b] + n], dst2[dst_off[b]:dst_off[b] + n])
+        ref = O.apc_density(imgs[b])
+        assert (s["h_out"], s["w_out"]) == (ref["H_out"], ref["W_out"])
+
+
+# ----------------------------------------------------------------------------------------------
+# attention importance
+# ----------------------------------------------------------------------------------------------
+def _vit_case(pace, lens, H=16, D=80, merge=4, seed=0, boost=None):
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    Qb = synth.random_small_qk(seed, int(cu[-1]), H, D)
+    Kb = synth.random_small_qk(seed + 1000, int(cu[-1]), H, D)
+    if boost is not None:        # a few rows with 4x norm (attention sinks)
+        Kb = synth.f32_to_bf16_bits(f64(Kb).astype(np.float32) * boost[:, None, None].astype(np.float32))
+    scale = 1.0 / math.sqrt(D)
+    out = pace.pace_vit_attn_importance(bf16_tensor(Qb), bf16_tensor(Kb), cu, scale, merge).cpu().numpy()
+    ref = O.vit_attn_importance(f64(Qb), f64(Kb), cu, scale, merge)
+    return out, ref, cu
+
+
+@pytest.mark.parametrize("lens", [[4], [64], [100], [128], [256], [300], [1024], [516, 4, 128, 388]])
+def test_vit_importance(pace, lens):
+    out, ref, cu = _vit_case(pace, lens)
+    assert_scores_close(out, ref, what="S_vis_raw")
+    for b in range(len(lens)):     # each image's map sums to N * heads
+        assert out[cu[b] // 4:cu[b + 1] // 4].sum() == pytest.approx(lens[b] * 16, rel=1e-4)
+    _no_device_error(pace)
+
+
+@pytest.mark.parametrize("D,H,merge", [(64, 4, 1), (128, 2, 2), (80, 3, 1)])
+def test_vit_importance_head_dims(pace, D, H, merge):
+    out, ref, _ = _vit_case(pace, [200, 36], H=H, D=D, merge=merge, seed=D)
+    assert_scores_close(out, ref, what=f"S_vis_raw D={D}")
+
+
+def test_vit_importance_sinks(pace):
+    n = 384
+    boost = np.ones(n)
+    boost[[5, 77, 300]] = 4.0
+    out, ref, _ = _vit_case(pace, [n], boost=boost, seed=11)
+    assert_scores_close(out, ref, what="S_vis_raw with sinks")
+
+
+def _llm_case(pace, tq, nv, Hq=28, Hkv=4, D=128, seed=0):
+    cq = np.concatenate([[0], np.cumsum(tq)]).astype(np.int32)
+    ck = np.concatenate([[0], np.cumsum(nv)]).astype(np.int32)
+    Qb = synth.random_small_qk(seed, int(cq[-1]), Hq, D)
+    Kb = synth.random_small_qk(seed + 1, int(ck[-1]), Hkv, D)
+    scale = 1.0 / math.sqrt(D)
+    out = pace.pace_llm_text_visual_importance(bf16_tensor(Qb), bf16_tensor(Kb), cq, ck, scale).cpu().numpy()
+    ref = O.llm_text_visual_importance(f64(Qb), f64(Kb), cq, ck, scale)
+    return out, ref, cq, ck
+
+
+@pytest.mark.parametrize("tq,nv", [([64], [256]), ([1], [1]), ([5], [300]), ([130], [129]), ([256], [2304]),
+                                   ([32, 200, 77], [100, 640, 3])])
+def test_llm_importance(pace, tq, nv):
+    out, ref, cq, ck = _llm_case(pace, tq, nv)
+    assert_scores_close(out, ref, what="S_llm_raw")
+    for b in range(len(tq)):
+        assert out[ck[b]:ck[b + 1]].sum() == pytest.approx(tq[b] * 28, rel=1e-4)
+    _no_device_error(pace)
+
+
+def test_llm_importance_gqa_shapes(pace):
+    for Hq, Hkv, D in ((8, 8, 64), (12, 2, 80), (4, 1, 128)):
+        out, ref, _, _ = _llm_case(pace, [40, 9], [70, 260], Hq=Hq, Hkv=Hkv, D=D, seed=Hq)
+        assert_scores_close(out, ref, what=f"S_llm_raw Hq={Hq} Hkv={Hkv}")
+
+
+def test_importance_rejects_bad_args(pace):
+    Q = torch.zeros((8, 2, 80), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(pace.PaceError):
+        pace.pace_vit_attn_importance(Q, Q, [0, 6], merge=4)          # 6 % 4 != 0
+    with pytest.raises(pace.PaceError):
+        pace.pace_vit_attn_importance(Q, Q, [0, 0, 8], merge=4)       # empty image
+    Q = torch.zeros((8, 2, 72), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(pace.PaceError):
+        pace.pace_vit_attn_importance(Q, Q, [0, 8], merge=4)          # head_dim 72
+
+
+# ----------------------------------------------------------------------------------------------
+# DDAE select
+# ----------------------------------------------------------------------------------------------
+def _select(pace, sl, sv, cu, keep, tau=0.5):
+    r = pace.pace_ddae_select(torch.from_numpy(sl.astype(np.float32)).cuda(),
+                              torch.from_numpy(sv.astype(np.float32)).cuda(), cu,
+                              np.concatenate([[0], np.cumsum(keep)]).astype(np.int32), pace.ddae_params(tau=tau))
+    return [x.cpu().numpy() for x in r]
+
+
+@pytest.mark.parametrize("lens,fracs", [([256], [0.1]), ([2584], [0.1]), ([10549], [0.05]), ([1], [1.0]),
+                                        ([7, 300, 1000, 24576], [0.25, 0.0, 1.0, 0.1])])
+def test_ddae_select_random(pace, lens, fracs):
+    rng = np.random.default_rng(len(lens) + lens[0])
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    sl = rng.gamma(0.5, 2.0, size=cu[-1]).astype(np.float32)
+    sv = rng.lognormal(0, 1, size=cu[-1]).astype(np.float32)
+    keep = [O.budget(n, f) for n, f in zip(lens, fracs)]
+    s_final, w, kept = _select(pace, sl, sv, cu, keep)
+    k0 = 0
+    for b, n in enumerate(lens):
+        v0, v1 = cu[b], cu[b + 1]
+        f = O.ddae_fuse(sl[v0:v1].astype(np.float64), sv[v0:v1].astype(np.float64))
+        assert_scores_close(s_final[v0:v1], f["S_final"], atol_frac=2e-3, what="S_final")
+        assert abs(w[b, 0] - f["alpha_w"]) < 2e-3 * f["alpha_w"] and abs(w[b, 1] - f["beta_w"]) < 2e-3 * f["beta_w"]
+        assert_kept_matches(kept[k0:k0 + keep[b]], f["S_final"], keep[b], offset=v0)
+        k0 += keep[b]
+
+
+def test_ddae_select_exact_decisions_with_ties(pace):
+    """S_llm == S_vis with min 0 and max 1: S_final = x exactly in fp32 and fp64, so the kept
+    set (ties broken by the lower index) must equal the oracle's bit for bit."""
+    rng = np.random.default_rng(9)
+    for n, K in ((1000, 100), (4096, 1), (333, 332), (50, 25)):
+        x = np.round(rng.uniform(size=n) * 16) / 16      # many exact ties
+        x[0], x[-1] = 0.0, 1.0
+        cu = np.array([0, n], dtype=np.int32)
+        s_final, w, kept = _select(pace, x, x, cu, [K])
+        np.testing.assert_array_equal(s_final, x.astype(np.float32))
+        assert w[0, 0] == 0.5 and w[0, 1] == 0.5
+        np.testing.assert_array_equal(kept, O.top_k_ascending(x, K))
+
+
+def test_ddae_select_golden_and_constant(pace, golden):
+    g = golden("ddae_four_tokens.txt")
+    sl, sv = np.array(g["s_llm_raw"]), np.array(g["s_vis_raw"])
+    s_final, w, kept = _select(pace, sl, sv, np.array([0, 4], np.int32), [2])
+    np.testing.assert_allclose(s_final, g["s_final"], atol=1e-6)
+    np.testing.assert_allclose(w[0], [g["alpha_w"], g["beta_w"]], atol=1e-6)
+    assert kept.tolist() == [int(v) for v in g["kept_top2"]]
+    s_final, w, kept = _select(pace, np.full(10, 3.0), np.arange(10.0), np.array([0, 10], np.int32), [3])
+    assert kept.tolist() == [7, 8, 9]
+
+
+def test_ddae_select_rejects(pace):
+    with pytest.raises(pace.PaceError):
+        _select(pace, np.zeros(5), np.zeros(5), np.array([0, 5], np.int32), [6])
+    with pytest.raises(pace.PaceError):
+        n = pace.PACE_DDAE_MAX_TOKENS + 1
+        _select(pace, np.zeros(n), np.zeros(n), np.array([0, n], np.int32), [1])
