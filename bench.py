@@ -1,0 +1,499 @@
+#!/usr/bin/env python3
+"""Benchmark of PACE's condense-and-extract hot path on GB300.
+
+One step = the whole hot path on one 4K image per GPU: APC density, APC resample
+(target size read on the device), ViT received attention, LLM text->visual attention,
+DDAE fusion + top-K, gather of the kept embedding rows.  Inputs are seeded synthetic
+arrays shaped like Qwen2.5-VL-7B (3836x2156 image: 42196 patches, ViT Q/K
+[42196,16,80] bf16; LLM Q [256,28,128], K [10549,4,128] bf16; embeddings
+[10549,3584] bf16; keep 10 % = 1055 tokens).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line.  `value` is microseconds per image with inputs resident in HBM,
+timed with CUDA events around each step (each libpace call replayed from a CUDA graph),
+L2 flushed by a 256 MiB write before every step.  `e2e` is the same metric through the
+Python binding with the inputs copied from pinned host memory and the results copied
+back inside the timed region.  Under torchrun every rank processes its own image
+(weak scaling, no collective on the data path); the max over ranks is reported.
+`--impl reference` times the fp64 CPU oracle on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "µs per image for APC+DDAE score/select (4K config); % tensor/HBM peak"
+UNIT = "us/image"
+WORKLOAD = "img4k"
+KEEP = 0.10
+FLUSH_BYTES = 256 << 20
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ----------------------------------------------------------------------------------------------
+# shared helpers
+# ----------------------------------------------------------------------------------------------
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload_config(wl, keep):
+    s = wl.specs[0]
+    return {
+        "workload": (f"{wl.name}: one {s.W}x{s.H} RGB uint8 image per GPU per step "
+                     f"({wl.n_patches[0]} patches, {wl.n_vis[0]} visual tokens); ViT Q/K bf16 "
+                     f"[{wl.n_patches[0]},16,80]; LLM Q bf16 [{s.tq},28,128], K bf16 [{wl.n_vis[0]},4,128]; "
+                     f"embeddings bf16 [{wl.n_vis[0]},3584]; keep {keep:.0%}"),
+        "images_per_step_per_gpu": 1,
+        "keep_fraction": keep,
+        "l2": "flushed before every timed step by a 256 MiB device write",
+        "timing": "CUDA events on the launching stream around each step; each libpace call replayed from a CUDA graph",
+    }
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during a timed region."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                                          "-i", str(self.dev), "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.2)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                    power.append(float(parts[3]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "power_w_max": max(power) if power else None, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------------------------
+# CPU oracle sample (the reference arm and the cpu_baseline leg)
+# ----------------------------------------------------------------------------------------------
+def oracle_sample(wl, keep, vit_rows=2048, crop_div=4):
+    """Times the fp64 oracle on a bounded sample of one image and scales it to a whole image.
+
+    density : oracle on a centred crop with 1/crop_div of each side, scaled by (N/N_crop)^2
+              (Eq. 1 is a double sum over all token pairs);
+    resample: whole image to the oracle's target size;
+    S_vis   : one head, the first vit_rows query rows against all keys, scaled by
+              heads x N / vit_rows;
+    S_llm, fusion, top-K, gather: whole image.
+    """
+    from oracle import pace_oracle as O
+    from paper_2608_27206_gb300 import synth
+    img = wl.images[0]
+    H, W = img.shape[:2]
+    t = {}
+    ch, cw = (H // crop_div) // 14 * 14, (W // crop_div) // 14 * 14
+    y0, x0 = (H - ch) // 2 // 14 * 14, (W - cw) // 2 // 14 * 14
+    crop = np.ascontiguousarray(img[y0:y0 + ch, x0:x0 + cw])
+    n_full, n_crop = (H // 14) * (W // 14), (ch // 14) * (cw // 14)
+    t0 = time.perf_counter()
+    O.apc_density(crop)
+    t["density"] = (time.perf_counter() - t0) * (n_full / n_crop) ** 2
+    st = O.apc_density_tokens(O.patch_tokens(crop))
+    ho, wo = O.target_size(H, W, O.retention_ratio(st["rho"]))
+    t0 = time.perf_counter()
+    O.apc_resample(img, ho, wo)
+    t["resample"] = time.perf_counter() - t0
+    q = synth.bf16_bits_to_f64(wl.vit_q[:vit_rows, 0])
+    k = synth.bf16_bits_to_f64(wl.vit_k[:, 0])
+    t0 = time.perf_counter()
+    O.received_attention(q, k, 1 / math.sqrt(80))
+    t["vit"] = (time.perf_counter() - t0) * wl.vit_q.shape[1] * (wl.vit_q.shape[0] / vit_rows)
+    ql, kl = synth.bf16_bits_to_f64(wl.llm_q), synth.bf16_bits_to_f64(wl.llm_k)
+    t0 = time.perf_counter()
+    s_llm = O.llm_text_visual_importance(ql, kl, wl.cu_q, wl.cu_vis, 1 / math.sqrt(128))
+    t["llm"] = time.perf_counter() - t0
+    s_vis = np.random.default_rng(0).lognormal(size=wl.n_vis[0])  # stand-in map for timing only
+    K = O.budget(wl.n_vis[0], keep)
+    t0 = time.perf_counter()
+    sel = O.ddae_select(s_llm, s_vis, wl.cu_vis, [K])
+    t["select"] = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    O.gather_rows(wl.embed, sel["kept"])
+    t["gather"] = time.perf_counter() - t0
+    total = sum(t.values())
+    sample = (f"fp64 numpy oracle on the host cores: density on a {cw}x{ch} centre crop scaled by (N/N_crop)^2, "
+              f"resample of the whole image, S_vis for 1 of 16 heads x {vit_rows} of {wl.vit_q.shape[0]} query rows "
+              f"scaled linearly, S_llm / fusion / top-K / gather on the whole image")
+    return total, t, sample
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from paper_2608_27206_gb300 import synth
+    wl = synth.make_workload(WORKLOAD, seed=0, keep=KEEP, parts=("image", "vit", "llm", "embed"))
+    for _ in range(args.warmup):
+        oracle_sample(wl, KEEP, vit_rows=args.ref_vit_rows)
+    times, parts, sample = [], None, ""
+    for _ in range(args.steps):
+        tot, parts, sample = oracle_sample(wl, KEEP, vit_rows=args.ref_vit_rows)
+        times.append(tot)
+    per_image_s = float(np.mean(times))
+    value = per_image_s * 1e6
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_image_s * 1e3, "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(wl, KEEP),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample,
+                         "parts_s": {k: round(v, 4) for k, v in parts.items()}},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ----------------------------------------------------------------------------------------------
+# GPU arm
+# ----------------------------------------------------------------------------------------------
+class Pipeline:
+    """Device-resident inputs, outputs and workspaces of one step, and the step itself."""
+
+    def __init__(self, wl, keep, device):
+        import torch
+        from paper_2608_27206_gb300 import pace as P
+        from paper_2608_27206_gb300 import synth
+        self.P, self.torch, self.dev = P, torch, device
+        img = wl.images[0]
+        self.H, self.W = img.shape[:2]
+        buf, off = synth.pack_images(wl.images)
+        self.off = off
+        self.host = {
+            "img": torch.from_numpy(buf),
+            "vit_q": torch.from_numpy(wl.vit_q.view(np.int16)).view(torch.bfloat16),
+            "vit_k": torch.from_numpy(wl.vit_k.view(np.int16)).view(torch.bfloat16),
+            "llm_q": torch.from_numpy(wl.llm_q.view(np.int16)).view(torch.bfloat16),
+            "llm_k": torch.from_numpy(wl.llm_k.view(np.int16)).view(torch.bfloat16),
+            "embed": torch.from_numpy(wl.embed.view(np.int16)).view(torch.bfloat16),
+        }
+        self.d = {k: v.to(device) for k, v in self.host.items()}
+        self.cu = wl.cu_patches
+        self.cu_q, self.cu_v = wl.cu_q, wl.cu_vis
+        self.K = P.pace_budget(wl.n_vis[0], keep)
+        self.cu_keep = np.array([0, self.K], dtype=np.int32)
+        n, nv = wl.n_patches[0], wl.n_vis[0]
+        f32 = torch.float32
+        self.dist = torch.empty(n, dtype=f32, device=device)
+        self.stats = torch.zeros((1, 10), dtype=torch.int32, device=device)
+        self.resized = torch.empty(self.H * self.W * 3, dtype=torch.uint8, device=device)
+        self.s_vis = torch.empty(nv, dtype=f32, device=device)
+        self.s_llm = torch.empty(nv, dtype=f32, device=device)
+        self.s_final = torch.empty(nv, dtype=f32, device=device)
+        self.weights = torch.empty((1, 2), dtype=f32, device=device)
+        self.kept = torch.empty(self.K, dtype=torch.int32, device=device)
+        self.rows = torch.empty((self.K, self.d["embed"].shape[1]), dtype=torch.bfloat16, device=device)
+        u8 = torch.uint8
+        self.ws_d = torch.empty(P.pace_apc_density_workspace_size([self.H], [self.W]), dtype=u8, device=device)
+        self.ws_v = torch.empty(P.pace_vit_attn_importance_workspace_size(self.cu, 16), dtype=u8, device=device)
+        self.ws_l = torch.empty(P.pace_llm_text_visual_importance_workspace_size(self.cu_q, self.cu_v, 28, 4),
+                                dtype=u8, device=device)
+        self.parts = [("density", self.density), ("resample", self.resample), ("vit", self.vit),
+                      ("llm", self.llm), ("select", self.select), ("gather", self.gather)]
+
+    def density(self):
+        self.P.pace_apc_density(self.d["img"], self.off, [self.H], [self.W], d_out=self.dist, stats=self.stats,
+                                ws=self.ws_d)
+
+    def resample(self):
+        self.P.pace_apc_resample(self.d["img"], self.off, [self.H], [self.W], self.stats, self.resized, [0])
+
+    def vit(self):
+        self.P.pace_vit_attn_importance(self.d["vit_q"], self.d["vit_k"], self.cu, 1 / math.sqrt(80), 4,
+                                        out=self.s_vis, ws=self.ws_v)
+
+    def llm(self):
+        self.P.pace_llm_text_visual_importance(self.d["llm_q"], self.d["llm_k"], self.cu_q, self.cu_v,
+                                               1 / math.sqrt(128), out=self.s_llm, ws=self.ws_l)
+
+    def select(self):
+        self.P.pace_ddae_select(self.s_llm, self.s_vis, self.cu_v, self.cu_keep, s_final=self.s_final,
+                                weights=self.weights, kept=self.kept)
+
+    def gather(self):
+        self.P.pace_gather(self.d["embed"], self.kept, dst=self.rows)
+
+    def step(self):
+        for _, f in self.parts:
+            f()
+
+    def capture(self):
+        """One CUDA graph per call, captured after an eager warm-up."""
+        torch = self.torch
+        self.graphs = []
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            self.step()
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        for name, f in self.parts:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                f()
+            self.graphs.append((name, g))
+        torch.cuda.synchronize()
+
+
+def algorithmic_counts(wl, keep, r_ratio):
+    """Algorithmic flops / bytes per step (one image), per part."""
+    n, nv = wl.n_patches[0], wl.n_vis[0]
+    H, W = wl.specs[0].H, wl.specs[0].W
+    tq = wl.specs[0].tq
+    K = int(math.floor(keep * nv + 0.5))
+    img_bytes = H * W * 3
+    s = math.sqrt(max(r_ratio, 0.0))
+    ho = min(H, max(28, 28 * int(math.floor(H * s / 28 + 0.5))))
+    wo = min(W, max(28, 28 * int(math.floor(W * s / 28 + 0.5))))
+    return {
+        "vit_flops": 2 * 2 * n * n * 80 * 16,            # two passes of 2 N^2 d H
+        "llm_flops": 2 * 2 * tq * 28 * nv * 128,
+        "density_bytes": img_bytes + 4 * n,                # image once + d_i
+        "resample_bytes": img_bytes + ho * wo * 3,
+        "select_bytes": 2 * 4 * nv + 4 * nv + 4 * K,       # two raw maps in, S_final + kept out
+        "gather_bytes": 2 * K * 3584 * 2,
+    }
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    device = torch.device("cuda", torch.cuda.current_device())
+    from paper_2608_27206_gb300 import build as pace_build
+    pace_build.build()
+    from paper_2608_27206_gb300 import pace as P
+    from paper_2608_27206_gb300 import synth
+    P.pace_init(torch.cuda.current_device())
+
+    wl = synth.make_workload(WORKLOAD, seed=rank, keep=KEEP)
+    pipe = Pipeline(wl, KEEP, device)
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
+
+    # launches per step (eager), then graphs
+    c0 = P.pace_kernel_launch_count()
+    pipe.step()
+    torch.cuda.synchronize()
+    launches_per_step = P.pace_kernel_launch_count() - c0
+    pipe.capture()
+    for _ in range(args.warmup):
+        flush.zero_()
+        for _, g in pipe.graphs:
+            g.replay()
+    torch.cuda.synchronize()
+    code, where = P.pace_device_status(clear=True)
+    if code != 0:
+        raise RuntimeError(f"device status {code} from kernel {where} during warm-up")
+
+    nparts = len(pipe.graphs)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nparts + 1)] for _ in range(args.steps)]
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_wall0 = time.perf_counter()
+    for k in range(args.steps):
+        flush.zero_()
+        ev[k][0].record()
+        for i, (_, g) in enumerate(pipe.graphs):
+            g.replay()
+            ev[k][i + 1].record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    t_wall = time.perf_counter() - t_wall0
+    clocks = sampler.stop()
+    part_ms = {name: [] for name, _ in pipe.graphs}
+    step_ms = []
+    for k in range(args.steps):
+        step_ms.append(ev[k][0].elapsed_time(ev[k][nparts]))
+        for i, (name, _) in enumerate(pipe.graphs):
+            part_ms[name].append(ev[k][i].elapsed_time(ev[k][i + 1]))
+    total_ms = float(sum(step_ms))
+    if world > 1:
+        tt = torch.tensor([total_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / args.steps
+    value = total_ms * 1e3 / (args.steps * world)       # us per image over all ranks
+
+    # correctness guard on the timed outputs
+    code, where = P.pace_device_status(clear=True)
+    if code != 0:
+        raise RuntimeError(f"device status {code} from kernel {where} in the timed region")
+    stats = P.stats_dict(pipe.stats)[0]
+
+    # e2e: pinned host inputs -> device, the public calls, results -> pinned host
+    pinned = {k: v.pin_memory() for k, v in pipe.host.items()}
+    out_host = {"kept": torch.empty(pipe.K, dtype=torch.int32).pin_memory(),
+                "rows": torch.empty(tuple(pipe.rows.shape), dtype=torch.bfloat16).pin_memory(),
+                "stats": torch.empty((1, 10), dtype=torch.int32).pin_memory(),
+                "s_final": torch.empty(pipe.s_final.numel(), dtype=torch.float32).pin_memory()}
+    h2d = sum(v.numel() * v.element_size() for v in pinned.values())
+    d2h = sum(v.numel() * v.element_size() for v in out_host.values())
+
+    def e2e_step():
+        for kname, v in pinned.items():
+            pipe.d[kname].copy_(v, non_blocking=True)
+        pipe.step()
+        out_host["kept"].copy_(pipe.kept, non_blocking=True)
+        out_host["rows"].copy_(pipe.rows, non_blocking=True)
+        out_host["stats"].copy_(pipe.stats, non_blocking=True)
+        out_host["s_final"].copy_(pipe.s_final, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize()
+    e_start, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e_start.record()
+    for _ in range(args.steps):
+        e2e_step()
+    e_end.record()
+    torch.cuda.synchronize()
+    e2e_ms = e_start.elapsed_time(e_end)
+    if world > 1:
+        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+        dist.barrier()
+    e2e_value = e2e_ms * 1e3 / (args.steps * world)
+
+    if rank == 0:
+        peaks, peak_src = load_peaks()
+        cnt = algorithmic_counts(wl, KEEP, stats["r"])
+        vit_ms = statistics.mean(part_ms["vit"])
+        achieved = cnt["vit_flops"] / (vit_ms * 1e-3) / 1e12
+        peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+        hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+        mean = {k: statistics.mean(v) for k, v in part_ms.items()}
+        other = {}
+        for name, key in (("density", "density_bytes"), ("resample", "resample_bytes"), ("select", "select_bytes"),
+                          ("gather", "gather_bytes")):
+            gbs = cnt[key] / (mean[name] * 1e-3) / 1e9
+            other[name] = {"bound": "hbm", "us": round(mean[name] * 1e3, 2), "achieved": round(gbs, 1),
+                           "peak": hbm, "unit": "GB/s", "frac": round(gbs / hbm, 4), "bytes": cnt[key]}
+        llm_tf = cnt["llm_flops"] / (mean["llm"] * 1e-3) / 1e12
+        other["llm"] = {"bound": "tensor", "us": round(mean["llm"] * 1e3, 2), "achieved": round(llm_tf, 1),
+                        "peak": peak, "unit": "TFLOP/s", "frac": round(llm_tf / peak, 4), "flops": cnt["llm_flops"]}
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            tot, parts, sample = oracle_sample(wl, KEEP, vit_rows=args.ref_vit_rows)
+            cpu = {"value": tot * 1e6, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample,
+                   "parts_s": {k: round(v, 4) for k, v in parts.items()}}
+        line = {
+            "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": workload_config(wl, KEEP),
+            "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
+                         "frac": round(achieved / peak, 4), "traffic": None,
+                         "kernel": "ViT received attention (attn_row_lse + attn_colsum + attn_reduce), one launch "
+                                   "of pace_vit_attn_importance",
+                         "algorithmic_flops": cnt["vit_flops"], "us": round(vit_ms * 1e3, 1),
+                         "peak_source": f"{peak_src} bf16 dense burst (MEASURED_PEAKS.json)"
+                         if peak_src == "measured" else "fallback 1.9 PFLOP/s bf16"},
+            "rooflines_other": other,
+            "breakdown_us": {k: round(v * 1e3, 2) for k, v in mean.items()},
+            "visual_tokens_scored_per_s": round(wl.n_vis[0] * world / (ms_per_step * 1e-3), 1),
+            "cpu_baseline": cpu,
+            "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clocks,
+            "apc": {"rho": round(stats["rho"], 5), "r": round(stats["r"], 5),
+                    "target": [stats["h_out"], stats["w_out"]]},
+            "wall_s_timed_region": round(t_wall, 4),
+        }
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--ref-vit-rows", type=int, default=2048)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -65,6 +65,10 @@ PACE_API pace_status_t pace_init(int device);
  * (0 if none).  With clear != 0 the word is reset to PACE_OK afterwards. */
 PACE_API pace_status_t pace_device_status(int* code, int* where, int clear);
 
+/* Number of CUDA kernels this library has launched in the calling process (all threads,
+ * all devices).  Instrumentation for benchmarks: counts launches, not completed work. */
+PACE_API uint64_t pace_kernel_launch_count(void);
+
 /* ==============================================================================
  * Condense — Adaptive Pixel Compressor (APC), Sec. 3.2, Eq. 1-6; App. B.3.
  * ============================================================================== */

@@ -24,6 +24,7 @@
 // head dimension per row), one tile per 16-wide slice of the head dimension.
 //
 // GQA: query head h reads KV head h / G.  The ViT case is G = 1.
+#include <atomic>
 #include <cmath>
 #include <mutex>
 
@@ -591,13 +592,21 @@ pace_status_t check_segments(int B, const int32_t* cu, int multiple) {
   return PACE_OK;
 }
 
+// Opts the two passes into their shared-memory size, once per device (so that later
+// calls, including ones made during stream capture, only launch).
 template <int D>
 pace_status_t set_smem_attrs(size_t* s1, size_t* s2) {
   using C = Cfg<D>;
   *s1 = 1024 + 2 * C::TILE_BYTES + C::STAGES * C::TILE_BYTES + sizeof(SmemCtl);
   *s2 = 1024 + 2 * C::TILE_BYTES + C::STAGES * C::TILE_BYTES + C::STAGES * kTile * 4 + sizeof(SmemCtl);
+  static std::atomic<uint64_t> done{0};
+  int dev = 0;
+  PACE_CUDA(cudaGetDevice(&dev));
+  const uint64_t bit = uint64_t{1} << (dev & 63);
+  if (done.load(std::memory_order_acquire) & bit) return PACE_OK;
   PACE_CUDA(cudaFuncSetAttribute(attn_row_lse<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(*s1)));
   PACE_CUDA(cudaFuncSetAttribute(attn_colsum<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(*s2)));
+  done.fetch_or(bit, std::memory_order_acq_rel);
   return PACE_OK;
 }
 

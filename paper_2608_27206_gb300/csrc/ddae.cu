@@ -8,6 +8,7 @@
 // ballots, the lower index winning among equal scores.
 //
 // pace_gather: one warp per kept row, 16-byte vector loads and stores.
+#include <atomic>
 #include <cfloat>
 #include <cmath>
 
@@ -281,8 +282,18 @@ extern "C" pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s
   if (!(tau > 0.f) || !std::isfinite(tau)) return PACE_ERR_INVALID_ARG;
   PACE_CHECK(check_device());
   const size_t smem = static_cast<size_t>(2 * max_nv) * sizeof(float);
-  PACE_CUDA(cudaFuncSetAttribute(ddae_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 static_cast<int>(smem)));
+  {
+    // opt in to the largest size once per device
+    static std::atomic<uint64_t> done{0};
+    int dev = 0;
+    PACE_CUDA(cudaGetDevice(&dev));
+    const uint64_t bit = uint64_t{1} << (dev & 63);
+    if (!(done.load(std::memory_order_acquire) & bit)) {
+      PACE_CUDA(cudaFuncSetAttribute(ddae_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(2 * PACE_DDAE_MAX_TOKENS * sizeof(float))));
+      done.fetch_or(bit, std::memory_order_acq_rel);
+    }
+  }
   for (int c0 = 0; c0 < B; c0 += kSelMaxB) {
     const int nb = (B - c0) < kSelMaxB ? (B - c0) : kSelMaxB;
     SelectTable t;

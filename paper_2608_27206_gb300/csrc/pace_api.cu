@@ -1,5 +1,6 @@
 // libpace host API: status strings, per-device initialisation (sm_103 check and
 // device status word), budget helper and parameter defaults.
+#include <atomic>
 #include <cmath>
 #include <mutex>
 
@@ -10,9 +11,10 @@ namespace pace {
 namespace {
 constexpr int kMaxDevices = 64;
 thread_local int t_last_cuda_error = 0;
+std::atomic<uint64_t> g_launches{0};
 std::mutex g_mutex;
-bool g_checked[kMaxDevices] = {};
-bool g_ok[kMaxDevices] = {};
+// Per-device state: 0 = not checked yet, 1 = sm_103 and initialised, 2 = unsupported.
+std::atomic<int> g_state[kMaxDevices];
 int* g_status[kMaxDevices] = {};
 
 // Status word of every device that loads the library: [code, kernel id].
@@ -26,13 +28,15 @@ pace_status_t set_cuda_error(cudaError_t e) {
 
 static pace_status_t init_device_locked(int dev) {
   if (dev < 0 || dev >= kMaxDevices) return PACE_ERR_INVALID_ARG;
-  if (g_checked[dev]) return g_ok[dev] ? PACE_OK : PACE_ERR_UNSUPPORTED_ARCH;
+  const int st = g_state[dev].load(std::memory_order_acquire);
+  if (st != 0) return st == 1 ? PACE_OK : PACE_ERR_UNSUPPORTED_ARCH;
   int major = 0, minor = 0;
   PACE_CUDA(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev));
   PACE_CUDA(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev));
-  g_checked[dev] = true;
-  g_ok[dev] = (major == 10 && minor == 3);
-  if (!g_ok[dev]) return PACE_ERR_UNSUPPORTED_ARCH;
+  if (!(major == 10 && minor == 3)) {
+    g_state[dev].store(2, std::memory_order_release);
+    return PACE_ERR_UNSUPPORTED_ARCH;
+  }
   int prev = -1;
   PACE_CUDA(cudaGetDevice(&prev));
   if (prev != dev) PACE_CUDA(cudaSetDevice(dev));
@@ -40,18 +44,19 @@ static pace_status_t init_device_locked(int dev) {
   cudaError_t e = cudaGetSymbolAddress(&p, g_status_word);
   if (e == cudaSuccess) e = cudaMemset(p, 0, 2 * sizeof(int));
   if (prev != dev) cudaSetDevice(prev);
-  if (e != cudaSuccess) {
-    g_checked[dev] = false;
-    return set_cuda_error(e);
-  }
+  if (e != cudaSuccess) return set_cuda_error(e);
   g_status[dev] = static_cast<int*>(p);
+  g_state[dev].store(1, std::memory_order_release);
   return PACE_OK;
 }
 
 pace_status_t check_device() {
   int dev = -1;
   PACE_CUDA(cudaGetDevice(&dev));
-  if (dev >= 0 && dev < kMaxDevices && g_checked[dev]) return g_ok[dev] ? PACE_OK : PACE_ERR_UNSUPPORTED_ARCH;
+  if (dev >= 0 && dev < kMaxDevices) {
+    const int st = g_state[dev].load(std::memory_order_acquire);
+    if (st != 0) return st == 1 ? PACE_OK : PACE_ERR_UNSUPPORTED_ARCH;
+  }
   std::lock_guard<std::mutex> lk(g_mutex);
   return init_device_locked(dev);
 }
@@ -59,12 +64,14 @@ pace_status_t check_device() {
 int* device_status_word() {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  if (g_state[dev].load(std::memory_order_acquire) != 1) return nullptr;
   return g_status[dev];
 }
 
 pace_status_t check_launch() {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return set_cuda_error(e);
+  g_launches.fetch_add(1, std::memory_order_relaxed);
   return PACE_OK;
 }
 
@@ -85,6 +92,8 @@ const char* pace_status_string(pace_status_t s) {
 }
 
 int pace_last_cuda_error(void) { return pace::t_last_cuda_error; }
+
+uint64_t pace_kernel_launch_count(void) { return pace::g_launches.load(std::memory_order_relaxed); }
 
 pace_status_t pace_init(int device) {
   std::lock_guard<std::mutex> lk(pace::g_mutex);

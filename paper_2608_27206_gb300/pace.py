@@ -45,6 +45,7 @@ _I64P = ctypes.POINTER(ctypes.c_int64)
 _SIGS = {
     "pace_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "pace_last_cuda_error": (ctypes.c_int, []),
+    "pace_kernel_launch_count": (ctypes.c_uint64, []),
     "pace_init": (ctypes.c_int, [ctypes.c_int]),
     "pace_device_status": (ctypes.c_int, [_I32P, _I32P, ctypes.c_int]),
     "pace_apc_params_default": (None, [ctypes.POINTER(ApcParams)]),
@@ -149,6 +150,11 @@ def pace_device_status(clear: bool = True):
     code, where = ctypes.c_int32(0), ctypes.c_int32(0)
     _check("pace_device_status", lib().pace_device_status(ctypes.byref(code), ctypes.byref(where), int(clear)))
     return code.value, where.value
+
+
+def pace_kernel_launch_count() -> int:
+    """Kernels launched by libpace so far in this process."""
+    return int(lib().pace_kernel_launch_count())
 
 
 def pace_budget(n_vis: int, frac: float) -> int:

@@ -56,12 +56,17 @@ def _rng(seed: int, workload: str, part: str, index: int = 0) -> np.random.Gener
 # ----------------------------------------------------------------------------------------------
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
     """Round fp32 values to bf16, round-to-nearest-even; returns uint16 bit patterns."""
-    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
-    r = (u >> 16) & np.uint32(1)
-    r += np.uint32(0x7FFF)
-    r += u                      # finite inputs never wrap: 0xFF7FFFFF + 0x8000 < 2**32
-    r >>= 16
-    return r.astype(np.uint16)
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).reshape(-1)
+    out = np.empty(u.shape, dtype=np.uint16)
+    step = 1 << 20                       # cache-sized chunks
+    for i in range(0, u.size, step):
+        c = u[i:i + step]
+        r = (c >> 16) & np.uint32(1)
+        r += np.uint32(0x7FFF)
+        r += c                           # finite inputs never wrap: 0xFF7FFFFF + 0x8000 < 2**32
+        r >>= 16
+        out[i:i + step] = r
+    return out.reshape(np.shape(x))
 
 
 def bf16_bits_to_f64(b: np.ndarray) -> np.ndarray:
@@ -117,7 +122,9 @@ def make_qk(rng: np.random.Generator, rows: int, heads: int, dim: int,
     s = rng.lognormal(0.0, 0.5, size=rows).astype(np.float32)
     if boost_rows is not None and len(boost_rows):
         s[boost_rows] *= np.float32(boost)
-    x *= s[:, None, None]
+    step = max(1, (1 << 20) // max(1, heads * dim))
+    for i in range(0, rows, step):
+        x[i:i + step] *= s[i:i + step, None, None]
     return f32_to_bf16_bits(x)
 
 
