@@ -123,6 +123,31 @@ PACE_API pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img_o
                                void* ws, size_t ws_bytes, pace_stream_t stream);
 
 /*
+ * pace_apc_density without caller scratch.  The paper has no counterpart to this call:
+ * it exists for callers that cannot allocate device memory themselves, such as a plugin
+ * running inside a host framework that owns every allocation, or a latency-critical path
+ * where cudaMalloc (which may synchronise the device) is not allowed.  It computes exactly
+ * what pace_apc_density computes, with the same kernels, but its scratch lives in one
+ * file-scope device array owned by the library (about 330 KB on every GPU that loads the
+ * library, held until the process exits).  It allocates and frees nothing.
+ *
+ *  - At most PACE_APC_STATIC_MAX_IMAGES images and PACE_APC_STATIC_MAX_PATCHES patches
+ *    (14x14) in total per call; larger calls return PACE_ERR_INVALID_ARG and launch nothing.
+ *  - d_out is required (the per-patch distances are an output, not scratch).
+ *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress)
+ *    with that device current; make that first call before any stream capture.
+ *  - Every call shares the one array and it keeps the last call's contents (the call clears
+ *    the part that must start at zero).  Calls whose work overlaps on the GPU — on different
+ *    streams, or from different threads — race on it; serialise them.
+ * Other arguments are as for pace_apc_density.
+ */
+#define PACE_APC_STATIC_MAX_IMAGES 16
+#define PACE_APC_STATIC_MAX_PATCHES 65536
+PACE_API pace_status_t pace_apc_density_static(const uint8_t* img, const int64_t* img_off, const int32_t* H,
+                                               const int32_t* W, int B, const pace_apc_params* params,
+                                               float* d_out, pace_apc_stats* stats, pace_stream_t stream);
+
+/*
  * APC resize (Sec. 3.2 "Adaptive Condensation"; App. B.3: width and height scaled by
  * sqrt(r), bicubic).  Separable cubic convolution (a = -0.5) with centre-aligned
  * sampling, support widened by the downscale factor (antialias), the window clipped

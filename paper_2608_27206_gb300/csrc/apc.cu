@@ -17,6 +17,7 @@
 // horizontally 8 at a time into shared memory and accumulated vertically in registers.
 #include <cfloat>
 #include <cmath>
+#include <mutex>
 
 #include "pace_common.cuh"
 
@@ -557,4 +558,97 @@ extern "C" pace_status_t pace_apc_resample_to(const uint8_t* src, const int64_t*
                                               const int32_t* W, const int32_t* H_out, const int32_t* W_out,
                                               uint8_t* dst, const int64_t* dst_off, int B, pace_stream_t stream) {
   return resample_impl(src, src_off, H, W, H_out, W_out, nullptr, dst, dst_off, B, stream);
+}
+
+// ------------------------------------------------------------------------------------------------
+// pace_apc_density_static: the same density computation with library-owned scratch
+// ------------------------------------------------------------------------------------------------
+// Scratch of pace_apc_density_static, in a file-scope device array instead of caller memory:
+// the per-image 589-entry fixed-point column sums, then the per-patch inverse token norms.
+// Every GPU that loads the library holds this array until the process exits.
+namespace pace {
+namespace {
+constexpr size_t kStaticSumsBytes =
+    static_cast<size_t>(PACE_APC_STATIC_MAX_IMAGES) * kTokDim * sizeof(unsigned long long);
+constexpr size_t kStaticInvOff = (kStaticSumsBytes + 255) / 256 * 256;
+constexpr size_t kStaticBytes = kStaticInvOff + static_cast<size_t>(PACE_APC_STATIC_MAX_PATCHES) * sizeof(float);
+
+static __device__ __align__(256) unsigned char g_apc_static_scratch[kStaticBytes];
+
+std::mutex g_static_mutex;
+void* g_static_ptr[64] = {};
+
+// Device address of the array for the current device.  The name g_apc_static_scratch in host
+// code is only a host-side handle, so the address is looked up once per device.
+pace_status_t static_scratch(unsigned char** out) {
+  int dev = -1;
+  PACE_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= 64) return PACE_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lk(g_static_mutex);
+  if (g_static_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    PACE_CUDA(cudaGetSymbolAddress(&p, g_apc_static_scratch));
+    if (p == nullptr) return set_cuda_error(cudaErrorInvalidSymbol);
+    g_static_ptr[dev] = p;
+  }
+  *out = static_cast<unsigned char*>(g_static_ptr[dev]);
+  return PACE_OK;
+}
+}  // namespace
+}  // namespace pace
+
+extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64_t* img_off, const int32_t* H,
+                                                 const int32_t* W, int B, const pace_apc_params* params,
+                                                 float* d_out, pace_apc_stats* stats, pace_stream_t stream) {
+  PACE_CHECK(check_images(img, img_off, H, W, B));
+  if (B == 0) return PACE_OK;
+  if (stats == nullptr || d_out == nullptr) return PACE_ERR_INVALID_ARG;
+  if (B > PACE_APC_STATIC_MAX_IMAGES) return PACE_ERR_INVALID_ARG;
+  int64_t n_total = 0;
+  for (int b = 0; b < B; ++b) n_total += static_cast<int64_t>(H[b] / kPatch) * (W[b] / kPatch);
+  if (n_total > PACE_APC_STATIC_MAX_PATCHES) return PACE_ERR_INVALID_ARG;
+  pace_apc_params p;
+  if (params) p = *params; else pace_apc_params_default(&p);
+  if (!(p.tail_frac > 0.f && p.tail_frac <= 1.f) || !(p.gamma > 0.f) || !(p.alpha >= 0.f && p.alpha <= 1.f) ||
+      !(p.r_min <= p.r_max) || p.align < 1)
+    return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(check_device());
+  unsigned char* scratch = nullptr;
+  PACE_CHECK(static_scratch(&scratch));
+  auto* sums = reinterpret_cast<unsigned long long*>(scratch);
+  auto* inv = reinterpret_cast<float*>(scratch + kStaticInvOff);
+  // the array keeps the previous call's contents: the column sums must start from zero
+  PACE_CUDA(cudaMemsetAsync(sums, 0, static_cast<size_t>(B) * kTokDim * sizeof(unsigned long long), stream));
+  ApcTable t{};
+  t.nb = B;
+  t.b_base = 0;
+  t.unit_prefix[0] = 0;
+  bool wide = true;
+  int patch0 = 0;
+  for (int b = 0; b < B; ++b) {
+    t.off[b] = img_off[b];
+    t.H[b] = H[b];
+    t.W[b] = W[b];
+    t.gw[b] = W[b] / kPatch;
+    t.chunks[b] = (t.gw[b] + kStrip - 1) / kStrip;
+    t.patch0[b] = patch0;
+    const int N = (H[b] / kPatch) * t.gw[b];
+    double kt = std::floor(static_cast<double>(p.tail_frac) * N + 0.5);
+    if (kt < 1) kt = 1;
+    if (kt > N) kt = N;
+    t.ktail[b] = static_cast<int>(kt);
+    patch0 += N;
+    t.unit_prefix[b + 1] = t.unit_prefix[b] + (H[b] / kPatch) * t.chunks[b];
+    if ((static_cast<int64_t>(W[b]) * 3) % 4 != 0 || (t.gw[b] % 2) != 0 || (img_off[b] % 4) != 0) wide = false;
+  }
+  const int units = t.unit_prefix[B];
+  if (wide) apc_pass1<true><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums);
+  else apc_pass1<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums);
+  PACE_CHECK(check_launch());
+  if (wide) apc_pass2<true><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d_out, stats);
+  else apc_pass2<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d_out, stats);
+  PACE_CHECK(check_launch());
+  TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
+  apc_tail<<<B, 1024, 0, stream>>>(t, d_out, tp, stats);
+  return check_launch();
 }

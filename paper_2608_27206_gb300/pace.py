@@ -52,6 +52,8 @@ _SIGS = {
     "pace_apc_density_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, _I32P]),
     "pace_apc_density": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, ctypes.c_int, ctypes.POINTER(ApcParams), _P, _P,
                                         _P, ctypes.c_size_t, _P]),
+    "pace_apc_density_static": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, ctypes.c_int, ctypes.POINTER(ApcParams),
+                                               _P, _P, _P]),
     "pace_apc_resample": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, _P, _P, _I64P, ctypes.c_int, _P]),
     "pace_apc_resample_to": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, _I32P, _I32P, _P, _I64P, ctypes.c_int, _P]),
     "pace_vit_attn_importance_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, ctypes.c_int]),
@@ -203,6 +205,34 @@ def pace_apc_density(img: torch.Tensor, img_off, H, W, params: Optional[ApcParam
                                 ctypes.byref(params) if params is not None else None, _dev(d_out), _dev(stats),
                                 _dev(ws), ws.numel() * ws.element_size(), _stream(stream))
     _check("pace_apc_density", st)
+    return d_out[:n], stats[:B]
+
+
+PACE_APC_STATIC_MAX_IMAGES = 16
+PACE_APC_STATIC_MAX_PATCHES = 65536
+
+
+def pace_apc_density_static(img: torch.Tensor, img_off, H, W, params: Optional[ApcParams] = None,
+                            d_out: Optional[torch.Tensor] = None, stats: Optional[torch.Tensor] = None,
+                            stream=None):
+    """pace_apc_density with the library's own static scratch: no workspace argument.
+
+    For callers that cannot allocate device scratch.  Limited to PACE_APC_STATIC_MAX_IMAGES
+    images and PACE_APC_STATIC_MAX_PATCHES patches per call; calls that overlap on the GPU
+    share one scratch array and must be serialised.  Returns (d, stats) like pace_apc_density.
+    """
+    off, h, w = _i64(img_off), _i32(H), _i32(W)
+    B = len(h)
+    n = int(((h // 14).astype(np.int64) * (w // 14)).sum())
+    dev = img.device
+    if d_out is None:
+        d_out = torch.empty(max(n, 1), dtype=torch.float32, device=dev)
+    if stats is None:
+        stats = torch.zeros((max(B, 1), 10), dtype=torch.int32, device=dev)
+    st = lib().pace_apc_density_static(_dev(img), _pi64(off), _pi32(h), _pi32(w), B,
+                                       ctypes.byref(params) if params is not None else None, _dev(d_out),
+                                       _dev(stats), _stream(stream))
+    _check("pace_apc_density_static", st)
     return d_out[:n], stats[:B]
 
 
