@@ -479,6 +479,30 @@ def run_gpu(args):
     return 0
 
 
+def run_profile(args):
+    """Runs one libpace call `--reps` times on the workload (for ncu captures; prints no result)."""
+    import torch
+    torch.cuda.set_device(0)
+    from paper_2608_27206_gb300 import build as pace_build
+    pace_build.build()
+    from paper_2608_27206_gb300 import pace as P
+    from paper_2608_27206_gb300 import synth
+    P.pace_init(0)
+    wl = synth.make_workload(args.workload, seed=0, keep=KEEP)
+    pipe = Pipeline(wl, KEEP, torch.device("cuda", 0))
+    fns = dict(pipe.parts)
+    needs = {"resample": ["density"], "select": ["vit", "llm"], "gather": ["vit", "llm", "select"]}
+    for name in needs.get(args.profile, []):      # producers of this call's inputs
+        fns[name]()
+    for _ in range(args.reps):
+        fns[args.profile]()
+    torch.cuda.synchronize()
+    code, where = P.pace_device_status(clear=True)
+    if code != 0:
+        raise RuntimeError(f"device status {code} from kernel {where}")
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -487,7 +511,13 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--ref-vit-rows", type=int, default=2048)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile", choices=("density", "resample", "vit", "llm", "select", "gather"),
+                    help="run only this call --reps times (for profiler captures)")
+    ap.add_argument("--reps", type=int, default=1)
+    ap.add_argument("--workload", default=WORKLOAD)
     args = ap.parse_args()
+    if args.profile:
+        return run_profile(args)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     if args.impl == "reference":

@@ -4,26 +4,37 @@
 // P_ij = exp(s_ij - lse_i), s_ij = scale q_i . k_j.  They are computed flash-style in two
 // passes so that the N x N score matrix is never stored:
 //
-//   pass 1  attn_row_lse   S = Q K^T tile by tile on tcgen05 (M = 128 query rows, N = 128
-//           keys), online row max / sum of exp2 on the CUDA cores, giving the base-2
-//           log-sum-exp L_i = log2 sum_j 2^(c s_ij), c = scale * log2(e).  Optionally split
-//           over key ranges (partial (m, l) pairs merged by attn_lse_combine).
-//   pass 2  attn_colsum    S^T = K Q^T (M = 128 keys, N = 128 queries): every TMEM lane is one
-//           key, so each epilogue thread owns one key and accumulates 2^(c s_ji - L_i) over
-//           the whole query stream in registers; no cross-thread reduction and no atomics.
+//   pass 1  attn_row_lse   S = Q K^T on tcgen05, online row max / sum of exp2 on the CUDA
+//           cores, giving the base-2 log-sum-exp L_i = log2 sum_j 2^(c s_ij),
+//           c = scale * log2(e), stored negated.  Optionally split over key ranges (partial
+//           (m, l) pairs merged by attn_lse_combine).
+//   pass 2  attn_colsum    S^T = K Q^T: every TMEM lane is one key, so each epilogue thread
+//           owns one key and accumulates 2^(c s_ji - L_i) over the whole query stream in
+//           registers; no cross-thread reduction and no atomics.
 //   reduce  attn_reduce    sums the per-head (or per KV-head) partial maps and pools the
 //           `merge` consecutive patches of each merged token.
 //
-// CTA layout of both passes (320 threads):
-//   warp 0      TMA producer (one lane): resident operand tiles once, then a 4-6 stage ring
-//   warp 1      TMEM allocation (512 columns) and MMA issue (one lane)
-//   warps 2-9   two epilogue warpgroups; warpgroup w owns resident tile w (two query tiles
-//               in pass 1, two key tiles in pass 2) and its two TMEM accumulators
-//               (double-buffered: columns w*256 + {0, 128})
-// Operands are K-major bf16 tiles staged by TMA with the 32-byte swizzle (16 elements of the
-// head dimension per row), one tile per 16-wide slice of the head dimension.
+// Both passes run on CTA pairs (clusters of 2) with the two-SM MMA: one 256 x 256 x 16
+// tcgen05.mma per K-step, A = 256 resident rows (128 in each CTA), B = 256 streamed rows
+// (128 loaded by each CTA), so each SM reads half of B and a 128 x 256 fp32 accumulator
+// lands in each CTA's TMEM.  N = 256 halves the shared-memory operand traffic per flop
+// compared with 128-wide tiles.
+//
+// CTA layout (576 threads, one CTA per SM):
+//   warp 0       TMA producer (one lane): this CTA's resident tile once, then its half of
+//                every streamed tile through a ring of stages; completion is counted on the
+//                even CTA's barriers
+//   warp 1       pair TMEM allocation (512 columns = two 128 x 256 accumulators) and, in the
+//                even CTA, MMA issue (one lane)
+//   warps 2-17   four epilogue warpgroups; warpgroup e = 2p + hh reads columns hh*128.. of
+//                accumulator p (stream tiles j with j % 2 == p); results of the four are
+//                merged at the end
+// Operands are K-major bf16 tiles staged by TMA: 64-column blocks with the 128-byte swizzle,
+// and a trailing 16-column slice with the 32-byte swizzle when the head dimension is not a
+// multiple of 64 (80 = 64 + 16).  MMA descriptors are built once and advanced by immediates.
 //
 // GQA: query head h reads KV head h / G.  The ViT case is G = 1.
+#include <algorithm>
 #include <atomic>
 #include <cmath>
 #include <mutex>
@@ -38,25 +49,33 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kTile = 128;
-constexpr int kThreads = 320;
+constexpr int kTile = 128;                // rows of a tile held by one CTA
+constexpr int kPair = 256;                // rows of a tile held by a CTA pair
+constexpr int kEpiWarps = 16;
+constexpr int kThreads = 64 + 32 * kEpiWarps;   // 576
 constexpr int kAttnMaxB = 64;
-constexpr int kSliceBytes = kTile * 32;   // one 128-row x 16-element bf16 slice
+constexpr int kBlock128 = kTile * 128;    // 128 rows x 64 bf16, 128-byte swizzle
+constexpr int kSlice32 = kTile * 32;      // 128 rows x 16 bf16, 32-byte swizzle
 constexpr uint32_t kTmemCols = 512;
-constexpr int kTargetItems = 304;         // 2 CTAs' worth per SM on 152 SMs
+constexpr int kTargetItems = 152;         // one CTA pair per two SMs, two waves
 
+// A 128-row operand tile of head dimension D is stored as NB blocks of 64 columns with the
+// 128-byte swizzle followed by R slices of 16 columns with the 32-byte swizzle
+// (D = 80: one block + one slice; D = 128: two blocks; D = 64: one block).
 template <int D>
 struct Cfg {
-  static constexpr int KC = D / 16;                       // slices of the head dimension
-  static constexpr int STAGES = (D == 128) ? 4 : (D == 80 ? 4 : 6);
-  static constexpr int TILE_BYTES = KC * kSliceBytes;
-  static constexpr uint32_t IDESC = idesc_bf16_f32(128, 128);
+  static constexpr int NB = D / 64;
+  static constexpr int R = (D % 64) / 16;
+  static constexpr int TILE_BYTES = NB * kBlock128 + R * kSlice32;
+  static constexpr int STAGES = (D == 128) ? 5 : 8;
+  static constexpr uint32_t IDESC = idesc_bf16_f32(256, 256);
+  static_assert(D % 16 == 0 && TILE_BYTES % 1024 == 0, "head dim");
 };
 
 struct AttnTable {
   int q0[kAttnMaxB], nq[kAttnMaxB];   // query rows of image b
   int k0[kAttnMaxB], nk[kAttnMaxB];   // key rows of image b
-  int lpad[kAttnMaxB];                // first padded L row of image b
+  int lpad[kAttnMaxB];                // first padded L row of image b (multiple of 256)
   int item_prefix[kAttnMaxB + 1];
   int nb;
   int H;        // query heads
@@ -73,9 +92,10 @@ __device__ __forceinline__ int find_image(const AttnTable& t, int item) {
 }
 
 struct SmemCtl {
-  uint64_t bars[32];
+  uint64_t bars[40];
   uint32_t tmem_base;
   int abort;
+  float xchg[3][2][kTile];   // hand-over between the four epilogue warpgroups
 };
 
 __device__ __forceinline__ void set_abort(SmemCtl* ctl, int* status, int kernel) {
@@ -86,17 +106,131 @@ __device__ __forceinline__ bool aborted(const SmemCtl* ctl) {
   return *reinterpret_cast<const volatile int*>(&ctl->abort) != 0;
 }
 
-// Loads 4 x 32 TMEM columns of this warp's 32 lanes into v[0..127] (fp32 bit patterns).
-__device__ __forceinline__ void load_row128(uint32_t taddr, uint32_t (&v)[4][32]) {
-  tmem_ld_32x32b_x32(taddr + 0, v[0]);
-  tmem_ld_32x32b_x32(taddr + 32, v[1]);
-  tmem_ld_32x32b_x32(taddr + 64, v[2]);
-  tmem_ld_32x32b_x32(taddr + 96, v[3]);
+// TMA of this CTA's 128 rows (y .. y + 127, columns x0 .. x0 + D) into dst; completion is
+// counted on the (possibly remote) barrier `bar`.
+template <int D>
+__device__ __forceinline__ void load_tile(uint8_t* dst, const CUtensorMap* m128, const CUtensorMap* m32, int x0,
+                                          int y, uint32_t bar) {
+  using C = Cfg<D>;
+#pragma unroll
+  for (int i = 0; i < C::NB; ++i) tma_load_2d_pair(smem_u32(dst + i * kBlock128), m128, x0 + 64 * i, y, bar);
+#pragma unroll
+  for (int r = 0; r < C::R; ++r)
+    tma_load_2d_pair(smem_u32(dst + C::NB * kBlock128 + r * kSlice32), m32, x0 + 64 * C::NB + 16 * r, y, bar);
+}
+
+// Shared-memory descriptors of a tile: [0] for its 128-byte-swizzled blocks, [1] for its
+// 32-byte-swizzled slices.  Adding (bytes >> 4) moves the start address.
+template <int D>
+__device__ __forceinline__ void tile_desc(const uint8_t* tile, uint64_t& d128, uint64_t& d32) {
+  d128 = smem_desc_kmajor_sw128(smem_u32(tile));
+  d32 = smem_desc_kmajor_sw32(smem_u32(tile + Cfg<D>::NB * kBlock128));
+}
+
+// Pair MMA D[tmem] = A B^T over the whole head dimension: 4 K-steps per 128-byte block,
+// 1 per 32-byte slice.
+template <int D>
+__device__ __forceinline__ void mma_tile(uint32_t d, uint64_t a128, uint64_t a32, uint64_t b128, uint64_t b32) {
+  using C = Cfg<D>;
+#pragma unroll
+  for (int i = 0; i < C::NB; ++i)
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint64_t off = static_cast<uint64_t>(i * (kBlock128 >> 4) + k * 2);
+      mma_bf16_ss_pair(d, a128 + off, b128 + off, C::IDESC, (i | k) != 0);
+    }
+#pragma unroll
+  for (int r = 0; r < C::R; ++r) {
+    const uint64_t off = static_cast<uint64_t>(r * (kSlice32 >> 4));
+    mma_bf16_ss_pair(d, a32 + off, b32 + off, C::IDESC, (C::NB | r) != 0);
+  }
+}
+
+// 64 TMEM columns of this warp's 32 lanes -> v[0..63] (fp32 bit patterns), ready to use.
+__device__ __forceinline__ void load_cols64(uint32_t taddr, uint32_t (&v)[64]) {
+  tmem_ld_32x32b_x64(taddr, v);
   tmem_wait_ld();
-  reg_fence32(v[0]);
-  reg_fence32(v[1]);
-  reg_fence32(v[2]);
-  reg_fence32(v[3]);
+  reg_fence64(v);
+}
+
+// Online (max, sum of exp2) update of one row with 64 new scores (raw dot products);
+// entries at and beyond `valid` are ignored.
+__device__ __forceinline__ void lse_update64(const uint32_t (&v)[64], int valid, float c, float& m_run,
+                                             float& l_run) {
+  if (valid <= 0) return;
+  float s[64];
+#pragma unroll
+  for (int e = 0; e < 64; ++e) s[e] = __uint_as_float(v[e]);
+  if (valid < 64) {
+#pragma unroll
+    for (int e = 0; e < 64; ++e)
+      if (e >= valid) s[e] = -INFINITY;
+  }
+  float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+#pragma unroll
+  for (int e = 0; e < 64; e += 8) {
+    mx0 = max3(mx0, s[e + 0], s[e + 1]);
+    mx1 = max3(mx1, s[e + 2], s[e + 3]);
+    mx2 = max3(mx2, s[e + 4], s[e + 5]);
+    mx3 = max3(mx3, s[e + 6], s[e + 7]);
+  }
+  const float mt = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * c;
+  if (mt > m_run) {
+    l_run *= ex2_approx(m_run - mt);
+    m_run = mt;
+  }
+  const float2 cc = make_float2(c, c);
+  const float2 nm = make_float2(-m_run, -m_run);
+  float2 a0 = make_float2(0.f, 0.f), a1 = a0;
+#pragma unroll
+  for (int e = 0; e < 64; e += 4) {
+    const float2 x0 = ffma2(make_float2(s[e], s[e + 1]), cc, nm);
+    const float2 x1 = ffma2(make_float2(s[e + 2], s[e + 3]), cc, nm);
+    a0 = fadd2(a0, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
+    a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
+  }
+  const float2 a = fadd2(a0, a1);
+  l_run += a.x + a.y;
+}
+
+// acc += sum_e 2^(c s_e + nL_e) over 64 columns; nL (negated base-2 LSE) from shared memory.
+__device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], const float* nL, float c, float2 acc) {
+  const float2 cc = make_float2(c, c);
+  const float4* L4 = reinterpret_cast<const float4*>(nL);
+  float2 a1 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int e = 0; e < 64; e += 4) {
+    const float4 l = L4[e / 4];
+    const float2 x0 = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), cc, make_float2(l.x, l.y));
+    const float2 x1 =
+        ffma2(make_float2(__uint_as_float(v[e + 2]), __uint_as_float(v[e + 3])), cc, make_float2(l.z, l.w));
+    acc = fadd2(acc, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
+    a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
+  }
+  return fadd2(acc, a1);
+}
+
+// Shared teardown: waits for the pair's MMAs, lets in-flight copies land after an abort, then
+// releases TMEM with both CTAs in step.
+__device__ __forceinline__ void pair_teardown(SmemCtl* ctl, uint32_t b_done, uint32_t tmem, int* status,
+                                              int kernel) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == 1 && lane == 0) {
+    if (!mbar_wait(b_done, 0, kWaitLimitNs)) record_error(status, PACE_ERR_TIMEOUT, kernel);
+  }
+  if (threadIdx.x == 0 && aborted(ctl)) {   // give outstanding TMA copies time to land
+    const uint64_t t0 = globaltimer_ns();
+    while (globaltimer_ns() - t0 < 100000ull) {
+    }
+  }
+  __syncthreads();
+  tc_fence_before_sync();
+  cluster_sync_all();
+  tc_fence_after_sync();
+  if (warp == 1) tmem_dealloc_pair(tmem, kTmemCols);
+  cluster_sync_all();
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -104,37 +238,39 @@ __device__ __forceinline__ void load_row128(uint32_t taddr, uint32_t (&v)[4][32]
 // ------------------------------------------------------------------------------------------------
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constant__ CUtensorMap tmq,
+                                                            const __grid_constant__ CUtensorMap tmq32,
                                                             const __grid_constant__ CUtensorMap tmk,
+                                                            const __grid_constant__ CUtensorMap tmk32,
                                                             const __grid_constant__ AttnTable t, float c,
-                                                            float* __restrict__ L_out,
+                                                            float* __restrict__ nL_out,
                                                             float2* __restrict__ ml_out, int* status) {
   using C = Cfg<D>;
-  constexpr int KC = C::KC, ST = C::STAGES;
+  constexpr int ST = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem;                                // 2 resident query tiles
-  uint8_t* sK = sQ + 2 * C::TILE_BYTES;              // ST key stages
+  uint8_t* sQ = smem;                                // this CTA's resident query tile
+  uint8_t* sK = sQ + C::TILE_BYTES;                  // ST stages of this CTA's half of a key tile
   SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + ST * C::TILE_BYTES);
-  const uint32_t b_qfull = smem_u32(&ctl->bars[0]);
-  const uint32_t b_done = smem_u32(&ctl->bars[1]);
-  auto b_kfull = [&](int s) { return smem_u32(&ctl->bars[2 + s]); };
-  auto b_kempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };
-  auto b_sfull = [&](int i) { return smem_u32(&ctl->bars[2 + 2 * ST + i]); };
-  auto b_sfree = [&](int i) { return smem_u32(&ctl->bars[2 + 2 * ST + 4 + i]); };
+  const uint32_t b_qfull = smem_u32(&ctl->bars[0]);     // even CTA: both Q halves landed
+  const uint32_t b_done = smem_u32(&ctl->bars[1]);      // both: all pair MMAs finished
+  auto b_kfull = [&](int s) { return smem_u32(&ctl->bars[2 + s]); };          // even CTA
+  auto b_kempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };    // both
+  auto b_sfull = [&](int p) { return smem_u32(&ctl->bars[2 + 2 * ST + p]); }; // both
+  auto b_sfree = [&](int p) { return smem_u32(&ctl->bars[4 + 2 * ST + p]); }; // even CTA
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int item = blockIdx.x;
+  const uint32_t rank = cluster_ctarank();
+  const int item = blockIdx.x >> 1;
   const int b = find_image(t, item);
   int r = item - t.item_prefix[b];
   const int split = r % t.splits;
   r /= t.splits;
-  const int npair = (t.nq[b] + 2 * kTile - 1) / (2 * kTile);
+  const int npair = (t.nq[b] + kPair - 1) / kPair;
   const int pair = r % npair;
   const int h = r / npair;
   const int g = h / t.G;
-  const int qrow0 = pair * 2 * kTile;                               // local query row of tile 0
-  const int nqt = min(2, (t.nq[b] - qrow0 + kTile - 1) / kTile);    // 1 or 2 valid query tiles
-  const int nkt_all = (t.nk[b] + kTile - 1) / kTile;
+  const int qrow0 = pair * kPair + kTile * static_cast<int>(rank);     // this CTA's first local query row
+  const int nkt_all = (t.nk[b] + kPair - 1) / kPair;
   const int kt0 = static_cast<int>((static_cast<int64_t>(split) * nkt_all) / t.splits);
   const int kt1 = static_cast<int>((static_cast<int64_t>(split + 1) * nkt_all) / t.splits);
   const int nj = kt1 - kt0;
@@ -146,32 +282,35 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
       mbar_init(b_kfull(s), 1);
       mbar_init(b_kempty(s), 1);
     }
-    for (int i = 0; i < 4; ++i) {
-      mbar_init(b_sfull(i), 1);
-      mbar_init(b_sfree(i), 4);
+    for (int p = 0; p < 2; ++p) {
+      mbar_init(b_sfull(p), 1);
+      mbar_init(b_sfree(p), 2 * 8);
     }
     ctl->abort = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&ctl->tmem_base), kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(&ctl->tmem_base), kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before_sync();
-  __syncthreads();
+  cluster_sync_all();
   tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
-  int issued = 0;
 
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmq);
       prefetch_tensormap(&tmk);
-      mbar_arrive_expect_tx(b_qfull, nqt * C::TILE_BYTES);
-      for (int qt = 0; qt < nqt; ++qt)
-        for (int kc = 0; kc < KC; ++kc)
-          tma_load_2d(smem_u32(sQ + (qt * KC + kc) * kSliceBytes), &tmq, h * D + kc * 16,
-                      t.q0[b] + qrow0 + qt * kTile, b_qfull);
+      if (C::R > 0) {
+        prefetch_tensormap(&tmq32);
+        prefetch_tensormap(&tmk32);
+      }
+      // the even CTA's full barriers count the bytes of both halves; the odd CTA's copies
+      // complete there too
+      const uint32_t qfull_L = mapa_shared(b_qfull, 0);
+      if (rank == 0) mbar_arrive_expect_tx(b_qfull, 2 * C::TILE_BYTES);
+      load_tile<D>(sQ, &tmq, &tmq32, h * D, t.q0[b] + qrow0, qfull_L);
       for (int j = 0; j < nj; ++j) {
         const int s = j % ST, u = j / ST;
         if (u > 0 && !mbar_wait(b_kempty(s), (u - 1) & 1, kWaitLimitNs)) {
@@ -179,130 +318,101 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
           break;
         }
         if (aborted(ctl)) break;
-        mbar_arrive_expect_tx(b_kfull(s), C::TILE_BYTES);
-        const int krow = t.k0[b] + (kt0 + j) * kTile;
-        for (int kc = 0; kc < KC; ++kc)
-          tma_load_2d(smem_u32(sK + (s * KC + kc) * kSliceBytes), &tmk, g * D + kc * 16, krow, b_kfull(s));
-        issued = j + 1;
+        const uint32_t kfull_L = mapa_shared(b_kfull(s), 0);
+        if (rank == 0) mbar_arrive_expect_tx(b_kfull(s), 2 * C::TILE_BYTES);
+        load_tile<D>(sK + s * C::TILE_BYTES, &tmk, &tmk32, g * D,
+                     t.k0[b] + (kt0 + j) * kPair + kTile * static_cast<int>(rank), kfull_L);
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && rank == 0) {
+      uint64_t aq128, aq32, bk128, bk32;
+      tile_desc<D>(sQ, aq128, aq32);
+      tile_desc<D>(sK, bk128, bk32);
       bool ok = mbar_wait(b_qfull, 0, kWaitLimitNs);
       if (!ok) set_abort(ctl, status, K_ATTN_ROW_LSE);
       for (int j = 0; ok && j < nj; ++j) {
         const int s = j % ST, u = j / ST;
-        if (!mbar_wait(b_kfull(s), u & 1, kWaitLimitNs) || aborted(ctl)) {
+        const int p = j & 1, v = j >> 1;
+        if (!mbar_wait(b_kfull(s), u & 1, kWaitLimitNs) ||
+            (v > 0 && !mbar_wait(b_sfree(p), (v - 1) & 1, kWaitLimitNs)) || aborted(ctl)) {
           set_abort(ctl, status, K_ATTN_ROW_LSE);
           break;
         }
         tc_fence_after_sync();
-        const int buf = j & 1, v = j >> 1;
-        for (int qt = 0; qt < nqt; ++qt) {
-          if (v > 0 && !mbar_wait(b_sfree(qt * 2 + buf), (v - 1) & 1, kWaitLimitNs)) {
-            set_abort(ctl, status, K_ATTN_ROW_LSE);
-            ok = false;
-            break;
-          }
-          tc_fence_after_sync();
-          const uint32_t d = tmem + qt * 256 + buf * 128;
-#pragma unroll
-          for (int kc = 0; kc < KC; ++kc)
-            mma_bf16_ss(d, smem_desc_kmajor_sw32(smem_u32(sQ + (qt * KC + kc) * kSliceBytes)),
-                        smem_desc_kmajor_sw32(smem_u32(sK + (s * KC + kc) * kSliceBytes)), C::IDESC, kc > 0);
-          mma_commit(b_sfull(qt * 2 + buf));
-        }
-        mma_commit(b_kempty(s));
+        const uint64_t so = static_cast<uint64_t>(s * (C::TILE_BYTES >> 4));
+        mma_tile<D>(tmem + p * 256, aq128, aq32, bk128 + so, bk32 + so);
+        mma_commit_pair_mc(b_sfull(p), 3);
+        mma_commit_pair_mc(b_kempty(s), 3);
       }
-      mma_commit(b_done);
-      if (!mbar_wait(b_done, 0, kWaitLimitNs)) record_error(status, PACE_ERR_TIMEOUT, K_ATTN_ROW_LSE);
+      mma_commit_pair_mc(b_done, 3);
     }
     __syncwarp();
   } else {
-    // epilogue: warpgroup qt = (warp - 2) / 4, TMEM lane quadrant = warp % 4
-    const int qt = (warp - 2) >> 2;
+    // epilogue warpgroup e = 2p + hh: accumulator p (key tiles j % 2 == p), columns hh * 128 ..
+    const int e = (warp - 2) >> 2;
+    const int p = e >> 1, hh = e & 1;
     const int quad = warp & 3;
     const int rr = quad * 32 + lane;
-    if (qt < nqt) {
-      float m_run = -INFINITY, l_run = 0.f;
-      const uint32_t trow = tmem + (static_cast<uint32_t>(quad * 32) << 16) + qt * 256;
-      for (int j = 0; j < nj; ++j) {
-        const int buf = j & 1, v = j >> 1;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(qt * 2 + buf), v & 1, kWaitLimitNs));
-        if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
-          set_abort(ctl, status, K_ATTN_ROW_LSE);
-          break;
-        }
-        tc_fence_after_sync();
-        uint32_t sv[4][32];
-        load_row128(trow + buf * 128, sv);
-        tc_fence_before_sync();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(b_sfree(qt * 2 + buf));
-        const int valid = t.nk[b] - (kt0 + j) * kTile;   // keys of this tile inside the image
-        if (valid < kTile) {
-#pragma unroll
-          for (int a = 0; a < 4; ++a)
-#pragma unroll
-            for (int e = 0; e < 32; ++e)
-              if (a * 32 + e >= valid) sv[a][e] = __float_as_uint(-INFINITY);
-        }
-        float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
-#pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          mx0 = max3(mx0, __uint_as_float(sv[0][e]), __uint_as_float(sv[0][e + 1]));
-          mx1 = max3(mx1, __uint_as_float(sv[1][e]), __uint_as_float(sv[1][e + 1]));
-          mx2 = max3(mx2, __uint_as_float(sv[2][e]), __uint_as_float(sv[2][e + 1]));
-          mx3 = max3(mx3, __uint_as_float(sv[3][e]), __uint_as_float(sv[3][e + 1]));
-        }
-        const float mt = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * c;
-        if (mt > m_run) {
-          l_run *= ex2_approx(m_run - mt);
-          m_run = mt;
-        }
-        const float nm = -m_run;
-        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          a0 += ex2_approx(fmaf(__uint_as_float(sv[0][e]), c, nm));
-          a1 += ex2_approx(fmaf(__uint_as_float(sv[1][e]), c, nm));
-          a2 += ex2_approx(fmaf(__uint_as_float(sv[2][e]), c, nm));
-          a3 += ex2_approx(fmaf(__uint_as_float(sv[3][e]), c, nm));
-        }
-        l_run += (a0 + a1) + (a2 + a3);
+    const uint32_t sfree_L = mapa_shared(b_sfree(p), 0);
+    float m_run = -INFINITY, l_run = 0.f;
+    const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
+    for (int j = p; j < nj; j += 2) {
+      const int v = j >> 1;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs));
+      if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
+        set_abort(ctl, status, K_ATTN_ROW_LSE);
+        break;
       }
-      const int row = qrow0 + qt * kTile + rr;          // local query row
+      tc_fence_after_sync();
+      const int valid = t.nk[b] - ((kt0 + j) * kPair + hh * kTile);   // keys of these columns in the image
+      uint32_t sv[64];
+      load_cols64(tbuf, sv);
+      lse_update64(sv, valid, c, m_run, l_run);
+      load_cols64(tbuf + 64, sv);
+      tc_fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(sfree_L);
+      if (valid > 64) lse_update64(sv, valid - 64, c, m_run, l_run);
+    }
+    // merge the four warpgroups' (m, l) of each row
+    if (e > 0) {
+      ctl->xchg[e - 1][0][rr] = m_run;
+      ctl->xchg[e - 1][1][rr] = l_run;
+    }
+    named_barrier_sync(1, 32 * kEpiWarps);
+    if (e == 0) {
+      float M = m_run;
+#pragma unroll
+      for (int i = 0; i < 3; ++i) M = fmaxf(M, ctl->xchg[i][0][rr]);
+      float l = l_run > 0.f ? l_run * ex2_approx(m_run - M) : 0.f;
+#pragma unroll
+      for (int i = 0; i < 3; ++i) {
+        const float li = ctl->xchg[i][1][rr];
+        if (li > 0.f) l += li * ex2_approx(ctl->xchg[i][0][rr] - M);
+      }
+      const int row = qrow0 + rr;                       // local query row
       const int64_t prow = static_cast<int64_t>(h) * t.prows + t.lpad[b] + row;
       if (t.splits == 1) {
-        L_out[prow] = row < t.nq[b] ? m_run + log2f(l_run) : INFINITY;
+        nL_out[prow] = row < t.nq[b] ? -(M + log2f(l)) : -INFINITY;
       } else {
         ml_out[static_cast<int64_t>(split) * t.H * t.prows + prow] =
-            row < t.nq[b] ? make_float2(m_run, l_run) : make_float2(-INFINITY, 0.f);
+            (row < t.nq[b] && l > 0.f) ? make_float2(M, l) : make_float2(-INFINITY, 0.f);
       }
     }
   }
-
-  // teardown: every wait above is bounded, so all threads arrive here
-  tc_fence_before_sync();
-  __syncthreads();
-  if (warp == 0 && lane == 0 && aborted(ctl)) {
-    // let in-flight TMA loads land before the CTA's shared memory is released
-    mbar_wait(b_qfull, 0, kWaitLimitNs);
-    for (int j = max(0, issued - ST); j < issued; ++j) mbar_wait(b_kfull(j % ST), (j / ST) & 1, kWaitLimitNs);
-  }
-  tc_fence_after_sync();
-  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+  pair_teardown(ctl, b_done, tmem, status, K_ATTN_ROW_LSE);
 }
 
-// Merges per-split (m, l) pairs into L = m + log2(l); rows past the image get +inf.
+// Merges per-split (m, l) pairs into -L = -(m + log2(l)); rows past the image get -inf.
 __global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ AttnTable t,
-                                                        const float2* __restrict__ ml, float* __restrict__ L_out) {
-  // blockIdx.x = (h, image, tile) flattened through per-image tile counts
+                                                        const float2* __restrict__ ml, float* __restrict__ nL_out) {
+  // blockIdx.x = (image, 128-row tile of its padded rows) flattened
   int rem = blockIdx.x;
   const int h = blockIdx.y;
   int b = 0;
   for (; b < t.nb; ++b) {
-    const int nt = (t.nq[b] + kTile - 1) / kTile;
+    const int nt = (t.nq[b] + kPair - 1) / kPair * 2;
     if (rem < nt) break;
     rem -= nt;
   }
@@ -310,7 +420,7 @@ __global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ 
   const int row = rem * kTile + threadIdx.x;
   const int64_t prow = static_cast<int64_t>(h) * t.prows + t.lpad[b] + row;
   if (row >= t.nq[b]) {
-    L_out[prow] = INFINITY;
+    nL_out[prow] = -INFINITY;
     return;
   }
   float M = -INFINITY;
@@ -320,7 +430,7 @@ __global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ 
     const float2 p = ml[static_cast<int64_t>(s) * t.H * t.prows + prow];
     if (p.y > 0.f) l += p.y * ex2_approx(p.x - M);
   }
-  L_out[prow] = M + log2f(l);
+  nL_out[prow] = -(M + log2f(l));
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -328,35 +438,38 @@ __global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ 
 // ------------------------------------------------------------------------------------------------
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant__ CUtensorMap tmq,
+                                                           const __grid_constant__ CUtensorMap tmq32,
                                                            const __grid_constant__ CUtensorMap tmk,
+                                                           const __grid_constant__ CUtensorMap tmk32,
                                                            const __grid_constant__ AttnTable t, float c,
-                                                           const float* __restrict__ L, float* __restrict__ part,
+                                                           const float* __restrict__ nL, float* __restrict__ part,
                                                            int* status) {
   using C = Cfg<D>;
-  constexpr int KC = C::KC, ST = C::STAGES;
+  constexpr int ST = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sA = smem;                                 // 2 resident key tiles
-  uint8_t* sQ = sA + 2 * C::TILE_BYTES;               // ST query stages
-  float* sL = reinterpret_cast<float*>(sQ + ST * C::TILE_BYTES);   // ST x 128 floats
-  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sL + ST * kTile);
-  const uint32_t b_afull = smem_u32(&ctl->bars[0]);
-  const uint32_t b_done = smem_u32(&ctl->bars[1]);
-  auto b_qfull = [&](int s) { return smem_u32(&ctl->bars[2 + s]); };
-  auto b_qempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };
-  auto b_sfull = [&](int i) { return smem_u32(&ctl->bars[2 + 2 * ST + i]); };
-  auto b_sfree = [&](int i) { return smem_u32(&ctl->bars[2 + 2 * ST + 4 + i]); };
+  uint8_t* sA = smem;                                 // this CTA's resident key tile
+  uint8_t* sQ = sA + C::TILE_BYTES;                   // ST stages of this CTA's half of a query tile
+  float* sL = reinterpret_cast<float*>(sQ + ST * C::TILE_BYTES);   // ST x 256 floats (-L of the whole tile)
+  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sL + ST * kPair);
+  const uint32_t b_afull = smem_u32(&ctl->bars[0]);     // even CTA
+  const uint32_t b_done = smem_u32(&ctl->bars[1]);      // both
+  auto b_qfull = [&](int s) { return smem_u32(&ctl->bars[2 + s]); };            // even CTA
+  auto b_qempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };      // both
+  auto b_lfull = [&](int s) { return smem_u32(&ctl->bars[2 + 2 * ST + s]); };   // both
+  auto b_sfull = [&](int p) { return smem_u32(&ctl->bars[2 + 3 * ST + p]); };   // both
+  auto b_sfree = [&](int p) { return smem_u32(&ctl->bars[4 + 3 * ST + p]); };   // even CTA
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int item = blockIdx.x;
+  const uint32_t rank = cluster_ctarank();
+  const int item = blockIdx.x >> 1;
   const int b = find_image(t, item);
   const int r = item - t.item_prefix[b];
-  const int nkp = (t.nk[b] + 2 * kTile - 1) / (2 * kTile);
+  const int nkp = (t.nk[b] + kPair - 1) / kPair;
   const int kp = r % nkp;
   const int g = r / nkp;
-  const int krow0 = kp * 2 * kTile;                                   // local key row of tile 0
-  const int nkt = min(2, (t.nk[b] - krow0 + kTile - 1) / kTile);
-  const int nqt = (t.nq[b] + kTile - 1) / kTile;
+  const int krow0 = kp * kPair + kTile * static_cast<int>(rank);     // this CTA's first local key row
+  const int nqt = (t.nq[b] + kPair - 1) / kPair;
   const int nj = t.G * nqt;                                           // stream: (head in group, query tile)
 
   if (threadIdx.x == 0) {
@@ -364,34 +477,36 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
     mbar_init(b_done, 1);
     for (int s = 0; s < ST; ++s) {
       mbar_init(b_qfull(s), 1);
-      mbar_init(b_qempty(s), 1 + 4 * nkt);
+      mbar_init(b_qempty(s), 1 + 8);   // pair MMA done + the 8 warps that read this stage's -L
+      mbar_init(b_lfull(s), 1);
     }
-    for (int i = 0; i < 4; ++i) {
-      mbar_init(b_sfull(i), 1);
-      mbar_init(b_sfree(i), 4);
+    for (int p = 0; p < 2; ++p) {
+      mbar_init(b_sfull(p), 1);
+      mbar_init(b_sfree(p), 2 * 8);
     }
     ctl->abort = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(&ctl->tmem_base), kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(&ctl->tmem_base), kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before_sync();
-  __syncthreads();
+  cluster_sync_all();
   tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
-  int issued = 0;
 
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmq);
       prefetch_tensormap(&tmk);
-      mbar_arrive_expect_tx(b_afull, nkt * C::TILE_BYTES);
-      for (int kt = 0; kt < nkt; ++kt)
-        for (int kc = 0; kc < KC; ++kc)
-          tma_load_2d(smem_u32(sA + (kt * KC + kc) * kSliceBytes), &tmk, g * D + kc * 16,
-                      t.k0[b] + krow0 + kt * kTile, b_afull);
+      if (C::R > 0) {
+        prefetch_tensormap(&tmq32);
+        prefetch_tensormap(&tmk32);
+      }
+      const uint32_t afull_L = mapa_shared(b_afull, 0);
+      if (rank == 0) mbar_arrive_expect_tx(b_afull, 2 * C::TILE_BYTES);
+      load_tile<D>(sA, &tmk, &tmk32, g * D, t.k0[b] + krow0, afull_L);
       for (int j = 0; j < nj; ++j) {
         const int s = j % ST, u = j / ST;
         if (u > 0 && !mbar_wait(b_qempty(s), (u - 1) & 1, kWaitLimitNs)) {
@@ -399,103 +514,83 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
           break;
         }
         if (aborted(ctl)) break;
-        const int hh = j / nqt, qt = j - hh * nqt;
-        const int h = g * t.G + hh;
-        mbar_arrive_expect_tx(b_qfull(s), C::TILE_BYTES + kTile * 4);
-        for (int kc = 0; kc < KC; ++kc)
-          tma_load_2d(smem_u32(sQ + (s * KC + kc) * kSliceBytes), &tmq, h * D + kc * 16, t.q0[b] + qt * kTile,
-                      b_qfull(s));
-        bulk_load(smem_u32(sL + s * kTile), L + static_cast<int64_t>(h) * t.prows + t.lpad[b] + qt * kTile,
-                  kTile * 4, b_qfull(s));
-        issued = j + 1;
+        const int hq = j / nqt, qt = j - hq * nqt;
+        const int h = g * t.G + hq;
+        const uint32_t qfull_L = mapa_shared(b_qfull(s), 0);
+        if (rank == 0) mbar_arrive_expect_tx(b_qfull(s), 2 * C::TILE_BYTES);
+        load_tile<D>(sQ + s * C::TILE_BYTES, &tmq, &tmq32, h * D,
+                     t.q0[b] + qt * kPair + kTile * static_cast<int>(rank), qfull_L);
+        mbar_arrive_expect_tx(b_lfull(s), kPair * 4);
+        bulk_load(smem_u32(sL + s * kPair), nL + static_cast<int64_t>(h) * t.prows + t.lpad[b] + qt * kPair,
+                  kPair * 4, b_lfull(s));
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && rank == 0) {
+      uint64_t ak128, ak32, bq128, bq32;
+      tile_desc<D>(sA, ak128, ak32);
+      tile_desc<D>(sQ, bq128, bq32);
       bool ok = mbar_wait(b_afull, 0, kWaitLimitNs);
       if (!ok) set_abort(ctl, status, K_ATTN_COLSUM);
       for (int j = 0; ok && j < nj; ++j) {
         const int s = j % ST, u = j / ST;
-        if (!mbar_wait(b_qfull(s), u & 1, kWaitLimitNs) || aborted(ctl)) {
+        const int p = j & 1, v = j >> 1;
+        if (!mbar_wait(b_qfull(s), u & 1, kWaitLimitNs) ||
+            (v > 0 && !mbar_wait(b_sfree(p), (v - 1) & 1, kWaitLimitNs)) || aborted(ctl)) {
           set_abort(ctl, status, K_ATTN_COLSUM);
           break;
         }
         tc_fence_after_sync();
-        const int buf = j & 1, v = j >> 1;
-        for (int kt = 0; kt < nkt; ++kt) {
-          if (v > 0 && !mbar_wait(b_sfree(kt * 2 + buf), (v - 1) & 1, kWaitLimitNs)) {
-            set_abort(ctl, status, K_ATTN_COLSUM);
-            ok = false;
-            break;
-          }
-          tc_fence_after_sync();
-          const uint32_t d = tmem + kt * 256 + buf * 128;
-#pragma unroll
-          for (int kc = 0; kc < KC; ++kc)
-            mma_bf16_ss(d, smem_desc_kmajor_sw32(smem_u32(sA + (kt * KC + kc) * kSliceBytes)),
-                        smem_desc_kmajor_sw32(smem_u32(sQ + (s * KC + kc) * kSliceBytes)), C::IDESC, kc > 0);
-          mma_commit(b_sfull(kt * 2 + buf));
-        }
-        mma_commit(b_qempty(s));
+        const uint64_t so = static_cast<uint64_t>(s * (C::TILE_BYTES >> 4));
+        mma_tile<D>(tmem + p * 256, ak128, ak32, bq128 + so, bq32 + so);
+        mma_commit_pair_mc(b_sfull(p), 3);
+        mma_commit_pair_mc(b_qempty(s), 3);
       }
-      mma_commit(b_done);
-      if (!mbar_wait(b_done, 0, kWaitLimitNs)) record_error(status, PACE_ERR_TIMEOUT, K_ATTN_COLSUM);
+      mma_commit_pair_mc(b_done, 3);
     }
     __syncwarp();
   } else {
-    const int kt = (warp - 2) >> 2;
+    // epilogue warpgroup e = 2p + hh: accumulator p (stream tiles j % 2 == p), query columns hh * 128 ..
+    const int e = (warp - 2) >> 2;
+    const int p = e >> 1, hh = e & 1;
     const int quad = warp & 3;
     const int rr = quad * 32 + lane;
-    if (kt < nkt) {
-      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-      const uint32_t trow = tmem + (static_cast<uint32_t>(quad * 32) << 16) + kt * 256;
-      for (int j = 0; j < nj; ++j) {
-        const int buf = j & 1, v = j >> 1;
-        const int s = j % ST, u = j / ST;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(kt * 2 + buf), v & 1, kWaitLimitNs));
-        if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
-          set_abort(ctl, status, K_ATTN_COLSUM);
-          break;
-        }
-        tc_fence_after_sync();
-        uint32_t sv[4][32];
-        load_row128(trow + buf * 128, sv);
-        tc_fence_before_sync();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(b_sfree(kt * 2 + buf));
-        if (!__all_sync(0xffffffffu, mbar_wait(b_qfull(s), u & 1, kWaitLimitNs))) {   // L of this stage (landed)
-          set_abort(ctl, status, K_ATTN_COLSUM);
-          break;
-        }
-        const float4* Lp = reinterpret_cast<const float4*>(sL + s * kTile);
-#pragma unroll
-        for (int a = 0; a < 4; ++a) {
-#pragma unroll
-          for (int e = 0; e < 32; e += 4) {
-            const float4 l4 = Lp[a * 8 + e / 4];
-            a0 += ex2_approx(fmaf(__uint_as_float(sv[a][e + 0]), c, -l4.x));
-            a1 += ex2_approx(fmaf(__uint_as_float(sv[a][e + 1]), c, -l4.y));
-            a2 += ex2_approx(fmaf(__uint_as_float(sv[a][e + 2]), c, -l4.z));
-            a3 += ex2_approx(fmaf(__uint_as_float(sv[a][e + 3]), c, -l4.w));
-          }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(b_qempty(s));
+    const uint32_t sfree_L = mapa_shared(b_sfree(p), 0);
+    float2 acc = make_float2(0.f, 0.f);
+    const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
+    for (int j = p; j < nj; j += 2) {
+      const int v = j >> 1;
+      const int s = j % ST, u = j / ST;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs) &&
+                                                  mbar_wait(b_lfull(s), u & 1, kWaitLimitNs));
+      if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
+        set_abort(ctl, status, K_ATTN_COLSUM);
+        break;
       }
-      const int key = krow0 + kt * kTile + rr;
-      if (key < t.nk[b]) part[static_cast<int64_t>(g) * t.ktot + t.k0[b] + key] = (a0 + a1) + (a2 + a3);
+      tc_fence_after_sync();
+      const float* Ls = sL + s * kPair + hh * kTile;
+      uint32_t sv[64];
+      load_cols64(tbuf, sv);
+      acc = colsum64(sv, Ls, c, acc);
+      load_cols64(tbuf + 64, sv);
+      tc_fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(sfree_L);
+      acc = colsum64(sv, Ls + 64, c, acc);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_qempty(s));
+    }
+    const float a = acc.x + acc.y;
+    if (e > 0) ctl->xchg[e - 1][0][rr] = a;
+    named_barrier_sync(1, 32 * kEpiWarps);
+    if (e == 0) {
+      const int key = krow0 + rr;
+      if (key < t.nk[b])
+        part[static_cast<int64_t>(g) * t.ktot + t.k0[b] + key] =
+            (a + ctl->xchg[0][0][rr]) + (ctl->xchg[1][0][rr] + ctl->xchg[2][0][rr]);
     }
   }
-
-  tc_fence_before_sync();
-  __syncthreads();
-  if (warp == 0 && lane == 0 && aborted(ctl)) {
-    // let in-flight TMA loads land before the CTA's shared memory is released
-    mbar_wait(b_afull, 0, kWaitLimitNs);
-    for (int j = max(0, issued - ST); j < issued; ++j) mbar_wait(b_qfull(j % ST), (j / ST) & 1, kWaitLimitNs);
-  }
-  tc_fence_after_sync();
-  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+  pair_teardown(ctl, b_done, tmem, status, K_ATTN_COLSUM);
 }
 
 // out[m] = sum over groups and the `merge` rows of token m of part[group][row].
@@ -531,17 +626,18 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// 2-D map over a row-major bf16 matrix [rows, cols]; box = 16 columns x 128 rows, 32-byte swizzle.
-pace_status_t make_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols) {
+// 2-D map over a row-major bf16 matrix [rows, cols]; box = 64 columns (128-byte swizzle) or
+// 16 columns (32-byte swizzle) x 128 rows.
+pace_status_t make_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, bool wide) {
   auto enc = tensor_map_encoder();
   if (enc == nullptr) return set_cuda_error(cudaErrorNotSupported);
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
   cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols * 2)};
-  cuuint32_t box[2] = {16, kTile};
+  cuuint32_t box[2] = {wide ? 64u : 16u, static_cast<cuuint32_t>(kTile)};
   cuuint32_t es[2] = {1, 1};
   CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, es,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_32B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, wide ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_32B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return PACE_ERR_INVALID_ARG;
   return PACE_OK;
 }
@@ -552,14 +648,14 @@ struct AttnLayout {
   size_t L_off, part_off, ml_off, total;
 };
 
-// Key splits of pass 1: enough items to cover the GPU about twice.
+// Key splits of pass 1: enough CTA pairs to cover the GPU about twice.
 int choose_splits(int B, const int32_t* cu_q, const int32_t* cu_k, int H) {
   int64_t items = 0;
   int max_kt = 1;
   for (int b = 0; b < B; ++b) {
     const int nq = cu_q[b + 1] - cu_q[b], nk = cu_k[b + 1] - cu_k[b];
-    items += static_cast<int64_t>(H) * ((nq + 2 * kTile - 1) / (2 * kTile));
-    max_kt = std::max(max_kt, (nk + kTile - 1) / kTile);
+    items += static_cast<int64_t>(H) * ((nq + kPair - 1) / kPair);
+    max_kt = std::max(max_kt, (nk + kPair - 1) / kPair);
   }
   if (items >= kTargetItems || items == 0) return 1;
   int s = static_cast<int>((kTargetItems + items - 1) / items);
@@ -573,8 +669,8 @@ AttnLayout attn_layout(int B, const int32_t* cu_q, const int32_t* cu_k, int H, i
   L.qtot = cu_q[B];
   L.ktot = cu_k[B];
   int64_t pr = 0;
-  for (int b = 0; b < B; ++b) pr += static_cast<int64_t>((cu_q[b + 1] - cu_q[b] + kTile - 1) / kTile) * kTile;
-  L.prows = pr;   // every image's L rows start on a 128-row (512-byte) boundary
+  for (int b = 0; b < B; ++b) pr += static_cast<int64_t>((cu_q[b + 1] - cu_q[b] + kPair - 1) / kPair) * kPair;
+  L.prows = pr;   // every image's L rows start on a 256-row (1 KB) boundary
   L.L_off = 0;
   L.part_off = align_up(static_cast<size_t>(H) * L.prows * sizeof(float), 256);
   L.ml_off = L.part_off + align_up(static_cast<size_t>(groups) * L.ktot * sizeof(float), 256);
@@ -597,8 +693,8 @@ pace_status_t check_segments(int B, const int32_t* cu, int multiple) {
 template <int D>
 pace_status_t set_smem_attrs(size_t* s1, size_t* s2) {
   using C = Cfg<D>;
-  *s1 = 1024 + 2 * C::TILE_BYTES + C::STAGES * C::TILE_BYTES + sizeof(SmemCtl);
-  *s2 = 1024 + 2 * C::TILE_BYTES + C::STAGES * C::TILE_BYTES + C::STAGES * kTile * 4 + sizeof(SmemCtl);
+  *s1 = 1024 + C::TILE_BYTES + C::STAGES * C::TILE_BYTES + sizeof(SmemCtl);
+  *s2 = 1024 + C::TILE_BYTES + C::STAGES * C::TILE_BYTES + C::STAGES * kPair * 4 + sizeof(SmemCtl);
   static std::atomic<uint64_t> done{0};
   int dev = 0;
   PACE_CUDA(cudaGetDevice(&dev));
@@ -608,6 +704,26 @@ pace_status_t set_smem_attrs(size_t* s1, size_t* s2) {
   PACE_CUDA(cudaFuncSetAttribute(attn_colsum<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(*s2)));
   done.fetch_or(bit, std::memory_order_acq_rel);
   return PACE_OK;
+}
+
+// Launches `items` CTA pairs (clusters of two CTAs along x).
+template <typename... Params, typename... Args>
+pace_status_t launch_pairs(void (*kernel)(Params...), int items, size_t smem, cudaStream_t stream, Args... args) {
+  if (items <= 0) return PACE_OK;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * static_cast<unsigned>(items));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  PACE_CUDA(cudaLaunchKernelEx(&cfg, kernel, args...));
+  return check_launch();
 }
 
 template <int D>
@@ -620,9 +736,12 @@ pace_status_t run_importance(const void* Q, const void* K, const int32_t* cu_q, 
   float* part = reinterpret_cast<float*>(w8 + Lay.part_off);
   float2* ml = Lay.splits > 1 ? reinterpret_cast<float2*>(w8 + Lay.ml_off) : nullptr;
   int* status = device_status_word();
-  CUtensorMap mq, mk;
-  PACE_CHECK(make_map(&mq, Q, std::max<int64_t>(Lay.qtot, 1), static_cast<int64_t>(Hq) * D));
-  PACE_CHECK(make_map(&mk, K, std::max<int64_t>(Lay.ktot, 1), static_cast<int64_t>(Hkv) * D));
+  CUtensorMap mq, mq32, mk, mk32;
+  const int64_t qrows = std::max<int64_t>(Lay.qtot, 1), krows = std::max<int64_t>(Lay.ktot, 1);
+  PACE_CHECK(make_map(&mq, Q, qrows, static_cast<int64_t>(Hq) * D, true));
+  PACE_CHECK(make_map(&mk, K, krows, static_cast<int64_t>(Hkv) * D, true));
+  PACE_CHECK(make_map(&mq32, Q, qrows, static_cast<int64_t>(Hq) * D, false));
+  PACE_CHECK(make_map(&mk32, K, krows, static_cast<int64_t>(Hkv) * D, false));
   size_t s1 = 0, s2 = 0;
   PACE_CHECK(set_smem_attrs<D>(&s1, &s2));
   const float c = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634);
@@ -645,24 +764,23 @@ pace_status_t run_importance(const void* Q, const void* K, const int32_t* cu_q, 
       t.k0[i] = cu_k[b];
       t.nk[i] = cu_k[b + 1] - cu_k[b];
       t.lpad[i] = lpad;
-      lpad += (t.nq[i] + kTile - 1) / kTile * kTile;
-      items1 += Hq * ((t.nq[i] + 2 * kTile - 1) / (2 * kTile)) * Lay.splits;
+      lpad += (t.nq[i] + kPair - 1) / kPair * kPair;
+      items1 += Hq * ((t.nq[i] + kPair - 1) / kPair) * Lay.splits;
       t.item_prefix[i + 1] = items1;
-      ctiles += (t.nq[i] + kTile - 1) / kTile;
+      ctiles += (t.nq[i] + kPair - 1) / kPair * 2;
     }
-    attn_row_lse<D><<<items1, kThreads, s1, stream>>>(mq, mk, t, c, Lw, ml, status);
-    PACE_CHECK(check_launch());
+    PACE_CHECK(launch_pairs(attn_row_lse<D>, items1, s1, stream, mq, mq32, mk, mk32, t, c, Lw, ml, status));
     if (Lay.splits > 1) {
       attn_lse_combine<<<dim3(ctiles, Hq), kTile, 0, stream>>>(t, ml, Lw);
       PACE_CHECK(check_launch());
     }
     int items2 = 0;
     for (int i = 0; i < nb; ++i) {
-      items2 += Hkv * ((t.nk[i] + 2 * kTile - 1) / (2 * kTile));
+      items2 += Hkv * ((t.nk[i] + kPair - 1) / kPair);
       t.item_prefix[i + 1] = items2;
     }
-    attn_colsum<D><<<items2, kThreads, s2, stream>>>(mq, mk, t, c, Lw, part, status);
-    PACE_CHECK(check_launch());
+    PACE_CHECK(launch_pairs(attn_colsum<D>, items2, s2, stream, mq, mq32, mk, mk32, t, c,
+                            static_cast<const float*>(Lw), part, status));
   }
   const int nout = static_cast<int>(Lay.ktot / merge);
   attn_reduce<<<(nout + 255) / 256, 256, 0, stream>>>(part, Hkv, static_cast<int>(Lay.ktot), merge, out);

@@ -5,7 +5,7 @@
 #include <cstdint>
 #include <cstddef>
 
-#include "../../include/pace.h"
+#include "pace.h"
 
 namespace pace {
 
