@@ -122,6 +122,22 @@ class ClockSampler:
                 "power_w_max": max(power) if power else None, "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def max_over_ranks(x: float, world: int, device) -> float:
+    """Maximum of a per-rank scalar over all ranks (the slowest rank sets the job time)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def per_image_us(total_ms: float, steps: int, world: int, images_per_step: int = 1) -> float:
+    """Whole-job time per image: every rank processes images_per_step images per step."""
+    return total_ms * 1e3 / (steps * world * images_per_step)
+
+
 # ----------------------------------------------------------------------------------------------
 # CPU oracle sample (the reference arm and the cpu_baseline leg)
 # ----------------------------------------------------------------------------------------------
@@ -206,92 +222,23 @@ def run_reference(args):
 # ----------------------------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------------------------
-class Pipeline:
-    """Device-resident inputs, outputs and workspaces of one step, and the step itself."""
-
-    def __init__(self, wl, keep, device):
-        import torch
-        from paper_2608_27206_gb300 import pace as P
-        from paper_2608_27206_gb300 import synth
-        self.P, self.torch, self.dev = P, torch, device
-        img = wl.images[0]
-        self.H, self.W = img.shape[:2]
-        buf, off = synth.pack_images(wl.images)
-        self.off = off
-        self.host = {
-            "img": torch.from_numpy(buf),
-            "vit_q": torch.from_numpy(wl.vit_q.view(np.int16)).view(torch.bfloat16),
-            "vit_k": torch.from_numpy(wl.vit_k.view(np.int16)).view(torch.bfloat16),
-            "llm_q": torch.from_numpy(wl.llm_q.view(np.int16)).view(torch.bfloat16),
-            "llm_k": torch.from_numpy(wl.llm_k.view(np.int16)).view(torch.bfloat16),
-            "embed": torch.from_numpy(wl.embed.view(np.int16)).view(torch.bfloat16),
-        }
-        self.d = {k: v.to(device) for k, v in self.host.items()}
-        self.cu = wl.cu_patches
-        self.cu_q, self.cu_v = wl.cu_q, wl.cu_vis
-        self.K = P.pace_budget(wl.n_vis[0], keep)
-        self.cu_keep = np.array([0, self.K], dtype=np.int32)
-        n, nv = wl.n_patches[0], wl.n_vis[0]
-        f32 = torch.float32
-        self.dist = torch.empty(n, dtype=f32, device=device)
-        self.stats = torch.zeros((1, 10), dtype=torch.int32, device=device)
-        self.resized = torch.empty(self.H * self.W * 3, dtype=torch.uint8, device=device)
-        self.s_vis = torch.empty(nv, dtype=f32, device=device)
-        self.s_llm = torch.empty(nv, dtype=f32, device=device)
-        self.s_final = torch.empty(nv, dtype=f32, device=device)
-        self.weights = torch.empty((1, 2), dtype=f32, device=device)
-        self.kept = torch.empty(self.K, dtype=torch.int32, device=device)
-        self.rows = torch.empty((self.K, self.d["embed"].shape[1]), dtype=torch.bfloat16, device=device)
-        u8 = torch.uint8
-        self.ws_d = torch.empty(P.pace_apc_density_workspace_size([self.H], [self.W]), dtype=u8, device=device)
-        self.ws_v = torch.empty(P.pace_vit_attn_importance_workspace_size(self.cu, 16), dtype=u8, device=device)
-        self.ws_l = torch.empty(P.pace_llm_text_visual_importance_workspace_size(self.cu_q, self.cu_v, 28, 4),
-                                dtype=u8, device=device)
-        self.parts = [("density", self.density), ("resample", self.resample), ("vit", self.vit),
-                      ("llm", self.llm), ("select", self.select), ("gather", self.gather)]
-
-    def density(self):
-        self.P.pace_apc_density(self.d["img"], self.off, [self.H], [self.W], d_out=self.dist, stats=self.stats,
-                                ws=self.ws_d)
-
-    def resample(self):
-        self.P.pace_apc_resample(self.d["img"], self.off, [self.H], [self.W], self.stats, self.resized, [0])
-
-    def vit(self):
-        self.P.pace_vit_attn_importance(self.d["vit_q"], self.d["vit_k"], self.cu, 1 / math.sqrt(80), 4,
-                                        out=self.s_vis, ws=self.ws_v)
-
-    def llm(self):
-        self.P.pace_llm_text_visual_importance(self.d["llm_q"], self.d["llm_k"], self.cu_q, self.cu_v,
-                                               1 / math.sqrt(128), out=self.s_llm, ws=self.ws_l)
-
-    def select(self):
-        self.P.pace_ddae_select(self.s_llm, self.s_vis, self.cu_v, self.cu_keep, s_final=self.s_final,
-                                weights=self.weights, kept=self.kept)
-
-    def gather(self):
-        self.P.pace_gather(self.d["embed"], self.kept, dst=self.rows)
-
-    def step(self):
-        for _, f in self.parts:
+def capture_graphs(pipe):
+    """One CUDA graph per libpace call of the step, captured after an eager warm-up."""
+    import torch
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        pipe.step()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    graphs = []
+    for name, f in pipe.parts:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
             f()
-
-    def capture(self):
-        """One CUDA graph per call, captured after an eager warm-up."""
-        torch = self.torch
-        self.graphs = []
-        s = torch.cuda.Stream()
-        s.wait_stream(torch.cuda.current_stream())
-        with torch.cuda.stream(s):
-            self.step()
-        torch.cuda.current_stream().wait_stream(s)
-        torch.cuda.synchronize()
-        for name, f in self.parts:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                f()
-            self.graphs.append((name, g))
-        torch.cuda.synchronize()
+        graphs.append((name, g))
+    torch.cuda.synchronize()
+    return graphs
 
 
 def algorithmic_counts(wl, keep, r_ratio):
@@ -332,8 +279,9 @@ def run_gpu(args):
     from paper_2608_27206_gb300 import synth
     P.pace_init(torch.cuda.current_device())
 
+    from paper_2608_27206_gb300.hotpath import HotPath
     wl = synth.make_workload(WORKLOAD, seed=rank, keep=KEEP)
-    pipe = Pipeline(wl, KEEP, device)
+    pipe = HotPath(wl, device)
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=device)
 
     # launches per step (eager), then graphs
@@ -341,17 +289,17 @@ def run_gpu(args):
     pipe.step()
     torch.cuda.synchronize()
     launches_per_step = P.pace_kernel_launch_count() - c0
-    pipe.capture()
+    graphs = capture_graphs(pipe)
     for _ in range(args.warmup):
         flush.zero_()
-        for _, g in pipe.graphs:
+        for _, g in graphs:
             g.replay()
     torch.cuda.synchronize()
     code, where = P.pace_device_status(clear=True)
     if code != 0:
         raise RuntimeError(f"device status {code} from kernel {where} during warm-up")
 
-    nparts = len(pipe.graphs)
+    nparts = len(graphs)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nparts + 1)] for _ in range(args.steps)]
     sampler = ClockSampler(torch.cuda.current_device())
     sampler.start()
@@ -362,7 +310,7 @@ def run_gpu(args):
     for k in range(args.steps):
         flush.zero_()
         ev[k][0].record()
-        for i, (_, g) in enumerate(pipe.graphs):
+        for i, (_, g) in enumerate(graphs):
             g.replay()
             ev[k][i + 1].record()
     torch.cuda.synchronize()
@@ -370,19 +318,15 @@ def run_gpu(args):
         dist.barrier()
     t_wall = time.perf_counter() - t_wall0
     clocks = sampler.stop()
-    part_ms = {name: [] for name, _ in pipe.graphs}
+    part_ms = {name: [] for name, _ in graphs}
     step_ms = []
     for k in range(args.steps):
         step_ms.append(ev[k][0].elapsed_time(ev[k][nparts]))
-        for i, (name, _) in enumerate(pipe.graphs):
+        for i, (name, _) in enumerate(graphs):
             part_ms[name].append(ev[k][i].elapsed_time(ev[k][i + 1]))
-    total_ms = float(sum(step_ms))
-    if world > 1:
-        tt = torch.tensor([total_ms], dtype=torch.float64, device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = max_over_ranks(float(sum(step_ms)), world, device)
     ms_per_step = total_ms / args.steps
-    value = total_ms * 1e3 / (args.steps * world)       # us per image over all ranks
+    value = per_image_us(total_ms, args.steps, world)
 
     # correctness guard on the timed outputs
     code, where = P.pace_device_status(clear=True)
@@ -392,7 +336,7 @@ def run_gpu(args):
 
     # e2e: pinned host inputs -> device, the public calls, results -> pinned host
     pinned = {k: v.pin_memory() for k, v in pipe.host.items()}
-    out_host = {"kept": torch.empty(pipe.K, dtype=torch.int32).pin_memory(),
+    out_host = {"kept": torch.empty(tuple(pipe.kept.shape), dtype=torch.int32).pin_memory(),
                 "rows": torch.empty(tuple(pipe.rows.shape), dtype=torch.bfloat16).pin_memory(),
                 "stats": torch.empty((1, 10), dtype=torch.int32).pin_memory(),
                 "s_final": torch.empty(pipe.s_final.numel(), dtype=torch.float32).pin_memory()}
@@ -420,13 +364,10 @@ def run_gpu(args):
         e2e_step()
     e_end.record()
     torch.cuda.synchronize()
-    e2e_ms = e_start.elapsed_time(e_end)
+    e2e_ms = max_over_ranks(e_start.elapsed_time(e_end), world, device)
     if world > 1:
-        tt = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
         dist.barrier()
-    e2e_value = e2e_ms * 1e3 / (args.steps * world)
+    e2e_value = per_image_us(e2e_ms, args.steps, world)
 
     if rank == 0:
         peaks, peak_src = load_peaks()
@@ -489,7 +430,8 @@ def run_profile(args):
     from paper_2608_27206_gb300 import synth
     P.pace_init(0)
     wl = synth.make_workload(args.workload, seed=0, keep=KEEP)
-    pipe = Pipeline(wl, KEEP, torch.device("cuda", 0))
+    from paper_2608_27206_gb300.hotpath import HotPath
+    pipe = HotPath(wl, torch.device("cuda", 0))
     fns = dict(pipe.parts)
     needs = {"resample": ["density"], "select": ["vit", "llm"], "gather": ["vit", "llm", "select"]}
     for name in needs.get(args.profile, []):      # producers of this call's inputs

@@ -65,6 +65,12 @@ PACE_API pace_status_t pace_init(int device);
  * (0 if none).  With clear != 0 the word is reset to PACE_OK afterwards. */
 PACE_API pace_status_t pace_device_status(int* code, int* where, int clear);
 
+/* Exercises the bounded-wait path: launches one CTA that waits on a barrier nothing ever
+ * arrives at.  After limit_us microseconds (1 .. 1000000) the wait gives up, the kernel
+ * records PACE_ERR_TIMEOUT (kernel id 11) in the device status word and returns; the CUDA
+ * context stays usable.  For failure-detection tests of callers. */
+PACE_API pace_status_t pace_selftest_wait_timeout(uint32_t limit_us, pace_stream_t stream);
+
 /* Number of CUDA kernels this library has launched in the calling process (all threads,
  * all devices).  Instrumentation for benchmarks: counts launches, not completed work. */
 PACE_API uint64_t pace_kernel_launch_count(void);

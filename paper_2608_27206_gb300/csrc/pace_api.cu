@@ -5,6 +5,7 @@
 #include <mutex>
 
 #include "pace_common.cuh"
+#include "pace_ptx.cuh"
 
 namespace pace {
 
@@ -75,6 +76,19 @@ pace_status_t check_launch() {
   return PACE_OK;
 }
 
+// One CTA waits on an mbarrier that nothing ever arrives at: the bounded wait must give up
+// after limit_ns and record PACE_ERR_TIMEOUT, leaving the context usable.
+__global__ void selftest_wait_kernel(uint64_t limit_ns, int* status) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(ptx::smem_u32(&bar), 1);
+    ptx::fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !ptx::mbar_wait(ptx::smem_u32(&bar), 0, limit_ns))
+    record_error(status, PACE_ERR_TIMEOUT, K_SELFTEST);
+}
+
 }  // namespace pace
 
 extern "C" {
@@ -111,6 +125,14 @@ pace_status_t pace_device_status(int* code, int* where, int clear) {
   if (where) *where = h[1];
   if (clear) PACE_CUDA(cudaMemset(w, 0, sizeof(h)));
   return PACE_OK;
+}
+
+pace_status_t pace_selftest_wait_timeout(uint32_t limit_us, pace_stream_t stream) {
+  if (limit_us == 0 || limit_us > 1000000u) return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(pace::check_device());
+  pace::selftest_wait_kernel<<<1, 32, 0, stream>>>(static_cast<uint64_t>(limit_us) * 1000ull,
+                                                   pace::device_status_word());
+  return pace::check_launch();
 }
 
 int32_t pace_budget(int32_t n_vis, double frac) {

@@ -21,6 +21,7 @@ enum KernelId : int {
   K_ATTN_REDUCE = 8,
   K_DDAE_SELECT = 9,
   K_GATHER = 10,
+  K_SELFTEST = 11,
 };
 
 // Device status word layout: [0] = code (pace_status_t), [1] = kernel id.

@@ -1,0 +1,105 @@
+"""One step of the condense-and-extract hot path over a batch of images, on the device.
+
+HotPath owns the device copies of a workload's inputs, the outputs and the scratch
+buffers, and issues the six libpace calls in pipeline order:
+
+    density -> resample (target size read on the device) -> ViT importance ->
+    LLM importance -> DDAE fusion + top-K -> gather of the kept embedding rows
+
+Everything is allocated once in the constructor, so a step only launches kernels and
+can be captured in a CUDA graph.  Used by bench.py and by the full-size parity tests,
+so both exercise exactly the same calls.
+"""
+from __future__ import annotations
+
+import math
+from typing import Optional, Sequence
+
+import numpy as np
+import torch
+
+from . import pace as P
+from . import synth
+
+
+def _bf16(bits: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16)
+
+
+class HotPath:
+    def __init__(self, wl: "synth.Workload", device, keep: Optional[Sequence[float]] = None):
+        self.wl = wl
+        self.dev = torch.device(device)
+        self.B = wl.B
+        self.H = [im.shape[0] for im in wl.images]
+        self.W = [im.shape[1] for im in wl.images]
+        buf, off = synth.pack_images(wl.images)
+        self.img_off = off
+        self.host = {
+            "img": torch.from_numpy(buf),
+            "vit_q": _bf16(wl.vit_q), "vit_k": _bf16(wl.vit_k),
+            "llm_q": _bf16(wl.llm_q), "llm_k": _bf16(wl.llm_k),
+            "embed": _bf16(wl.embed),
+        }
+        self.d = {k: v.to(self.dev) for k, v in self.host.items()}
+        self.cu_patches, self.cu_q, self.cu_vis = wl.cu_patches, wl.cu_q, wl.cu_vis
+        fracs = list(keep) if keep is not None else wl.keep_fracs
+        self.K = [P.pace_budget(n, f) for n, f in zip(wl.n_vis, fracs)]
+        self.cu_keep = np.concatenate([[0], np.cumsum(self.K)]).astype(np.int32)
+        sizes = [h * w * 3 for h, w in zip(self.H, self.W)]
+        self.dst_off = np.concatenate([[0], np.cumsum([(s + 255) // 256 * 256 for s in sizes])])[:-1].astype(np.int64)
+        f32, i32, u8 = torch.float32, torch.int32, torch.uint8
+        n, nv = int(self.cu_patches[-1]), int(self.cu_vis[-1])
+        dev = self.dev
+        self.dist = torch.empty(max(n, 1), dtype=f32, device=dev)
+        self.stats = torch.zeros((max(self.B, 1), 10), dtype=i32, device=dev)
+        self.resized = torch.zeros(int(self.dst_off[-1] + sizes[-1]) if self.B else 1, dtype=u8, device=dev)
+        self.s_vis = torch.empty(max(nv, 1), dtype=f32, device=dev)
+        self.s_llm = torch.empty(max(nv, 1), dtype=f32, device=dev)
+        self.s_final = torch.empty(max(nv, 1), dtype=f32, device=dev)
+        self.weights = torch.empty((max(self.B, 1), 2), dtype=f32, device=dev)
+        k_tot = int(self.cu_keep[-1])
+        self.kept = torch.empty(max(k_tot, 1), dtype=i32, device=dev)
+        self.rows = torch.empty((max(k_tot, 1), self.d["embed"].shape[1]), dtype=torch.bfloat16, device=dev)
+        self.ws_density = torch.empty(max(P.pace_apc_density_workspace_size(self.H, self.W), 16), dtype=u8,
+                                      device=dev)
+        self.ws_vit = torch.empty(max(P.pace_vit_attn_importance_workspace_size(self.cu_patches, synth.VIT_HEADS),
+                                      16), dtype=u8, device=dev)
+        self.ws_llm = torch.empty(max(P.pace_llm_text_visual_importance_workspace_size(
+            self.cu_q, self.cu_vis, synth.LLM_QHEADS, synth.LLM_KVHEADS), 16), dtype=u8, device=dev)
+        self.parts = [("density", self.density), ("resample", self.resample), ("vit", self.vit),
+                      ("llm", self.llm), ("select", self.select), ("gather", self.gather)]
+
+    # -- the six calls ---------------------------------------------------------------------------
+    def density(self):
+        P.pace_apc_density(self.d["img"], self.img_off, self.H, self.W, d_out=self.dist, stats=self.stats,
+                           ws=self.ws_density)
+
+    def resample(self):
+        P.pace_apc_resample(self.d["img"], self.img_off, self.H, self.W, self.stats, self.resized, self.dst_off)
+
+    def vit(self):
+        P.pace_vit_attn_importance(self.d["vit_q"], self.d["vit_k"], self.cu_patches,
+                                   1.0 / math.sqrt(synth.VIT_DIM), 4, out=self.s_vis, ws=self.ws_vit)
+
+    def llm(self):
+        P.pace_llm_text_visual_importance(self.d["llm_q"], self.d["llm_k"], self.cu_q, self.cu_vis,
+                                          1.0 / math.sqrt(synth.LLM_DIM), out=self.s_llm, ws=self.ws_llm)
+
+    def select(self):
+        P.pace_ddae_select(self.s_llm, self.s_vis, self.cu_vis, self.cu_keep, s_final=self.s_final,
+                           weights=self.weights, kept=self.kept)
+
+    def gather(self):
+        P.pace_gather(self.d["embed"], self.kept[: int(self.cu_keep[-1])], dst=self.rows)
+
+    def step(self):
+        for _, f in self.parts:
+            f()
+
+    # -- results on the host ---------------------------------------------------------------------
+    def resized_images(self):
+        st = P.stats_dict(self.stats[: self.B])
+        flat = self.resized.cpu().numpy()
+        return [flat[o:o + s["h_out"] * s["w_out"] * 3].reshape(s["h_out"], s["w_out"], 3)
+                for o, s in zip(self.dst_off, st)]

@@ -46,6 +46,7 @@ _SIGS = {
     "pace_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "pace_last_cuda_error": (ctypes.c_int, []),
     "pace_kernel_launch_count": (ctypes.c_uint64, []),
+    "pace_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_uint32, _P]),
     "pace_init": (ctypes.c_int, [ctypes.c_int]),
     "pace_device_status": (ctypes.c_int, [_I32P, _I32P, ctypes.c_int]),
     "pace_apc_params_default": (None, [ctypes.POINTER(ApcParams)]),
@@ -152,6 +153,11 @@ def pace_device_status(clear: bool = True):
     code, where = ctypes.c_int32(0), ctypes.c_int32(0)
     _check("pace_device_status", lib().pace_device_status(ctypes.byref(code), ctypes.byref(where), int(clear)))
     return code.value, where.value
+
+
+def pace_selftest_wait_timeout(limit_us: int, stream=None) -> None:
+    """Launches a kernel whose bounded wait must run out and report PACE_ERR_TIMEOUT."""
+    _check("pace_selftest_wait_timeout", lib().pace_selftest_wait_timeout(int(limit_us), _stream(stream)))
 
 
 def pace_kernel_launch_count() -> int:
