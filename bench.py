@@ -21,9 +21,11 @@ back inside the timed region.  Under torchrun every rank processes its own image
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -54,6 +56,23 @@ def load_peaks():
         return p, "measured"
     except (OSError, ValueError):
         return dict(FALLBACK_PEAKS), "fallback"
+
+
+def profiled_traffic():
+    """DRAM bytes per ViT-importance call from the committed ncu summary, or None when the
+    kernel source has changed since those counters were taken."""
+    path = os.path.join(ROOT, "profiles", "vit_importance_img4k.md")
+    src = os.path.join(ROOT, "paper_2608_27206_gb300", "csrc", "attn.cu")
+    try:
+        text = open(path).read()
+        t = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
+        h = re.search(r"sha256\[:16\]\s*([0-9a-f]{16})", text)
+        cur = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if t and h and h.group(1) == cur:
+            return int(t.group(1))
+    except OSError:
+        pass
+    return None
 
 
 def workload_config(wl, keep):
@@ -397,7 +416,8 @@ def run_gpu(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": workload_config(wl, KEEP),
             "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
-                         "frac": round(achieved / peak, 4), "traffic": None,
+                         "frac": round(achieved / peak, 4), "traffic": profiled_traffic(),
+                         "traffic_unit": "bytes per call (ncu dram read+write, profiles/vit_importance_img4k.md)",
                          "kernel": "ViT received attention (attn_row_lse + attn_colsum + attn_reduce), one launch "
                                    "of pace_vit_attn_importance",
                          "algorithmic_flops": cnt["vit_flops"], "us": round(vit_ms * 1e3, 1),
