@@ -13,13 +13,17 @@
 //              the staged pixels (no 2 - 2cos cancellation).
 //   apc_tail   one CTA per image: radix select of the k_tail-th largest d_i (fp32 bits),
 //              tail mean, rho_d, rho, r and the target size.
-// Resize: apc_resample, one CTA per 8 x 32 output tile; input rows are filtered
-// horizontally 8 at a time into shared memory and accumulated vertically in registers.
+// Resize: apc_resample, one CTA per 32 x 64 output tile; for downscales up to 2.75x per side
+// the input window is staged in shared memory and filtered there with precomputed weights,
+// steeper downscales take a generic path with per-tap weights.
+#include <algorithm>
+#include <atomic>
 #include <cfloat>
 #include <cmath>
 #include <mutex>
 
 #include "pace_common.cuh"
+#include "pace_select.cuh"
 
 namespace pace {
 namespace {
@@ -76,15 +80,32 @@ __device__ __forceinline__ void load_strip(const uint8_t* __restrict__ img, int 
   }
 }
 
-__device__ __forceinline__ int warp_sum_int(int v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
 __device__ __forceinline__ float warp_sum_f(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
+}
+
+// Exact uint8 -> float without the conversion pipe: 2^23 + v has v in its low mantissa bits.
+__device__ __forceinline__ float byte_to_float(uint32_t v) { return __uint_as_float(0x4B000000u | v) - 8388608.0f; }
+
+// Sum of squares of the 42 bytes at s (2-byte aligned): 4-byte words with dp4a, the unaligned
+// ends as 16-bit loads.
+__device__ __forceinline__ uint32_t row_sumsq42(const uint8_t* s) {
+  uint32_t acc = 0u;
+  const int lead = (reinterpret_cast<uintptr_t>(s) & 3u) ? 1 : 0;   // one 16-bit head to reach 4-byte alignment
+  if (lead) {
+    const uint32_t h = *reinterpret_cast<const uint16_t*>(s);
+    acc = __dp4a(h, h, acc);
+  }
+  const uint32_t* w = reinterpret_cast<const uint32_t*>(s + 2 * lead);
+#pragma unroll
+  for (int i = 0; i < 10; ++i) acc = __dp4a(w[i], w[i], acc);
+  if (!lead) {
+    const uint32_t h = *reinterpret_cast<const uint16_t*>(s + 40);
+    acc = __dp4a(h, h, acc);
+  }
+  return acc;
 }
 
 template <bool WIDE>
@@ -93,6 +114,7 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restri
                                                          float* __restrict__ inv_norm,
                                                          unsigned long long* __restrict__ sums) {
   __shared__ __align__(16) uint8_t s[kPatch * kStripRowBytes];
+  __shared__ uint32_t ssq[8][kStrip];
   __shared__ float inv[kStrip];
   const int unit = blockIdx.x;
   const int b = find_image(t, unit);
@@ -102,36 +124,48 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restri
   const int np = min(kStrip, t.gw[b] - px0);
   load_strip<WIDE>(img + t.off[b], t.W[b], py, px0, np, s);
   __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int p = warp; p < np; p += kApcThreads / 32) {
-    int ss = 0;
-    for (int i = lane; i < kPatchBytes; i += 32) {
-      const int y = i / 42, k = i - y * 42;
-      const int v = s[y * kStripRowBytes + p * 42 + k];
-      ss += v * v;
+  // |x|^2 of every patch: thread (p = tid % 32, rows yg and yg + 8)
+  {
+    const int p = threadIdx.x & 31, yg = threadIdx.x >> 5;
+    uint32_t a = 0u;
+    if (p < np) {
+      a = row_sumsq42(s + yg * kStripRowBytes + p * 42);
+      if (yg + 8 < kPatch) a += row_sumsq42(s + (yg + 8) * kStripRowBytes + p * 42);
     }
-    ss = warp_sum_int(ss);
-    if (lane == 0) {
-      const float n2 = static_cast<float>(ss) * (1.0f / 65025.0f) + 1.0f;
-      const float iv = 1.0f / sqrtf(n2);
-      inv[p] = iv;
-      inv_norm[t.patch0[b] + py * t.gw[b] + px0 + p] = iv;
-    }
+    ssq[yg][p] = a;
   }
   __syncthreads();
+  if (threadIdx.x < np) {
+    const int p = threadIdx.x;
+    uint32_t ss = 0u;
+#pragma unroll
+    for (int g = 0; g < 8; ++g) ss += ssq[g][p];
+    const float n2 = static_cast<float>(ss) * (1.0f / 65025.0f) + 1.0f;
+    const float iv = 1.0f / sqrtf(n2);
+    inv[p] = iv;
+    inv_norm[t.patch0[b] + py * t.gw[b] + px0 + p] = iv;
+  }
+  __syncthreads();
+  // weighted column sums: thread j owns columns 2j, 2j+1 (a pair never crosses a 42-byte row)
   unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * kTokDim;
-  for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) {
-    float acc = 0.f;
-    if (k < kPatchBytes) {
-      const int y = k / 42, kk = k - y * 42;
-      const uint8_t* col = s + y * kStripRowBytes + kk;
-      for (int p = 0; p < np; ++p) acc = fmaf(inv[p], static_cast<float>(col[p * 42]), acc);
-      acc *= (1.0f / 255.0f);
+  for (int j = threadIdx.x; j < kPatchBytes / 2 + 1; j += kApcThreads) {
+    if (j < kPatchBytes / 2) {
+      const int k = 2 * j, y = k / 42, kk = k - y * 42;
+      const uint16_t* col = reinterpret_cast<const uint16_t*>(s + y * kStripRowBytes + kk);
+      float a0 = 0.f, a1 = 0.f;
+      for (int p = 0; p < np; ++p) {
+        const uint32_t v = col[p * 21];
+        a0 = fmaf(inv[p], byte_to_float(v & 255u), a0);
+        a1 = fmaf(inv[p], byte_to_float(v >> 8), a1);
+      }
+      atomicAdd(sb + k, static_cast<unsigned long long>(llrint(static_cast<double>(a0 * (1.0f / 255.0f)) * kFix)));
+      atomicAdd(sb + k + 1,
+                static_cast<unsigned long long>(llrint(static_cast<double>(a1 * (1.0f / 255.0f)) * kFix)));
     } else {
-      for (int p = 0; p < np; ++p) acc += inv[p];
+      float a = 0.f;
+      for (int p = 0; p < np; ++p) a += inv[p];
+      atomicAdd(sb + kPatchBytes, static_cast<unsigned long long>(llrint(static_cast<double>(a) * kFix)));
     }
-    const unsigned long long q = static_cast<unsigned long long>(llrint(static_cast<double>(acc) * kFix));
-    atomicAdd(sb + k, q);
   }
 }
 
@@ -143,7 +177,7 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
                                                          float* __restrict__ d_out,
                                                          pace_apc_stats* __restrict__ stats) {
   __shared__ __align__(16) uint8_t s[kPatch * kStripRowBytes];
-  __shared__ float chat[kTokDim + 3];
+  __shared__ __align__(8) float chat[kTokDim + 3];
   __shared__ float red[kApcThreads / 32];
   const int unit = blockIdx.x;
   const int b = find_image(t, unit);
@@ -178,17 +212,23 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
     stats[t.b_base + b].k_tail = t.ktail[b];
   }
   __syncthreads();
+  // d_i = |t_i - c_hat| computed directly: warp per patch, lanes over column pairs
   const float* pinv = inv_norm + t.patch0[b] + py * t.gw[b] + px0;
+  const float2* chat2 = reinterpret_cast<const float2*>(chat);
   for (int p = warp; p < np; p += kApcThreads / 32) {
     const float iv = pinv[p];
     const float sc = iv * (1.0f / 255.0f);
-    float acc = 0.f;
-    for (int i = lane; i < kPatchBytes; i += 32) {
-      const int y = i / 42, k = i - y * 42;
-      const float v = fmaf(static_cast<float>(s[y * kStripRowBytes + p * 42 + k]), sc, -chat[i]);
-      acc = fmaf(v, v, acc);
+    float acc0 = 0.f, acc1 = 0.f;
+    for (int j = lane; j < kPatchBytes / 2; j += 32) {
+      const int k = 2 * j, y = k / 42, kk = k - y * 42;
+      const uint32_t v = *reinterpret_cast<const uint16_t*>(s + y * kStripRowBytes + p * 42 + kk);
+      const float2 ch = chat2[j];
+      const float e0 = fmaf(byte_to_float(v & 255u), sc, -ch.x);
+      const float e1 = fmaf(byte_to_float(v >> 8), sc, -ch.y);
+      acc0 = fmaf(e0, e0, acc0);
+      acc1 = fmaf(e1, e1, acc1);
     }
-    acc = warp_sum_f(acc);
+    float acc = warp_sum_f(acc0 + acc1);
     if (lane == 0) {
       const float v = iv - chat[kPatchBytes];
       d_out[t.patch0[b] + py * t.gw[b] + px0 + p] = sqrtf(fmaf(v, v, acc));
@@ -201,8 +241,11 @@ struct TailParams {
   int align;
 };
 
+constexpr int kTailSmemMax = 48 * 1024;   // d values staged in shared memory (floats)
+
 __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTable t, const float* __restrict__ d,
                                                  TailParams prm, pace_apc_stats* __restrict__ stats) {
+  extern __shared__ float sd[];
   __shared__ unsigned hist[256];
   __shared__ unsigned sel[2];
   __shared__ float red[32];
@@ -210,26 +253,28 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
   const int b = blockIdx.x;
   const int N = (t.H[b] / kPatch) * t.gw[b];
   const float* db = d + t.patch0[b];
+  if (N <= kTailSmemMax) {   // one coalesced read of the distances, then work from shared memory
+    for (int i = threadIdx.x; i < N; i += blockDim.x) sd[i] = db[i];
+    __syncthreads();
+    db = sd;
+  }
   const unsigned k = static_cast<unsigned>(t.ktail[b]);
   unsigned prefix = 0u, mask = 0u, remaining = k;
+  const int lane_id = threadIdx.x & 31;
   for (int shift = 24; shift >= 0; shift -= 8) {
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0u;
     __syncthreads();
-    for (int i = threadIdx.x; i < N; i += blockDim.x) {
-      const unsigned key = __float_as_uint(db[i]);
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    // lanes holding the same digit are combined before the shared atomic
+    for (int base = 0; base < N; base += blockDim.x) {
+      const int i = base + threadIdx.x;
+      const unsigned key = i < N ? __float_as_uint(db[i]) : 0u;
+      const bool in = i < N && (key & mask) == prefix;
+      const unsigned digit = in ? ((key >> shift) & 255u) : 256u;
+      const unsigned peers = __match_any_sync(0xffffffffu, digit);
+      if (in && lane_id == __ffs(peers) - 1) atomicAdd(&hist[digit], static_cast<unsigned>(__popc(peers)));
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned above = 0u;
-      int dg = 255;
-      for (; dg > 0; --dg) {
-        if (above + hist[dg] >= remaining) break;
-        above += hist[dg];
-      }
-      sel[0] = static_cast<unsigned>(dg);
-      sel[1] = above;
-    }
+    if (threadIdx.x < 32) warp_digit_search(hist, remaining, sel);
     __syncthreads();
     prefix |= sel[0] << shift;
     mask |= 255u << shift;
@@ -330,21 +375,15 @@ __device__ __forceinline__ void window_1d(int o, int n_in, int n_out, int& lo, i
   inorm = 1.0f / s;
 }
 
-__global__ void __launch_bounds__(256) apc_resample(const uint8_t* __restrict__ src,
-                                                    const __grid_constant__ ResampleTable t,
-                                                    const pace_apc_stats* __restrict__ stats,
-                                                    uint8_t* __restrict__ dst) {
+// Any downscale: one 8 x 32 output tile, weights evaluated per tap, input read through L1.
+__device__ void resample_tile_generic(const uint8_t* __restrict__ img, int H, int W, int Ho, int Wo, int ox0,
+                                      int oy0, uint8_t* __restrict__ out) {
   __shared__ int xlo[kRsTW], xn[kRsTW];
   __shared__ float xoff[kRsTW], xifs[kRsTW], xnorm[kRsTW];
   __shared__ int ylo[kRsTH], yn[kRsTH];
   __shared__ float yoff[kRsTH], yifs[kRsTH], ynorm[kRsTH];
   __shared__ float hbuf[kRsChunk][kRsTW][3];
-  const int b = blockIdx.z;
-  const int H = t.H[b], W = t.W[b];
-  const int Ho = stats ? stats[t.b_base + b].h_out : t.Ho[b];
-  const int Wo = stats ? stats[t.b_base + b].w_out : t.Wo[b];
-  const int ox0 = blockIdx.x * kRsTW, oy0 = blockIdx.y * kRsTH;
-  if (ox0 >= Wo || oy0 >= Ho || Ho < 1 || Wo < 1 || Ho > H || Wo > W) return;
+  if (ox0 >= Wo || oy0 >= Ho) return;
   const int tid = threadIdx.x;
   if (tid < kRsTW) {
     const int ox = min(ox0 + tid, Wo - 1);
@@ -358,7 +397,6 @@ __global__ void __launch_bounds__(256) apc_resample(const uint8_t* __restrict__ 
   const int nrows = min(kRsTH, Ho - oy0);
   const int iy_lo = ylo[0];
   const int iy_hi = ylo[nrows - 1] + yn[nrows - 1];  // exclusive
-  const uint8_t* img = src + t.src_off[b];
   const int64_t pitch = static_cast<int64_t>(W) * 3;
   // this thread's output pixel
   const int my_r = tid / kRsTW, my_c = tid % kRsTW;
@@ -399,10 +437,125 @@ __global__ void __launch_bounds__(256) apc_resample(const uint8_t* __restrict__ 
   const int oy = oy0 + my_r, ox = ox0 + my_c;
   if (my_r < nrows && ox < Wo) {
     const float nrm = ynorm[my_r];
-    uint8_t* o = dst + t.dst_off[b] + (static_cast<int64_t>(oy) * Wo + ox) * 3;
+    uint8_t* o = out + (static_cast<int64_t>(oy) * Wo + ox) * 3;
     o[0] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc0 * nrm))));
     o[1] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc1 * nrm))));
     o[2] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc2 * nrm))));
+  }
+  __syncthreads();   // shared tile buffers are reused by the next call
+}
+
+// Downscale of at most kFMaxScale per side: one 32 x 64 output tile.  The CTA stages its whole
+// input window in shared memory with 4-byte loads (every image starts 16-byte aligned and
+// holds a multiple of 4 bytes, so the rounded loads stay inside it), precomputes the
+// normalised tap weights of its rows and columns once, then runs the horizontal pass into a
+// shared fp32 buffer and the vertical pass from there.
+constexpr int kFTH = 32, kFTW = 64, kFMaxTaps = 14;
+constexpr double kFMaxScale = 2.75;
+constexpr int kFRows = 102;                  // >= 32 * 2.75 + 14 staged input rows
+constexpr int kFCols = 190;                  // >= 64 * 2.75 + 14 staged input pixels per row
+constexpr int kFPitch = 576;                 // bytes per staged row: 3 * kFCols + 3 alignment slack, rounded
+static_assert(kFPitch >= 3 * kFCols + 6, "staged row pitch");
+static_assert(kFRows >= 32 * 2.75 + 14 && kFCols >= 64 * 2.75 + 14, "staged window");
+constexpr size_t kFSmem = static_cast<size_t>(kFRows) * kFPitch + static_cast<size_t>(kFRows) * kFTW * 3 * 4 +
+                          (kFTW + kFTH) * kFMaxTaps * 4 + (2 * kFTW + 2 * kFTH + kFRows + 4) * 4;
+
+// Normalised weights of the window of output index o (reading R5); returns the tap count.
+__device__ __forceinline__ int window_weights(int o, int n_in, int n_out, int& lo, float* w) {
+  const double scale = static_cast<double>(n_in) / n_out;
+  const double fs = scale > 1.0 ? scale : 1.0;
+  const double centre = (o + 0.5) * scale;
+  int a = static_cast<int>(floor(centre - 2.0 * fs));
+  int e = static_cast<int>(ceil(centre + 2.0 * fs));
+  if (a < 0) a = 0;
+  if (e > n_in) e = n_in;
+  const int n = e - a;
+  if (n > kFMaxTaps) return n;
+  const float off0 = static_cast<float>((a + 0.5 - centre) / fs), ifs = static_cast<float>(1.0 / fs);
+  float sum = 0.f;
+  for (int i = 0; i < n; ++i) {
+    w[i] = cubic_w(fmaf(static_cast<float>(i), ifs, off0));
+    sum += w[i];
+  }
+  const float inv = 1.0f / sum;
+  for (int i = 0; i < n; ++i) w[i] *= inv;
+  lo = a;
+  return n;
+}
+
+__global__ void __launch_bounds__(256) apc_resample(const uint8_t* __restrict__ src,
+                                                    const __grid_constant__ ResampleTable t,
+                                                    const pace_apc_stats* __restrict__ stats,
+                                                    uint8_t* __restrict__ dst) {
+  extern __shared__ __align__(16) unsigned char rs_smem[];
+  const int b = blockIdx.z;
+  const int H = t.H[b], W = t.W[b];
+  const int Ho = stats ? stats[t.b_base + b].h_out : t.Ho[b];
+  const int Wo = stats ? stats[t.b_base + b].w_out : t.Wo[b];
+  const int ox0 = blockIdx.x * kFTW, oy0 = blockIdx.y * kFTH;
+  if (ox0 >= Wo || oy0 >= Ho || Ho < 1 || Wo < 1 || Ho > H || Wo > W) return;
+  const uint8_t* img = src + t.src_off[b];
+  uint8_t* out = dst + t.dst_off[b];
+  const int tid = threadIdx.x;
+  const bool fast = static_cast<double>(W) / Wo <= kFMaxScale && static_cast<double>(H) / Ho <= kFMaxScale;
+  if (!fast) {
+    for (int sy = 0; sy < kFTH; sy += kRsTH)
+      for (int sx = 0; sx < kFTW; sx += kRsTW) resample_tile_generic(img, H, W, Ho, Wo, ox0 + sx, oy0 + sy, out);
+    return;
+  }
+  unsigned char* sin = rs_smem;                                           // [kFRows][kFPitch] bytes
+  float* sh = reinterpret_cast<float*>(sin + kFRows * kFPitch);            // [kFRows][kFTW][3]
+  float* wx = sh + kFRows * kFTW * 3;                                     // [kFTW][kFMaxTaps]
+  float* wy = wx + kFTW * kFMaxTaps;                                       // [kFTH][kFMaxTaps]
+  int* xlo = reinterpret_cast<int*>(wy + kFTH * kFMaxTaps);
+  int* xn = xlo + kFTW;
+  int* ylo = xn + kFTW;
+  int* yn = ylo + kFTH;
+  int* shift = yn + kFTH;                                                  // [kFRows]
+  const int ncol = min(kFTW, Wo - ox0), nrow = min(kFTH, Ho - oy0);
+  // with both scales <= kFMaxScale every window has <= 4 * 2.75 + 2 = 13 taps (min() is a guard)
+  if (tid < ncol) xn[tid] = min(kFMaxTaps, window_weights(ox0 + tid, W, Wo, xlo[tid], wx + tid * kFMaxTaps));
+  if (tid >= 64 && tid < 64 + nrow)
+    yn[tid - 64] =
+        min(kFMaxTaps, window_weights(oy0 + tid - 64, H, Ho, ylo[tid - 64], wy + (tid - 64) * kFMaxTaps));
+  __syncthreads();
+  const int x0 = xlo[0], x1 = xlo[ncol - 1] + xn[ncol - 1];
+  const int y0 = ylo[0], y1 = ylo[nrow - 1] + yn[nrow - 1];
+  const int nin_c = x1 - x0, nin_r = y1 - y0;
+  // stage the input window (4-byte words covering each row segment)
+  const int64_t pitch = static_cast<int64_t>(W) * 3;
+  const int words = (nin_c * 3 + 3 + 3) >> 2;
+  for (int i = tid; i < nin_r * words; i += 256) {
+    const int r = i / words, w = i - r * words;
+    const int64_t start = (static_cast<int64_t>(y0 + r) * pitch + static_cast<int64_t>(x0) * 3);
+    const int64_t a = start & ~int64_t{3};
+    if (w == 0) shift[r] = static_cast<int>(start - a);
+    const int64_t byte = a + 4 * w;
+    if (byte < static_cast<int64_t>(H) * pitch)
+      *reinterpret_cast<uint32_t*>(sin + r * kFPitch + 4 * w) = __ldg(reinterpret_cast<const uint32_t*>(img + byte));
+  }
+  __syncthreads();
+  // horizontal pass: staged rows x output columns x channels
+  for (int i = tid; i < nin_r * ncol * 3; i += 256) {
+    const int ch = i % 3, rc = i / 3;
+    const int c = rc % ncol, r = rc / ncol;
+    const unsigned char* px = sin + r * kFPitch + shift[r] + (xlo[c] - x0) * 3 + ch;
+    const float* w = wx + c * kFMaxTaps;
+    float acc = 0.f;
+    for (int k = 0; k < xn[c]; ++k) acc = fmaf(w[k], static_cast<float>(px[3 * k]), acc);
+    sh[(r * kFTW + c) * 3 + ch] = acc;
+  }
+  __syncthreads();
+  // vertical pass and the uint8 store
+  for (int i = tid; i < nrow * ncol * 3; i += 256) {
+    const int ch = i % 3, rc = i / 3;
+    const int c = rc % ncol, r = rc / ncol;
+    const float* w = wy + r * kFMaxTaps;
+    const float* col = sh + ((ylo[r] - y0) * kFTW + c) * 3 + ch;
+    float acc = 0.f;
+    for (int k = 0; k < yn[r]; ++k) acc = fmaf(w[k], col[k * kFTW * 3], acc);
+    out[(static_cast<int64_t>(oy0 + r) * Wo + ox0 + c) * 3 + ch] =
+        static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc))));
   }
 }
 
@@ -424,6 +577,26 @@ DensityLayout density_layout(int B, const int32_t* H, const int32_t* W) {
   L.d_off = L.inv_off + align_up(static_cast<size_t>(n) * sizeof(float), 256);
   L.total = L.d_off + align_up(static_cast<size_t>(n) * sizeof(float), 256);
   return L;
+}
+
+// Dynamic shared memory of apc_tail: the largest image's distances when they fit.
+size_t tail_smem(const ApcTable& t) {
+  int n = 0;
+  for (int i = 0; i < t.nb; ++i) n = std::max(n, (t.H[i] / kPatch) * t.gw[i]);
+  return n <= kTailSmemMax ? static_cast<size_t>(n) * sizeof(float) : 0;
+}
+
+pace_status_t tail_smem_attr() {
+  static std::atomic<uint64_t> done{0};
+  int dev = 0;
+  PACE_CUDA(cudaGetDevice(&dev));
+  const uint64_t bit = uint64_t{1} << (dev & 63);
+  if (!(done.load(std::memory_order_acquire) & bit)) {
+    PACE_CUDA(cudaFuncSetAttribute(apc_tail, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   static_cast<int>(kTailSmemMax * sizeof(float))));
+    done.fetch_or(bit, std::memory_order_acq_rel);
+  }
+  return PACE_OK;
 }
 
 pace_status_t check_images(const uint8_t* img, const int64_t* off, const int32_t* H, const int32_t* W, int B) {
@@ -465,6 +638,7 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
   const DensityLayout L = density_layout(B, H, W);
   if (ws == nullptr || ws_bytes < L.total || reinterpret_cast<uintptr_t>(ws) % 16) return PACE_ERR_WORKSPACE;
   PACE_CHECK(check_device());
+  PACE_CHECK(tail_smem_attr());
   uint8_t* w8 = static_cast<uint8_t*>(ws);
   auto* sums = reinterpret_cast<unsigned long long*>(w8 + L.sums_off);
   auto* inv = reinterpret_cast<float*>(w8 + L.inv_off);
@@ -503,7 +677,7 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
     else apc_pass2<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d, stats);
     PACE_CHECK(check_launch());
     TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
-    apc_tail<<<nb, 1024, 0, stream>>>(t, d, tp, stats);
+    apc_tail<<<nb, 1024, tail_smem(t), stream>>>(t, d, tp, stats);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;
@@ -523,6 +697,17 @@ static pace_status_t resample_impl(const uint8_t* src, const int64_t* src_off, c
   for (int b = 0; b < B; ++b)
     if (dst_off[b] < 0) return PACE_ERR_INVALID_ARG;
   PACE_CHECK(check_device());
+  {
+    static std::atomic<uint64_t> done{0};   // opt in to the fast path's shared memory once per device
+    int dev = 0;
+    PACE_CUDA(cudaGetDevice(&dev));
+    const uint64_t bit = uint64_t{1} << (dev & 63);
+    if (!(done.load(std::memory_order_acquire) & bit)) {
+      PACE_CUDA(cudaFuncSetAttribute(apc_resample, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(kFSmem)));
+      done.fetch_or(bit, std::memory_order_acq_rel);
+    }
+  }
   for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
     const int nb = (B - c0) < kApcMaxB ? (B - c0) : kApcMaxB;
     ResampleTable t{};
@@ -540,8 +725,8 @@ static pace_status_t resample_impl(const uint8_t* src, const int64_t* src_off, c
       if (t.Ho[i] > hmax) hmax = t.Ho[i];
       if (t.Wo[i] > wmax) wmax = t.Wo[i];
     }
-    dim3 grid((wmax + kRsTW - 1) / kRsTW, (hmax + kRsTH - 1) / kRsTH, nb);
-    apc_resample<<<grid, 256, 0, stream>>>(src, t, stats, dst);
+    dim3 grid((wmax + kFTW - 1) / kFTW, (hmax + kFTH - 1) / kFTH, nb);
+    apc_resample<<<grid, 256, kFSmem, stream>>>(src, t, stats, dst);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;
@@ -613,6 +798,7 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
       !(p.r_min <= p.r_max) || p.align < 1)
     return PACE_ERR_INVALID_ARG;
   PACE_CHECK(check_device());
+  PACE_CHECK(tail_smem_attr());
   unsigned char* scratch = nullptr;
   PACE_CHECK(static_scratch(&scratch));
   auto* sums = reinterpret_cast<unsigned long long*>(scratch);
@@ -649,6 +835,6 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
   else apc_pass2<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d_out, stats);
   PACE_CHECK(check_launch());
   TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
-  apc_tail<<<B, 1024, 0, stream>>>(t, d_out, tp, stats);
+  apc_tail<<<B, 1024, tail_smem(t), stream>>>(t, d_out, tp, stats);
   return check_launch();
 }

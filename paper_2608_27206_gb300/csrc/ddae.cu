@@ -13,6 +13,7 @@
 #include <cmath>
 
 #include "pace_common.cuh"
+#include "pace_select.cuh"
 
 namespace pace {
 namespace {
@@ -63,29 +64,6 @@ __device__ __forceinline__ float2 block_reduce2(float a, float b, float* red) {
   }
   __syncthreads();
   return make_float2(red[0], red[32]);
-}
-
-// Exclusive prefix count of `flag` over the block in thread order; returns (prefix, total).
-__device__ __forceinline__ int2 block_scan_flag(bool flag, int* wsum) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const unsigned bal = __ballot_sync(0xffffffffu, flag);
-  const int in_warp = __popc(bal & ((1u << lane) - 1u));
-  __syncthreads();
-  if (lane == 0) wsum[warp] = __popc(bal);
-  __syncthreads();
-  if (warp == 0) {
-    int v = wsum[lane];
-    int incl = v;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      int n = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += n;
-    }
-    wsum[lane] = incl - v;       // exclusive prefix of warp totals
-    if (lane == 31) wsum[32] = incl;
-  }
-  __syncthreads();
-  return make_int2(wsum[warp] + in_warp, wsum[32]);
 }
 
 __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* __restrict__ s_llm,
@@ -163,24 +141,22 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
   }
   unsigned prefix = 0u, mask = 0u;
   unsigned remaining = static_cast<unsigned>(K);
+  const int lane = tid & 31;
   for (int shift = 24; shift >= 0; shift -= 8) {
     for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
     __syncthreads();
-    for (int i = tid; i < nv; i += kSelThreads) {
-      const unsigned key = __float_as_uint(A[i]);
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    // histogram of the next digit; lanes holding the same digit are combined first, so a
+    // narrow value range costs one shared atomic per distinct digit per warp
+    for (int base = 0; base < nv; base += kSelThreads) {
+      const int i = base + tid;
+      const unsigned key = i < nv ? __float_as_uint(A[i]) : 0u;
+      const bool in = i < nv && (key & mask) == prefix;
+      const unsigned digit = in ? ((key >> shift) & 255u) : 256u;
+      const unsigned peers = __match_any_sync(0xffffffffu, digit);
+      if (in && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], static_cast<unsigned>(__popc(peers)));
     }
     __syncthreads();
-    if (tid == 0) {
-      unsigned above = 0u;
-      int d = 255;
-      for (; d > 0; --d) {
-        if (above + hist[d] >= remaining) break;
-        above += hist[d];
-      }
-      sel[0] = static_cast<unsigned>(d);
-      sel[1] = above;
-    }
+    if (tid < 32) warp_digit_search(hist, remaining, sel);
     __syncthreads();
     prefix |= sel[0] << shift;
     mask |= 255u << shift;
@@ -190,19 +166,39 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
   const unsigned T = prefix;  // bit pattern of the K-th largest S_final
   // `remaining` = how many keys equal to T are kept (lowest indices first)
 
-  // 5. ascending compaction
-  int eq_before = 0, taken_before = 0;
+  // 5. ascending compaction: the kept tokens before index i are the keys > T before i plus
+  // min(keys == T before i, remaining), so one packed prefix count per chunk places them
+  int gt_run = 0, eq_run = 0;
+  const unsigned lt_mask = (1u << lane) - 1u;
+  const int warp = tid >> 5;
   for (int base = 0; base < nv; base += kSelThreads) {
     const int i = base + tid;
     const unsigned key = i < nv ? __float_as_uint(A[i]) : 0u;
     const bool gt = i < nv && key > T;
     const bool eq = i < nv && key == T;
-    const int2 er = block_scan_flag(eq, wsum);
-    const bool take = gt || (eq && static_cast<unsigned>(eq_before + er.x) < remaining);
-    const int2 tr = block_scan_flag(take, wsum);
-    if (take) kept[k0 + taken_before + tr.x] = v0 + i;
-    eq_before += er.y;
-    taken_before += tr.y;
+    const unsigned bg = __ballot_sync(0xffffffffu, gt), be = __ballot_sync(0xffffffffu, eq);
+    if (lane == 0) wsum[warp] = static_cast<int>(__popc(bg) | (__popc(be) << 16));
+    __syncthreads();
+    if (warp == 0) {
+      const int v = wsum[lane];
+      int incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+      }
+      wsum[lane] = incl - v;
+      if (lane == 31) wsum[32] = incl;
+    }
+    __syncthreads();
+    const int wp = wsum[warp];
+    const int gt_before = gt_run + (wp & 0xffff) + __popc(bg & lt_mask);
+    const int eq_before = eq_run + (wp >> 16) + __popc(be & lt_mask);
+    if (gt || (eq && static_cast<unsigned>(eq_before) < remaining))
+      kept[k0 + gt_before + min(eq_before, static_cast<int>(remaining))] = v0 + i;
+    gt_run += wsum[32] & 0xffff;
+    eq_run += wsum[32] >> 16;
+    __syncthreads();
   }
 }
 
@@ -213,7 +209,7 @@ __global__ void __launch_bounds__(256) gather_rows_v16(const uint4* __restrict__
   const int lane = threadIdx.x & 31;
   const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
-  constexpr int U = 8;
+  constexpr int U = 16;
   for (int64_t r = warp0; r < n_idx; r += nwarps) {
     const int64_t s = idx[r];
     uint4* dp = dst + r * row_vec;
