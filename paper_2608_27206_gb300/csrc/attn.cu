@@ -95,6 +95,7 @@ struct SmemCtl {
   uint64_t bars[40];
   uint32_t tmem_base;
   int abort;
+  int redo;                  // pass 1: some row overflowed the fixed-shift round
   float xchg[3][2][kTile];   // hand-over between the four epilogue warpgroups
 };
 
@@ -193,6 +194,56 @@ __device__ __forceinline__ void lse_update64(const uint32_t (&v)[64], int valid,
   l_run += a.x + a.y;
 }
 
+// Fixed-shift row update with 64 new scores: the shift m is the base-2 maximum of the row's
+// first chunk and then never moves, so there is no maximum in the common path.  Every term
+// 2^(c s - m) is computed to full relative precision whatever its size, and the largest term
+// of the row is >= 1, so nothing underflows; the only failure is overflow (a score more than
+// about 127 - log2(N) above m), which leaves l = inf or NaN and is caught by the caller.
+template <bool FIRST>
+__device__ __forceinline__ void lse_fixed64(const uint32_t (&v)[64], int valid, float c, float& m_run,
+                                            float& l_run) {
+  float s[64];
+#pragma unroll
+  for (int e = 0; e < 64; ++e) s[e] = __uint_as_float(v[e]);
+  if (valid < 64) {
+#pragma unroll
+    for (int e = 0; e < 64; ++e)
+      if (e >= valid) s[e] = -INFINITY;
+  }
+  if (FIRST) {
+    float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+#pragma unroll
+    for (int e = 0; e < 64; e += 8) {
+      mx0 = max3(mx0, s[e + 0], s[e + 1]);
+      mx1 = max3(mx1, s[e + 2], s[e + 3]);
+      mx2 = max3(mx2, s[e + 4], s[e + 5]);
+      mx3 = max3(mx3, s[e + 6], s[e + 7]);
+    }
+    m_run = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * c;
+  }
+  const float2 cc = make_float2(c, c);
+  const float2 nm = make_float2(-m_run, -m_run);
+  float2 a0 = make_float2(0.f, 0.f), a1 = a0;
+#pragma unroll
+  for (int e = 0; e < 64; e += 4) {
+    const float2 x0 = ffma2(make_float2(s[e], s[e + 1]), cc, nm);
+    const float2 x1 = ffma2(make_float2(s[e + 2], s[e + 3]), cc, nm);
+    a0 = fadd2(a0, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
+    a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
+  }
+  const float2 a = fadd2(a0, a1);
+  l_run += a.x + a.y;
+}
+
+// Dispatch of the fixed-shift update: the first chunk with keys sets the shift.  The two
+// cases are separate instantiations so that the maximum is not issued (predicated off) for
+// every chunk.
+__device__ __forceinline__ void lse_fixed(const uint32_t (&v)[64], int valid, float c, float& m_run, float& l_run) {
+  if (valid <= 0) return;
+  if (m_run == -INFINITY) lse_fixed64<true>(v, valid, c, m_run, l_run);
+  else lse_fixed64<false>(v, valid, c, m_run, l_run);
+}
+
 // acc += sum_e 2^(c s_e + nL_e) over 64 columns; nL (negated base-2 LSE) from shared memory.
 __device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], const float* nL, float c, float2 acc) {
   const float2 cc = make_float2(c, c);
@@ -210,15 +261,15 @@ __device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], const float*
   return fadd2(acc, a1);
 }
 
-// Shared teardown: waits for the pair's MMAs, lets in-flight copies land after an abort, then
-// releases TMEM with both CTAs in step.
-__device__ __forceinline__ void pair_teardown(SmemCtl* ctl, uint32_t b_done, uint32_t tmem, int* status,
-                                              int kernel) {
+// Brings the pair to a quiet point: waits for the pair's MMAs (phase `done_phase` of b_done),
+// lets in-flight copies land after an abort, and synchronises both CTAs; TMEM stays allocated.
+__device__ __forceinline__ void pair_quiesce(SmemCtl* ctl, uint32_t b_done, uint32_t done_phase, int* status,
+                                             int kernel) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   tc_fence_before_sync();
   __syncthreads();
   if (warp == 1 && lane == 0) {
-    if (!mbar_wait(b_done, 0, kWaitLimitNs)) record_error(status, PACE_ERR_TIMEOUT, kernel);
+    if (!mbar_wait(b_done, done_phase, kWaitLimitNs)) record_error(status, PACE_ERR_TIMEOUT, kernel);
   }
   if (threadIdx.x == 0 && aborted(ctl)) {   // give outstanding TMA copies time to land
     const uint64_t t0 = globaltimer_ns();
@@ -229,8 +280,19 @@ __device__ __forceinline__ void pair_teardown(SmemCtl* ctl, uint32_t b_done, uin
   tc_fence_before_sync();
   cluster_sync_all();
   tc_fence_after_sync();
-  if (warp == 1) tmem_dealloc_pair(tmem, kTmemCols);
+}
+
+// Releases the pair's TMEM with both CTAs in step (after pair_quiesce).
+__device__ __forceinline__ void pair_release_tmem(uint32_t tmem) {
+  if ((threadIdx.x >> 5) == 1) tmem_dealloc_pair(tmem, kTmemCols);
   cluster_sync_all();
+}
+
+// Shared teardown: pair_quiesce, then TMEM release.
+__device__ __forceinline__ void pair_teardown(SmemCtl* ctl, uint32_t b_done, uint32_t tmem, int* status,
+                                              int kernel) {
+  pair_quiesce(ctl, b_done, 0, status, kernel);
+  pair_release_tmem(tmem);
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -287,6 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
       mbar_init(b_sfree(p), 2 * 8);
     }
     ctl->abort = 0;
+    ctl->redo = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -298,110 +361,137 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
   tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
 
-  if (warp == 0) {
-    if (lane == 0) {
-      prefetch_tensormap(&tmq);
-      prefetch_tensormap(&tmk);
-      if (C::R > 0) {
-        prefetch_tensormap(&tmq32);
-        prefetch_tensormap(&tmk32);
-      }
-      // the even CTA's full barriers count the bytes of both halves; the odd CTA's copies
-      // complete there too
-      const uint32_t qfull_L = mapa_shared(b_qfull, 0);
-      if (rank == 0) mbar_arrive_expect_tx(b_qfull, 2 * C::TILE_BYTES);
-      load_tile<D>(sQ, &tmq, &tmq32, h * D, t.q0[b] + qrow0, qfull_L);
-      for (int j = 0; j < nj; ++j) {
-        const int s = j % ST, u = j / ST;
-        if (u > 0 && !mbar_wait(b_kempty(s), (u - 1) & 1, kWaitLimitNs)) {
-          set_abort(ctl, status, K_ATTN_ROW_LSE);
-          break;
-        }
-        if (aborted(ctl)) break;
-        const uint32_t kfull_L = mapa_shared(b_kfull(s), 0);
-        if (rank == 0) mbar_arrive_expect_tx(b_kfull(s), 2 * C::TILE_BYTES);
-        load_tile<D>(sK + s * C::TILE_BYTES, &tmk, &tmk32, g * D,
-                     t.k0[b] + (kt0 + j) * kPair + kTile * static_cast<int>(rank), kfull_L);
-      }
+  // Round 0 uses the fixed-shift update; if any row of the pair overflowed it, round 1
+  // streams the keys again with the exact online-maximum update.  Stream tiles are counted
+  // across rounds (it = round * nj + j), so every barrier keeps its phase sequence.
+  const int e = (warp - 2) >> 2;            // epilogue warpgroup (warps 2..17)
+  const int p = e >> 1, hh = e & 1;
+  const int quad = warp & 3;
+  const int rr = quad * 32 + lane;
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmq);
+    prefetch_tensormap(&tmk);
+    if (C::R > 0) {
+      prefetch_tensormap(&tmq32);
+      prefetch_tensormap(&tmk32);
     }
-  } else if (warp == 1) {
-    if (lane == 0 && rank == 0) {
-      uint64_t aq128, aq32, bk128, bk32;
-      tile_desc<D>(sQ, aq128, aq32);
-      tile_desc<D>(sK, bk128, bk32);
-      bool ok = mbar_wait(b_qfull, 0, kWaitLimitNs);
-      if (!ok) set_abort(ctl, status, K_ATTN_ROW_LSE);
-      for (int j = 0; ok && j < nj; ++j) {
-        const int s = j % ST, u = j / ST;
-        const int p = j & 1, v = j >> 1;
-        if (!mbar_wait(b_kfull(s), u & 1, kWaitLimitNs) ||
-            (v > 0 && !mbar_wait(b_sfree(p), (v - 1) & 1, kWaitLimitNs)) || aborted(ctl)) {
+    // the even CTA's full barriers count the bytes of both halves; the odd CTA's copies
+    // complete there too
+    const uint32_t qfull_L = mapa_shared(b_qfull, 0);
+    if (rank == 0) mbar_arrive_expect_tx(b_qfull, 2 * C::TILE_BYTES);
+    load_tile<D>(sQ, &tmq, &tmq32, h * D, t.q0[b] + qrow0, qfull_L);
+  }
+  auto run_round = [&](int round) {
+    const int it0 = round * nj;
+    if (warp == 0) {
+      if (lane == 0) {
+        for (int j = 0; j < nj; ++j) {
+          const int it = it0 + j;
+          const int s = it % ST, u = it / ST;
+          if (u > 0 && !mbar_wait(b_kempty(s), (u - 1) & 1, kWaitLimitNs)) {
+            set_abort(ctl, status, K_ATTN_ROW_LSE);
+            break;
+          }
+          if (aborted(ctl)) break;
+          const uint32_t kfull_L = mapa_shared(b_kfull(s), 0);
+          if (rank == 0) mbar_arrive_expect_tx(b_kfull(s), 2 * C::TILE_BYTES);
+          load_tile<D>(sK + s * C::TILE_BYTES, &tmk, &tmk32, g * D,
+                       t.k0[b] + (kt0 + j) * kPair + kTile * static_cast<int>(rank), kfull_L);
+        }
+      }
+    } else if (warp == 1) {
+      if (lane == 0 && rank == 0) {
+        uint64_t aq128, aq32, bk128, bk32;
+        tile_desc<D>(sQ, aq128, aq32);
+        tile_desc<D>(sK, bk128, bk32);
+        const bool ok = mbar_wait(b_qfull, 0, kWaitLimitNs);
+        if (!ok) set_abort(ctl, status, K_ATTN_ROW_LSE);
+        for (int j = 0; ok && j < nj; ++j) {
+          const int it = it0 + j;
+          const int s = it % ST, u = it / ST;
+          const int pa = it & 1, v = it >> 1;
+          if (!mbar_wait(b_kfull(s), u & 1, kWaitLimitNs) ||
+              (v > 0 && !mbar_wait(b_sfree(pa), (v - 1) & 1, kWaitLimitNs)) || aborted(ctl)) {
+            set_abort(ctl, status, K_ATTN_ROW_LSE);
+            break;
+          }
+          tc_fence_after_sync();
+          const uint64_t so = static_cast<uint64_t>(s * (C::TILE_BYTES >> 4));
+          mma_tile<D>(tmem + pa * 256, aq128, aq32, bk128 + so, bk32 + so);
+          mma_commit_pair_mc(b_sfull(pa), 3);
+          mma_commit_pair_mc(b_kempty(s), 3);
+        }
+        mma_commit_pair_mc(b_done, 3);
+      }
+      __syncwarp();
+    } else {
+      // epilogue warpgroup e = 2p + hh: accumulator p (stream tiles it % 2 == p), columns hh * 128 ..
+      float m_run = -INFINITY, l_run = 0.f;
+      const uint32_t sfree_L = mapa_shared(b_sfree(p), 0);
+      const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
+      for (int j = (p - it0) & 1; j < nj; j += 2) {
+        const int it = it0 + j;
+        const int v = it >> 1;
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs));
+        if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
           set_abort(ctl, status, K_ATTN_ROW_LSE);
           break;
         }
         tc_fence_after_sync();
-        const uint64_t so = static_cast<uint64_t>(s * (C::TILE_BYTES >> 4));
-        mma_tile<D>(tmem + p * 256, aq128, aq32, bk128 + so, bk32 + so);
-        mma_commit_pair_mc(b_sfull(p), 3);
-        mma_commit_pair_mc(b_kempty(s), 3);
+        const int valid = t.nk[b] - ((kt0 + j) * kPair + hh * kTile);   // keys of these columns in the image
+        uint32_t sv[64];
+        load_cols64(tbuf, sv);
+        if (round == 0) lse_fixed(sv, valid, c, m_run, l_run);
+        else lse_update64(sv, valid, c, m_run, l_run);
+        load_cols64(tbuf + 64, sv);
+        tc_fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote(sfree_L);
+        if (round == 0) lse_fixed(sv, valid - 64, c, m_run, l_run);
+        else if (valid > 64) lse_update64(sv, valid - 64, c, m_run, l_run);
       }
-      mma_commit_pair_mc(b_done, 3);
-    }
-    __syncwarp();
-  } else {
-    // epilogue warpgroup e = 2p + hh: accumulator p (key tiles j % 2 == p), columns hh * 128 ..
-    const int e = (warp - 2) >> 2;
-    const int p = e >> 1, hh = e & 1;
-    const int quad = warp & 3;
-    const int rr = quad * 32 + lane;
-    const uint32_t sfree_L = mapa_shared(b_sfree(p), 0);
-    float m_run = -INFINITY, l_run = 0.f;
-    const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
-    for (int j = p; j < nj; j += 2) {
-      const int v = j >> 1;
-      const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs));
-      if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
-        set_abort(ctl, status, K_ATTN_ROW_LSE);
-        break;
+      if (!(l_run < INFINITY)) ctl->redo = 1;   // inf or NaN: this row needs the exact round
+      // merge the four warpgroups' (m, l) of each row
+      if (e > 0) {
+        ctl->xchg[e - 1][0][rr] = m_run;
+        ctl->xchg[e - 1][1][rr] = l_run;
       }
-      tc_fence_after_sync();
-      const int valid = t.nk[b] - ((kt0 + j) * kPair + hh * kTile);   // keys of these columns in the image
-      uint32_t sv[64];
-      load_cols64(tbuf, sv);
-      lse_update64(sv, valid, c, m_run, l_run);
-      load_cols64(tbuf + 64, sv);
-      tc_fence_before_sync();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_remote(sfree_L);
-      if (valid > 64) lse_update64(sv, valid - 64, c, m_run, l_run);
-    }
-    // merge the four warpgroups' (m, l) of each row
-    if (e > 0) {
-      ctl->xchg[e - 1][0][rr] = m_run;
-      ctl->xchg[e - 1][1][rr] = l_run;
-    }
-    named_barrier_sync(1, 32 * kEpiWarps);
-    if (e == 0) {
-      float M = m_run;
+      named_barrier_sync(1, 32 * kEpiWarps);
+      if (e == 0) {
+        float M = m_run;
 #pragma unroll
-      for (int i = 0; i < 3; ++i) M = fmaxf(M, ctl->xchg[i][0][rr]);
-      float l = l_run > 0.f ? l_run * ex2_approx(m_run - M) : 0.f;
+        for (int i = 0; i < 3; ++i) M = fmaxf(M, ctl->xchg[i][0][rr]);
+        float l = l_run > 0.f ? l_run * ex2_approx(m_run - M) : 0.f;
 #pragma unroll
-      for (int i = 0; i < 3; ++i) {
-        const float li = ctl->xchg[i][1][rr];
-        if (li > 0.f) l += li * ex2_approx(ctl->xchg[i][0][rr] - M);
-      }
-      const int row = qrow0 + rr;                       // local query row
-      const int64_t prow = static_cast<int64_t>(h) * t.prows + t.lpad[b] + row;
-      if (t.splits == 1) {
-        nL_out[prow] = row < t.nq[b] ? -(M + log2f(l)) : -INFINITY;
-      } else {
-        ml_out[static_cast<int64_t>(split) * t.H * t.prows + prow] =
-            (row < t.nq[b] && l > 0.f) ? make_float2(M, l) : make_float2(-INFINITY, 0.f);
+        for (int i = 0; i < 3; ++i) {
+          const float li = ctl->xchg[i][1][rr];
+          if (li > 0.f) l += li * ex2_approx(ctl->xchg[i][0][rr] - M);
+        }
+        const int row = qrow0 + rr;                       // local query row
+        const int64_t prow = static_cast<int64_t>(h) * t.prows + t.lpad[b] + row;
+        if (t.splits == 1) {
+          nL_out[prow] = row < t.nq[b] ? -(M + log2f(l)) : -INFINITY;
+        } else {
+          ml_out[static_cast<int64_t>(split) * t.H * t.prows + prow] =
+              (row < t.nq[b] && l > 0.f) ? make_float2(M, l) : make_float2(-INFINITY, 0.f);
+        }
       }
     }
+  };
+
+  run_round(0);
+  pair_quiesce(ctl, b_done, 0, status, K_ATTN_ROW_LSE);
+  // If a row of either CTA overflowed the fixed shift, the pair streams the keys again with
+  // the exact update and overwrites its outputs (stream tiles continue at it = nj ..).
+  const uint32_t peer = rank ^ 1u;
+  const int redo_any = ctl->redo | static_cast<int>(ld_shared_cluster_u32(mapa_shared(smem_u32(&ctl->redo), peer)));
+  const int abort_any = ctl->abort | static_cast<int>(ld_shared_cluster_u32(mapa_shared(smem_u32(&ctl->abort), peer)));
+  if (redo_any != 0 && abort_any == 0) {
+    cluster_sync_all();   // both CTAs have read the flags before either one changes them
+    run_round(1);
+    pair_quiesce(ctl, b_done, 1, status, K_ATTN_ROW_LSE);
   }
-  pair_teardown(ctl, b_done, tmem, status, K_ATTN_ROW_LSE);
+  pair_release_tmem(tmem);
 }
 
 // Merges per-split (m, l) pairs into -L = -(m + log2(l)); rows past the image get -inf.

@@ -228,6 +228,62 @@ def test_vit_importance_sinks(pace):
     assert_scores_close(out, ref, what="S_vis_raw with sinks")
 
 
+def _spiked_qk(n, H, D, seed, spikes):
+    """Random Q/K with planted score spikes: for (key, rows, norm) the key and the query rows
+    get the same direction u with length `norm`, so those rows score norm^2 against that key,
+    far above everything before it in the row."""
+    rng = np.random.default_rng(seed)
+    Q = f64(synth.random_small_qk(seed, n, H, D))
+    K = f64(synth.random_small_qk(seed + 1000, n, H, D))
+    for key, rows, norm in spikes:
+        u = rng.standard_normal((H, D))
+        u /= np.linalg.norm(u, axis=1, keepdims=True)
+        K[key] = norm * u
+        Q[rows] = norm * u + 0.05 * rng.standard_normal((len(rows), H, D))
+    return (synth.f32_to_bf16_bits(Q.astype(np.float32)), synth.f32_to_bf16_bits(K.astype(np.float32)))
+
+
+def test_vit_importance_wide_score_range(pace):
+    """Rows whose maximum lies 88 and 244 (base 2) above the scores of their first keys: the
+    first stays finite in a fixed-shift sum, the second overflows exp2 and must be redone
+    with an exact running maximum."""
+    n, H, D = 1024, 2, 80
+    Qb, Kb = _spiked_qk(n, H, D, seed=5, spikes=[(700, np.arange(0, 200), 25.0),
+                                                 (900, np.arange(300, 340), 40.0)])
+    cu = np.array([0, n], np.int32)
+    scale = 1.0 / math.sqrt(D)
+    out = pace.pace_vit_attn_importance(bf16_tensor(Qb), bf16_tensor(Kb), cu, scale, 1).cpu().numpy()
+    ref = O.vit_attn_importance(f64(Qb), f64(Kb), cu, scale, 1)
+    assert ref[700] > 150 and ref[900] > 30       # the spikes dominate their rows
+    assert_scores_close(out, ref, what="S_vis_raw with score spikes")
+    _no_device_error(pace)
+
+
+def test_llm_importance_wide_score_range(pace):
+    """A spike 200 (base 2) above the other scores through the GQA path with key splits (few
+    query tiles, many key tiles): exp2 overflows in the first round of every split that holds
+    the spike key."""
+    nq, nk, Hq, Hkv, D = 64, 2304, 4, 2, 128
+    Qs, _ = _spiked_qk(nq, Hq, D, seed=6, spikes=[])
+    rng = np.random.default_rng(6)
+    Q = f64(Qs)
+    K = f64(synth.random_small_qk(7, nk, Hkv, D))
+    for g in range(Hkv):
+        u = rng.standard_normal(D)
+        u /= np.linalg.norm(u)
+        K[2000, g] = 40.0 * u
+        for h in range(g * (Hq // Hkv), (g + 1) * (Hq // Hkv)):
+            Q[:32, h] = 40.0 * u
+    Qb, Kb = synth.f32_to_bf16_bits(Q.astype(np.float32)), synth.f32_to_bf16_bits(K.astype(np.float32))
+    cq, ck = np.array([0, nq], np.int32), np.array([0, nk], np.int32)
+    scale = 1.0 / math.sqrt(D)
+    out = pace.pace_llm_text_visual_importance(bf16_tensor(Qb), bf16_tensor(Kb), cq, ck, scale).cpu().numpy()
+    ref = O.llm_text_visual_importance(f64(Qb), f64(Kb), cq, ck, scale)
+    assert ref[2000] > 32 * Hq * 0.9
+    assert_scores_close(out, ref, what="S_llm_raw with score spikes")
+    _no_device_error(pace)
+
+
 def _llm_case(pace, tq, nv, Hq=28, Hkv=4, D=128, seed=0):
     cq = np.concatenate([[0], np.cumsum(tq)]).astype(np.int32)
     ck = np.concatenate([[0], np.cumsum(nv)]).astype(np.int32)
