@@ -244,6 +244,12 @@ __device__ __forceinline__ void lse_fixed(const uint32_t (&v)[64], int valid, fl
   else lse_fixed64<false>(v, valid, c, m_run, l_run);
 }
 
+// Number of the 16 four-column steps of a 64-column chunk whose exp2 runs on the FMA pipe
+// (exp2_fma2) instead of the MUFU; the two pipes then share the work.
+constexpr int kPolySteps = 2;
+
+__device__ __forceinline__ constexpr bool poly_step(int k) { return (k * kPolySteps) % 16 < kPolySteps; }
+
 // acc += sum_e 2^(c s_e + nL_e) over 64 columns; nL (negated base-2 LSE) from shared memory.
 __device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], const float* nL, float c, float2 acc) {
   const float2 cc = make_float2(c, c);
@@ -255,8 +261,13 @@ __device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], const float*
     const float2 x0 = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), cc, make_float2(l.x, l.y));
     const float2 x1 =
         ffma2(make_float2(__uint_as_float(v[e + 2]), __uint_as_float(v[e + 3])), cc, make_float2(l.z, l.w));
-    acc = fadd2(acc, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
-    a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
+    if (poly_step(e / 4)) {
+      acc = fadd2(acc, exp2_fma2(x0));
+      a1 = fadd2(a1, exp2_fma2(x1));
+    } else {
+      acc = fadd2(acc, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
+      a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
+    }
   }
   return fadd2(acc, a1);
 }
