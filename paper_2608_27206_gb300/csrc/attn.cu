@@ -4,34 +4,37 @@
 // P_ij = exp(s_ij - lse_i), s_ij = scale q_i . k_j.  They are computed flash-style in two
 // passes so that the N x N score matrix is never stored:
 //
-//   pass 1  attn_row_lse   S = Q K^T on tcgen05, online row max / sum of exp2 on the CUDA
-//           cores, giving the base-2 log-sum-exp L_i = log2 sum_j 2^(c s_ij),
-//           c = scale * log2(e), stored negated.  Optionally split over key ranges (partial
-//           (m, l) pairs merged by attn_lse_combine).
-//   pass 2  attn_colsum    S^T = K Q^T: every TMEM lane is one key, so each epilogue thread
-//           owns one key and accumulates 2^(c s_ji - L_i) over the whole query stream in
-//           registers; no cross-thread reduction and no atomics.
+//   pass 1  attn_row_lse   S = Q K^T on tcgen05 and, on the CUDA cores, the base-2 row
+//           log-sum-exp L_i = log2 sum_j 2^(c s_ij), c = scale * log2(e).  Each row's shift
+//           is fixed at the maximum of its first chunk of scores, so the common path has no
+//           running maximum; a CTA whose rows overflowed that shift streams its keys a second
+//           time with the exact online maximum.  Optionally split over key ranges (partial
+//           (m, l) pairs merged by attn_lse_combine).  The result is stored as a 16-column
+//           bf16 "shift row" per query: -L_i / c as hi + mid + lo, then zeros.
+//   pass 2  attn_colsum    S^T = K Q^T with one extra K-step that multiplies the keys' ones
+//           slice [1, 1, 1, 0, ...] by the queries' shift rows, so the accumulator already
+//           holds s_ji - L_i / c.  Every TMEM lane is one key: each epilogue thread owns one key
+//           and accumulates 2^(c a_ji) over the whole query stream in registers, with no
+//           per-column loads, cross-thread reduction or atomics.
 //   reduce  attn_reduce    sums the per-head (or per KV-head) partial maps and pools the
 //           `merge` consecutive patches of each merged token.
 //
-// Both passes run on CTA pairs (clusters of 2) with the two-SM MMA: one 256 x 256 x 16
-// tcgen05.mma per K-step, A = 256 resident rows (128 in each CTA), B = 256 streamed rows
-// (128 loaded by each CTA), so each SM reads half of B and a 128 x 256 fp32 accumulator
-// lands in each CTA's TMEM.  N = 256 halves the shared-memory operand traffic per flop
-// compared with 128-wide tiles.
+// Every CTA works alone (one-SM MMA, local barriers only): it holds 128 resident rows and
+// streams whole 256-row tiles, one 128 x 256 x 16 tcgen05.mma per K-step into a 128 x 256
+// fp32 TMEM accumulator.  A work item is 256 resident rows, i.e. two CTAs.
 //
 // CTA layout (576 threads, one CTA per SM):
-//   warp 0       TMA producer (one lane): this CTA's resident tile once, then its half of
-//                every streamed tile through a ring of stages; completion is counted on the
-//                even CTA's barriers
-//   warp 1       pair TMEM allocation (512 columns = two 128 x 256 accumulators) and, in the
-//                even CTA, MMA issue (one lane)
+//   warp 0       TMA producer (one lane): the resident tile once, then every streamed tile
+//                through a ring of stages
+//   warp 1       TMEM allocation (512 columns = two 128 x 256 accumulators) and MMA issue
+//                (one lane)
 //   warps 2-17   four epilogue warpgroups; warpgroup e = 2p + hh reads columns hh*128.. of
 //                accumulator p (stream tiles j with j % 2 == p); results of the four are
 //                merged at the end
 // Operands are K-major bf16 tiles staged by TMA: 64-column blocks with the 128-byte swizzle,
-// and a trailing 16-column slice with the 32-byte swizzle when the head dimension is not a
-// multiple of 64 (80 = 64 + 16).  MMA descriptors are built once and advanced by immediates.
+// and 16-column slices with the 32-byte swizzle (the tail of a head dimension that is not a
+// multiple of 64, 80 = 64 + 16, and the shift slices of pass 2).  MMA descriptors are built
+// once and advanced by immediates.
 //
 // GQA: query head h reads KV head h / G.  The ViT case is G = 1.
 #include <algorithm>
@@ -39,6 +42,7 @@
 #include <cmath>
 #include <mutex>
 
+#include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
 #include "pace_common.cuh"
@@ -49,28 +53,70 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kTile = 128;                // rows of a tile held by one CTA
-constexpr int kPair = 256;                // rows of a tile held by a CTA pair
+constexpr int kTile = 128;                // resident rows held by one CTA
+constexpr int kPair = 256;                // rows of one work item (two CTAs, 128 rows each)
+constexpr int kStream = 256;              // streamed rows per tile
 constexpr int kEpiWarps = 16;
 constexpr int kThreads = 64 + 32 * kEpiWarps;   // 576
 constexpr int kAttnMaxB = 64;
-constexpr int kBlock128 = kTile * 128;    // 128 rows x 64 bf16, 128-byte swizzle
-constexpr int kSlice32 = kTile * 32;      // 128 rows x 16 bf16, 32-byte swizzle
 constexpr uint32_t kTmemCols = 512;
-constexpr int kTargetItems = 152;         // one CTA pair per two SMs, two waves
+constexpr int kTargetItems = 152;         // work items (two CTAs each): two waves over the SMs
 
-// A 128-row operand tile of head dimension D is stored as NB blocks of 64 columns with the
-// 128-byte swizzle followed by R slices of 16 columns with the 32-byte swizzle
-// (D = 80: one block + one slice; D = 128: two blocks; D = 64: one block).
-template <int D>
-struct Cfg {
+// An operand tile of ROWS rows and head dimension D is stored as NB blocks of 64 columns
+// (ROWS x 128 bytes, 128-byte swizzle) followed by R slices of 16 columns (ROWS x 32 bytes,
+// 32-byte swizzle); D = 80: one block + one slice; D = 128: two blocks; D = 64: one block.
+template <int D, int ROWS>
+struct TileFmt {
   static constexpr int NB = D / 64;
   static constexpr int R = (D % 64) / 16;
-  static constexpr int TILE_BYTES = NB * kBlock128 + R * kSlice32;
-  static constexpr int STAGES = (D == 128) ? 5 : 8;
-  static constexpr uint32_t IDESC = idesc_bf16_f32(256, 256);
-  static_assert(D % 16 == 0 && TILE_BYTES % 1024 == 0, "head dim");
+  static constexpr int BLOCK = ROWS * 128;
+  static constexpr int SLICE = ROWS * 32;
+  static constexpr int BYTES = NB * BLOCK + R * SLICE;
+  static_assert(D % 16 == 0 && BYTES % 1024 == 0 && ROWS % kTile == 0, "tile format");
 };
+
+template <int D>
+struct Cfg {
+  using A = TileFmt<D, kTile>;      // resident tile
+  using B = TileFmt<D, kStream>;    // streamed tile
+  static constexpr int STAGES = (D == 128) ? 2 : (D == 80) ? 4 : 5;
+  static constexpr uint32_t IDESC = idesc_bf16_f32(kTile, kStream);
+};
+
+// Extra K slice of pass 2 (16 bf16 columns, 32 bytes per row).  Query row i carries the
+// negated base-2 LSE divided by c, split into three bf16 terms hi + mid + lo (the rest of the
+// 32 bytes zero); key rows carry [1, 1, 1, 0, ...].  One more K-step of the MMA then
+// accumulates s_ji - L_i / c, so the epilogue needs no per-column shift.
+constexpr int kShiftCols = 16;
+constexpr uint16_t kBf16One = 0x3F80;
+constexpr uint16_t kBf16NegHuge = 0xF180;   // -2^100: zero weight for padded query rows
+
+struct alignas(256) OnesSlice {
+  uint16_t v[kTile * kShiftCols];
+  constexpr OnesSlice() : v() {
+    for (int i = 0; i < kTile * kShiftCols; ++i) v[i] = (i % kShiftCols) < 3 ? kBf16One : 0;
+  }
+};
+__device__ const OnesSlice g_ones_slice{};
+
+// Writes the 32-byte shift row of one query: v = -L / c (or -inf for a padded row).
+__device__ __forceinline__ void store_shift_row(uint16_t* row, float v) {
+  uint32_t w0, w1;
+  if (v > -INFINITY) {
+    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+    const float r1 = v - __bfloat162float(hi);
+    const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+    const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+    w0 = static_cast<uint32_t>(__bfloat16_as_ushort(hi)) | (static_cast<uint32_t>(__bfloat16_as_ushort(mid)) << 16);
+    w1 = static_cast<uint32_t>(__bfloat16_as_ushort(lo));
+  } else {
+    w0 = kBf16NegHuge;
+    w1 = 0u;
+  }
+  uint4* p = reinterpret_cast<uint4*>(row);
+  p[0] = make_uint4(w0, w1, 0u, 0u);
+  p[1] = make_uint4(0u, 0u, 0u, 0u);
+}
 
 struct AttnTable {
   int q0[kAttnMaxB], nq[kAttnMaxB];   // query rows of image b
@@ -107,44 +153,50 @@ __device__ __forceinline__ bool aborted(const SmemCtl* ctl) {
   return *reinterpret_cast<const volatile int*>(&ctl->abort) != 0;
 }
 
-// TMA of this CTA's 128 rows (y .. y + 127, columns x0 .. x0 + D) into dst; completion is
-// counted on the (possibly remote) barrier `bar`.
-template <int D>
+// TMA of ROWS rows (y .. y + ROWS - 1, columns x0 .. x0 + D) into dst in 128-row boxes;
+// completion is counted on the barrier `bar`.
+template <int D, int ROWS>
 __device__ __forceinline__ void load_tile(uint8_t* dst, const CUtensorMap* m128, const CUtensorMap* m32, int x0,
                                           int y, uint32_t bar) {
-  using C = Cfg<D>;
+  using F = TileFmt<D, ROWS>;
 #pragma unroll
-  for (int i = 0; i < C::NB; ++i) tma_load_2d_pair(smem_u32(dst + i * kBlock128), m128, x0 + 64 * i, y, bar);
+  for (int q = 0; q < ROWS / kTile; ++q) {
 #pragma unroll
-  for (int r = 0; r < C::R; ++r)
-    tma_load_2d_pair(smem_u32(dst + C::NB * kBlock128 + r * kSlice32), m32, x0 + 64 * C::NB + 16 * r, y, bar);
+    for (int i = 0; i < F::NB; ++i)
+      tma_load_2d(smem_u32(dst + i * F::BLOCK + q * kTile * 128), m128, x0 + 64 * i, y + q * kTile, bar);
+#pragma unroll
+    for (int r = 0; r < F::R; ++r)
+      tma_load_2d(smem_u32(dst + F::NB * F::BLOCK + r * F::SLICE + q * kTile * 32), m32, x0 + 64 * F::NB + 16 * r,
+                  y + q * kTile, bar);
+  }
 }
 
 // Shared-memory descriptors of a tile: [0] for its 128-byte-swizzled blocks, [1] for its
 // 32-byte-swizzled slices.  Adding (bytes >> 4) moves the start address.
-template <int D>
+template <int D, int ROWS>
 __device__ __forceinline__ void tile_desc(const uint8_t* tile, uint64_t& d128, uint64_t& d32) {
   d128 = smem_desc_kmajor_sw128(smem_u32(tile));
-  d32 = smem_desc_kmajor_sw32(smem_u32(tile + Cfg<D>::NB * kBlock128));
+  d32 = smem_desc_kmajor_sw32(smem_u32(tile + TileFmt<D, ROWS>::NB * TileFmt<D, ROWS>::BLOCK));
 }
 
-// Pair MMA D[tmem] = A B^T over the whole head dimension: 4 K-steps per 128-byte block,
-// 1 per 32-byte slice.
+// MMA D[tmem] = A B^T (128 x 256) over the whole head dimension: 4 K-steps per 128-byte
+// block, 1 per 32-byte slice.
 template <int D>
 __device__ __forceinline__ void mma_tile(uint32_t d, uint64_t a128, uint64_t a32, uint64_t b128, uint64_t b32) {
-  using C = Cfg<D>;
+  using FA = typename Cfg<D>::A;
+  using FB = typename Cfg<D>::B;
 #pragma unroll
-  for (int i = 0; i < C::NB; ++i)
+  for (int i = 0; i < FA::NB; ++i)
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-      const uint64_t off = static_cast<uint64_t>(i * (kBlock128 >> 4) + k * 2);
-      mma_bf16_ss_pair(d, a128 + off, b128 + off, C::IDESC, (i | k) != 0);
+      const uint64_t oa = static_cast<uint64_t>(i * (FA::BLOCK >> 4) + k * 2);
+      const uint64_t ob = static_cast<uint64_t>(i * (FB::BLOCK >> 4) + k * 2);
+      mma_bf16_ss(d, a128 + oa, b128 + ob, Cfg<D>::IDESC, (i | k) != 0);
     }
 #pragma unroll
-  for (int r = 0; r < C::R; ++r) {
-    const uint64_t off = static_cast<uint64_t>(r * (kSlice32 >> 4));
-    mma_bf16_ss_pair(d, a32 + off, b32 + off, C::IDESC, (C::NB | r) != 0);
-  }
+  for (int r = 0; r < FA::R; ++r)
+    mma_bf16_ss(d, a32 + static_cast<uint64_t>(r * (FA::SLICE >> 4)), b32 + static_cast<uint64_t>(r * (FB::SLICE >> 4)),
+                Cfg<D>::IDESC, (FA::NB | r) != 0);
 }
 
 // 64 TMEM columns of this warp's 32 lanes -> v[0..63] (fp32 bit patterns), ready to use.
@@ -244,38 +296,25 @@ __device__ __forceinline__ void lse_fixed(const uint32_t (&v)[64], int valid, fl
   else lse_fixed64<false>(v, valid, c, m_run, l_run);
 }
 
-// Number of the 16 four-column steps of a 64-column chunk whose exp2 runs on the FMA pipe
-// (exp2_fma2) instead of the MUFU; the two pipes then share the work.
-constexpr int kPolySteps = 2;
-
-__device__ __forceinline__ constexpr bool poly_step(int k) { return (k * kPolySteps) % 16 < kPolySteps; }
-
-// acc += sum_e 2^(c s_e + nL_e) over 64 columns; nL (negated base-2 LSE) from shared memory.
-__device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], const float* nL, float c, float2 acc) {
+// acc += sum_e 2^(c a_e) over 64 columns, a_e = s_e - L / c straight from the MMA.
+__device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], float c, float2 acc) {
   const float2 cc = make_float2(c, c);
-  const float4* L4 = reinterpret_cast<const float4*>(nL);
-  float2 a1 = make_float2(0.f, 0.f);
+  const float2 zero = make_float2(0.f, 0.f);
+  float2 a1 = zero;
 #pragma unroll
   for (int e = 0; e < 64; e += 4) {
-    const float4 l = L4[e / 4];
-    const float2 x0 = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), cc, make_float2(l.x, l.y));
-    const float2 x1 =
-        ffma2(make_float2(__uint_as_float(v[e + 2]), __uint_as_float(v[e + 3])), cc, make_float2(l.z, l.w));
-    if (poly_step(e / 4)) {
-      acc = fadd2(acc, exp2_fma2(x0));
-      a1 = fadd2(a1, exp2_fma2(x1));
-    } else {
-      acc = fadd2(acc, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
-      a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
-    }
+    const float2 x0 = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), cc, zero);
+    const float2 x1 = ffma2(make_float2(__uint_as_float(v[e + 2]), __uint_as_float(v[e + 3])), cc, zero);
+    acc = fadd2(acc, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
+    a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
   }
   return fadd2(acc, a1);
 }
 
-// Brings the pair to a quiet point: waits for the pair's MMAs (phase `done_phase` of b_done),
-// lets in-flight copies land after an abort, and synchronises both CTAs; TMEM stays allocated.
-__device__ __forceinline__ void pair_quiesce(SmemCtl* ctl, uint32_t b_done, uint32_t done_phase, int* status,
-                                             int kernel) {
+// Brings the CTA to a quiet point: waits for its MMAs (phase `done_phase` of b_done) and lets
+// in-flight copies land after an abort; TMEM stays allocated.
+__device__ __forceinline__ void cta_quiesce(SmemCtl* ctl, uint32_t b_done, uint32_t done_phase, int* status,
+                                            int kernel) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   tc_fence_before_sync();
   __syncthreads();
@@ -287,23 +326,14 @@ __device__ __forceinline__ void pair_quiesce(SmemCtl* ctl, uint32_t b_done, uint
     while (globaltimer_ns() - t0 < 100000ull) {
     }
   }
-  __syncthreads();
   tc_fence_before_sync();
-  cluster_sync_all();
+  __syncthreads();
   tc_fence_after_sync();
 }
 
-// Releases the pair's TMEM with both CTAs in step (after pair_quiesce).
-__device__ __forceinline__ void pair_release_tmem(uint32_t tmem) {
-  if ((threadIdx.x >> 5) == 1) tmem_dealloc_pair(tmem, kTmemCols);
-  cluster_sync_all();
-}
-
-// Shared teardown: pair_quiesce, then TMEM release.
-__device__ __forceinline__ void pair_teardown(SmemCtl* ctl, uint32_t b_done, uint32_t tmem, int* status,
-                                              int kernel) {
-  pair_quiesce(ctl, b_done, 0, status, kernel);
-  pair_release_tmem(tmem);
+// Releases the CTA's TMEM (after cta_quiesce).
+__device__ __forceinline__ void cta_release_tmem(uint32_t tmem) {
+  if ((threadIdx.x >> 5) == 1) tmem_dealloc(tmem, kTmemCols);
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -315,24 +345,24 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
                                                             const __grid_constant__ CUtensorMap tmk,
                                                             const __grid_constant__ CUtensorMap tmk32,
                                                             const __grid_constant__ AttnTable t, float c,
-                                                            float* __restrict__ nL_out,
+                                                            uint16_t* __restrict__ shift_out,
                                                             float2* __restrict__ ml_out, int* status) {
   using C = Cfg<D>;
   constexpr int ST = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;                                // this CTA's resident query tile
-  uint8_t* sK = sQ + C::TILE_BYTES;                  // ST stages of this CTA's half of a key tile
-  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + ST * C::TILE_BYTES);
-  const uint32_t b_qfull = smem_u32(&ctl->bars[0]);     // even CTA: both Q halves landed
-  const uint32_t b_done = smem_u32(&ctl->bars[1]);      // both: all pair MMAs finished
-  auto b_kfull = [&](int s) { return smem_u32(&ctl->bars[2 + s]); };          // even CTA
-  auto b_kempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };    // both
-  auto b_sfull = [&](int p) { return smem_u32(&ctl->bars[2 + 2 * ST + p]); }; // both
-  auto b_sfree = [&](int p) { return smem_u32(&ctl->bars[4 + 2 * ST + p]); }; // even CTA
+  uint8_t* sK = sQ + C::A::BYTES;                    // ST stages of a key tile
+  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + ST * C::B::BYTES);
+  const uint32_t b_qfull = smem_u32(&ctl->bars[0]);     // query tile landed
+  const uint32_t b_done = smem_u32(&ctl->bars[1]);      // all MMAs of a round finished
+  auto b_kfull = [&](int s) { return smem_u32(&ctl->bars[2 + s]); };
+  auto b_kempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };
+  auto b_sfull = [&](int p) { return smem_u32(&ctl->bars[2 + 2 * ST + p]); };
+  auto b_sfree = [&](int p) { return smem_u32(&ctl->bars[4 + 2 * ST + p]); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t rank = cluster_ctarank();
+  const uint32_t rank = blockIdx.x & 1u;       // which 128-row half of the item
   const int item = blockIdx.x >> 1;
   const int b = find_image(t, item);
   int r = item - t.item_prefix[b];
@@ -343,7 +373,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
   const int h = r / npair;
   const int g = h / t.G;
   const int qrow0 = pair * kPair + kTile * static_cast<int>(rank);     // this CTA's first local query row
-  const int nkt_all = (t.nk[b] + kPair - 1) / kPair;
+  const int nkt_all = (t.nk[b] + kStream - 1) / kStream;
   const int kt0 = static_cast<int>((static_cast<int64_t>(split) * nkt_all) / t.splits);
   const int kt1 = static_cast<int>((static_cast<int64_t>(split + 1) * nkt_all) / t.splits);
   const int nj = kt1 - kt0;
@@ -357,22 +387,22 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
     }
     for (int p = 0; p < 2; ++p) {
       mbar_init(b_sfull(p), 1);
-      mbar_init(b_sfree(p), 2 * 8);
+      mbar_init(b_sfree(p), 8);   // the eight warps of warpgroup pair p
     }
     ctl->abort = 0;
     ctl->redo = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc_pair(smem_u32(&ctl->tmem_base), kTmemCols);
-    tmem_relinquish_pair();
+    tmem_alloc(smem_u32(&ctl->tmem_base), kTmemCols);
+    tmem_relinquish();
   }
   tc_fence_before_sync();
-  cluster_sync_all();
+  __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
 
-  // Round 0 uses the fixed-shift update; if any row of the pair overflowed it, round 1
+  // Round 0 uses the fixed-shift update; if any row of the CTA overflowed it, round 1
   // streams the keys again with the exact online-maximum update.  Stream tiles are counted
   // across rounds (it = round * nj + j), so every barrier keeps its phase sequence.
   const int e = (warp - 2) >> 2;            // epilogue warpgroup (warps 2..17)
@@ -382,15 +412,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&tmq);
     prefetch_tensormap(&tmk);
-    if (C::R > 0) {
+    if (C::A::R > 0) {
       prefetch_tensormap(&tmq32);
       prefetch_tensormap(&tmk32);
     }
-    // the even CTA's full barriers count the bytes of both halves; the odd CTA's copies
-    // complete there too
-    const uint32_t qfull_L = mapa_shared(b_qfull, 0);
-    if (rank == 0) mbar_arrive_expect_tx(b_qfull, 2 * C::TILE_BYTES);
-    load_tile<D>(sQ, &tmq, &tmq32, h * D, t.q0[b] + qrow0, qfull_L);
+    mbar_arrive_expect_tx(b_qfull, C::A::BYTES);
+    load_tile<D, kTile>(sQ, &tmq, &tmq32, h * D, t.q0[b] + qrow0, b_qfull);
   }
   auto run_round = [&](int round) {
     const int it0 = round * nj;
@@ -404,17 +431,15 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
             break;
           }
           if (aborted(ctl)) break;
-          const uint32_t kfull_L = mapa_shared(b_kfull(s), 0);
-          if (rank == 0) mbar_arrive_expect_tx(b_kfull(s), 2 * C::TILE_BYTES);
-          load_tile<D>(sK + s * C::TILE_BYTES, &tmk, &tmk32, g * D,
-                       t.k0[b] + (kt0 + j) * kPair + kTile * static_cast<int>(rank), kfull_L);
+          mbar_arrive_expect_tx(b_kfull(s), C::B::BYTES);
+          load_tile<D, kStream>(sK + s * C::B::BYTES, &tmk, &tmk32, g * D, t.k0[b] + (kt0 + j) * kStream, b_kfull(s));
         }
       }
     } else if (warp == 1) {
-      if (lane == 0 && rank == 0) {
+      if (lane == 0) {
         uint64_t aq128, aq32, bk128, bk32;
-        tile_desc<D>(sQ, aq128, aq32);
-        tile_desc<D>(sK, bk128, bk32);
+        tile_desc<D, kTile>(sQ, aq128, aq32);
+        tile_desc<D, kStream>(sK, bk128, bk32);
         const bool ok = mbar_wait(b_qfull, 0, kWaitLimitNs);
         if (!ok) set_abort(ctl, status, K_ATTN_ROW_LSE);
         for (int j = 0; ok && j < nj; ++j) {
@@ -427,18 +452,17 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
             break;
           }
           tc_fence_after_sync();
-          const uint64_t so = static_cast<uint64_t>(s * (C::TILE_BYTES >> 4));
+          const uint64_t so = static_cast<uint64_t>(s * (C::B::BYTES >> 4));
           mma_tile<D>(tmem + pa * 256, aq128, aq32, bk128 + so, bk32 + so);
-          mma_commit_pair_mc(b_sfull(pa), 3);
-          mma_commit_pair_mc(b_kempty(s), 3);
+          mma_commit(b_sfull(pa));
+          mma_commit(b_kempty(s));
         }
-        mma_commit_pair_mc(b_done, 3);
+        mma_commit(b_done);
       }
       __syncwarp();
     } else {
       // epilogue warpgroup e = 2p + hh: accumulator p (stream tiles it % 2 == p), columns hh * 128 ..
       float m_run = -INFINITY, l_run = 0.f;
-      const uint32_t sfree_L = mapa_shared(b_sfree(p), 0);
       const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
       for (int j = (p - it0) & 1; j < nj; j += 2) {
         const int it = it0 + j;
@@ -449,7 +473,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
           break;
         }
         tc_fence_after_sync();
-        const int valid = t.nk[b] - ((kt0 + j) * kPair + hh * kTile);   // keys of these columns in the image
+        const int valid = t.nk[b] - ((kt0 + j) * kStream + hh * 128);   // keys of these columns in the image
         uint32_t sv[64];
         load_cols64(tbuf, sv);
         if (round == 0) lse_fixed(sv, valid, c, m_run, l_run);
@@ -457,7 +481,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         load_cols64(tbuf + 64, sv);
         tc_fence_before_sync();
         __syncwarp();
-        if (lane == 0) mbar_arrive_remote(sfree_L);
+        if (lane == 0) mbar_arrive(b_sfree(p));
         if (round == 0) lse_fixed(sv, valid - 64, c, m_run, l_run);
         else if (valid > 64) lse_update64(sv, valid - 64, c, m_run, l_run);
       }
@@ -481,7 +505,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         const int row = qrow0 + rr;                       // local query row
         const int64_t prow = static_cast<int64_t>(h) * t.prows + t.lpad[b] + row;
         if (t.splits == 1) {
-          nL_out[prow] = row < t.nq[b] ? -(M + log2f(l)) : -INFINITY;
+          store_shift_row(shift_out + prow * kShiftCols, row < t.nq[b] ? -(M + log2f(l)) / c : -INFINITY);
         } else {
           ml_out[static_cast<int64_t>(split) * t.H * t.prows + prow] =
               (row < t.nq[b] && l > 0.f) ? make_float2(M, l) : make_float2(-INFINITY, 0.f);
@@ -491,23 +515,21 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
   };
 
   run_round(0);
-  pair_quiesce(ctl, b_done, 0, status, K_ATTN_ROW_LSE);
-  // If a row of either CTA overflowed the fixed shift, the pair streams the keys again with
-  // the exact update and overwrites its outputs (stream tiles continue at it = nj ..).
-  const uint32_t peer = rank ^ 1u;
-  const int redo_any = ctl->redo | static_cast<int>(ld_shared_cluster_u32(mapa_shared(smem_u32(&ctl->redo), peer)));
-  const int abort_any = ctl->abort | static_cast<int>(ld_shared_cluster_u32(mapa_shared(smem_u32(&ctl->abort), peer)));
-  if (redo_any != 0 && abort_any == 0) {
-    cluster_sync_all();   // both CTAs have read the flags before either one changes them
+  cta_quiesce(ctl, b_done, 0, status, K_ATTN_ROW_LSE);
+  // If a row overflowed the fixed shift, the CTA streams the keys again with the exact update
+  // and overwrites its outputs (stream tiles continue at it = nj ..).
+  if (ctl->redo != 0 && !aborted(ctl)) {
+    __syncthreads();   // every thread has read the flags before round 1 can change them
     run_round(1);
-    pair_quiesce(ctl, b_done, 1, status, K_ATTN_ROW_LSE);
+    cta_quiesce(ctl, b_done, 1, status, K_ATTN_ROW_LSE);
   }
-  pair_release_tmem(tmem);
+  cta_release_tmem(tmem);
 }
 
-// Merges per-split (m, l) pairs into -L = -(m + log2(l)); rows past the image get -inf.
-__global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ AttnTable t,
-                                                        const float2* __restrict__ ml, float* __restrict__ nL_out) {
+// Merges per-split (m, l) pairs into the shift row of -L / c, L = m + log2(l); rows past the
+// image get the padded-row shift.
+__global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ AttnTable t, float c,
+                                                        const float2* __restrict__ ml, uint16_t* __restrict__ shift_out) {
   // blockIdx.x = (image, 128-row tile of its padded rows) flattened
   int rem = blockIdx.x;
   const int h = blockIdx.y;
@@ -521,7 +543,7 @@ __global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ 
   const int row = rem * kTile + threadIdx.x;
   const int64_t prow = static_cast<int64_t>(h) * t.prows + t.lpad[b] + row;
   if (row >= t.nq[b]) {
-    nL_out[prow] = -INFINITY;
+    store_shift_row(shift_out + prow * kShiftCols, -INFINITY);
     return;
   }
   float M = -INFINITY;
@@ -531,7 +553,7 @@ __global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ 
     const float2 p = ml[static_cast<int64_t>(s) * t.H * t.prows + prow];
     if (p.y > 0.f) l += p.y * ex2_approx(p.x - M);
   }
-  nL_out[prow] = -(M + log2f(l));
+  store_shift_row(shift_out + prow * kShiftCols, -(M + log2f(l)) / c);
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -542,27 +564,28 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
                                                            const __grid_constant__ CUtensorMap tmq32,
                                                            const __grid_constant__ CUtensorMap tmk,
                                                            const __grid_constant__ CUtensorMap tmk32,
+                                                           const __grid_constant__ CUtensorMap tmshift,
+                                                           const __grid_constant__ CUtensorMap tmones,
                                                            const __grid_constant__ AttnTable t, float c,
-                                                           const float* __restrict__ nL, float* __restrict__ part,
-                                                           int* status) {
+                                                           float* __restrict__ part, int* status) {
   using C = Cfg<D>;
   constexpr int ST = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;                                 // this CTA's resident key tile
-  uint8_t* sQ = sA + C::TILE_BYTES;                   // ST stages of this CTA's half of a query tile
-  float* sL = reinterpret_cast<float*>(sQ + ST * C::TILE_BYTES);   // ST x 256 floats (-L of the whole tile)
-  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sL + ST * kPair);
-  const uint32_t b_afull = smem_u32(&ctl->bars[0]);     // even CTA
-  const uint32_t b_done = smem_u32(&ctl->bars[1]);      // both
-  auto b_qfull = [&](int s) { return smem_u32(&ctl->bars[2 + s]); };            // even CTA
-  auto b_qempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };      // both
-  auto b_lfull = [&](int s) { return smem_u32(&ctl->bars[2 + 2 * ST + s]); };   // both
-  auto b_sfull = [&](int p) { return smem_u32(&ctl->bars[2 + 3 * ST + p]); };   // both
-  auto b_sfree = [&](int p) { return smem_u32(&ctl->bars[4 + 3 * ST + p]); };   // even CTA
+  constexpr int A2 = C::A::BYTES + kTile * kShiftCols * 2;        // key tile + ones slice
+  constexpr int B2 = C::B::BYTES + kStream * kShiftCols * 2;      // query tile + shift slice
+  uint8_t* sQ = sA + A2;                               // ST stages of a query tile
+  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sQ + ST * B2);
+  const uint32_t b_afull = smem_u32(&ctl->bars[0]);
+  const uint32_t b_done = smem_u32(&ctl->bars[1]);
+  auto b_qfull = [&](int s) { return smem_u32(&ctl->bars[2 + s]); };
+  auto b_qempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };
+  auto b_sfull = [&](int p) { return smem_u32(&ctl->bars[2 + 2 * ST + p]); };
+  auto b_sfree = [&](int p) { return smem_u32(&ctl->bars[4 + 2 * ST + p]); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t rank = cluster_ctarank();
+  const uint32_t rank = blockIdx.x & 1u;       // which 128-row half of the item
   const int item = blockIdx.x >> 1;
   const int b = find_image(t, item);
   const int r = item - t.item_prefix[b];
@@ -570,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
   const int kp = r % nkp;
   const int g = r / nkp;
   const int krow0 = kp * kPair + kTile * static_cast<int>(rank);     // this CTA's first local key row
-  const int nqt = (t.nq[b] + kPair - 1) / kPair;
+  const int nqt = (t.nq[b] + kStream - 1) / kStream;
   const int nj = t.G * nqt;                                           // stream: (head in group, query tile)
 
   if (threadIdx.x == 0) {
@@ -578,22 +601,21 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
     mbar_init(b_done, 1);
     for (int s = 0; s < ST; ++s) {
       mbar_init(b_qfull(s), 1);
-      mbar_init(b_qempty(s), 1 + 8);   // pair MMA done + the 8 warps that read this stage's -L
-      mbar_init(b_lfull(s), 1);
+      mbar_init(b_qempty(s), 1);
     }
     for (int p = 0; p < 2; ++p) {
       mbar_init(b_sfull(p), 1);
-      mbar_init(b_sfree(p), 2 * 8);
+      mbar_init(b_sfree(p), 8);
     }
     ctl->abort = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc_pair(smem_u32(&ctl->tmem_base), kTmemCols);
-    tmem_relinquish_pair();
+    tmem_alloc(smem_u32(&ctl->tmem_base), kTmemCols);
+    tmem_relinquish();
   }
   tc_fence_before_sync();
-  cluster_sync_all();
+  __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
 
@@ -601,13 +623,14 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
     if (lane == 0) {
       prefetch_tensormap(&tmq);
       prefetch_tensormap(&tmk);
-      if (C::R > 0) {
+      if (C::A::R > 0) {
         prefetch_tensormap(&tmq32);
         prefetch_tensormap(&tmk32);
       }
-      const uint32_t afull_L = mapa_shared(b_afull, 0);
-      if (rank == 0) mbar_arrive_expect_tx(b_afull, 2 * C::TILE_BYTES);
-      load_tile<D>(sA, &tmk, &tmk32, g * D, t.k0[b] + krow0, afull_L);
+      prefetch_tensormap(&tmshift);
+      mbar_arrive_expect_tx(b_afull, A2);
+      load_tile<D, kTile>(sA, &tmk, &tmk32, g * D, t.k0[b] + krow0, b_afull);
+      tma_load_2d(smem_u32(sA + C::A::BYTES), &tmones, 0, 0, b_afull);
       for (int j = 0; j < nj; ++j) {
         const int s = j % ST, u = j / ST;
         if (u > 0 && !mbar_wait(b_qempty(s), (u - 1) & 1, kWaitLimitNs)) {
@@ -617,20 +640,23 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
         if (aborted(ctl)) break;
         const int hq = j / nqt, qt = j - hq * nqt;
         const int h = g * t.G + hq;
-        const uint32_t qfull_L = mapa_shared(b_qfull(s), 0);
-        if (rank == 0) mbar_arrive_expect_tx(b_qfull(s), 2 * C::TILE_BYTES);
-        load_tile<D>(sQ + s * C::TILE_BYTES, &tmq, &tmq32, h * D,
-                     t.q0[b] + qt * kPair + kTile * static_cast<int>(rank), qfull_L);
-        mbar_arrive_expect_tx(b_lfull(s), kPair * 4);
-        bulk_load(smem_u32(sL + s * kPair), nL + static_cast<int64_t>(h) * t.prows + t.lpad[b] + qt * kPair,
-                  kPair * 4, b_lfull(s));
+        uint8_t* st = sQ + s * B2;
+        mbar_arrive_expect_tx(b_qfull(s), B2);
+        load_tile<D, kStream>(st, &tmq, &tmq32, h * D, t.q0[b] + qt * kStream, b_qfull(s));
+        const int srow = h * t.prows + t.lpad[b] + qt * kStream;
+#pragma unroll
+        for (int q = 0; q < kStream / kTile; ++q)
+          tma_load_2d(smem_u32(st + C::B::BYTES + q * kTile * kShiftCols * 2), &tmshift, 0, srow + q * kTile,
+                      b_qfull(s));
       }
     }
   } else if (warp == 1) {
-    if (lane == 0 && rank == 0) {
+    if (lane == 0) {
       uint64_t ak128, ak32, bq128, bq32;
-      tile_desc<D>(sA, ak128, ak32);
-      tile_desc<D>(sQ, bq128, bq32);
+      tile_desc<D, kTile>(sA, ak128, ak32);
+      tile_desc<D, kStream>(sQ, bq128, bq32);
+      const uint64_t aone = smem_desc_kmajor_sw32(smem_u32(sA + C::A::BYTES));
+      const uint64_t bshift = smem_desc_kmajor_sw32(smem_u32(sQ + C::B::BYTES));
       bool ok = mbar_wait(b_afull, 0, kWaitLimitNs);
       if (!ok) set_abort(ctl, status, K_ATTN_COLSUM);
       for (int j = 0; ok && j < nj; ++j) {
@@ -642,12 +668,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
           break;
         }
         tc_fence_after_sync();
-        const uint64_t so = static_cast<uint64_t>(s * (C::TILE_BYTES >> 4));
+        const uint64_t so = static_cast<uint64_t>(s * (B2 >> 4));
         mma_tile<D>(tmem + p * 256, ak128, ak32, bq128 + so, bq32 + so);
-        mma_commit_pair_mc(b_sfull(p), 3);
-        mma_commit_pair_mc(b_qempty(s), 3);
+        mma_bf16_ss(tmem + p * 256, aone, bshift + so, C::IDESC, 1);   // + (-L_i / c)
+        mma_commit(b_sfull(p));
+        mma_commit(b_qempty(s));
       }
-      mma_commit_pair_mc(b_done, 3);
+      mma_commit(b_done);
     }
     __syncwarp();
   } else {
@@ -656,30 +683,24 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
     const int p = e >> 1, hh = e & 1;
     const int quad = warp & 3;
     const int rr = quad * 32 + lane;
-    const uint32_t sfree_L = mapa_shared(b_sfree(p), 0);
     float2 acc = make_float2(0.f, 0.f);
     const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
     for (int j = p; j < nj; j += 2) {
       const int v = j >> 1;
-      const int s = j % ST, u = j / ST;
-      const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs) &&
-                                                  mbar_wait(b_lfull(s), u & 1, kWaitLimitNs));
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs));
       if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
         set_abort(ctl, status, K_ATTN_COLSUM);
         break;
       }
       tc_fence_after_sync();
-      const float* Ls = sL + s * kPair + hh * kTile;
       uint32_t sv[64];
       load_cols64(tbuf, sv);
-      acc = colsum64(sv, Ls, c, acc);
+      acc = colsum64(sv, c, acc);
       load_cols64(tbuf + 64, sv);
       tc_fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive_remote(sfree_L);
-      acc = colsum64(sv, Ls + 64, c, acc);
-      __syncwarp();
-      if (lane == 0) mbar_arrive(b_qempty(s));
+      if (lane == 0) mbar_arrive(b_sfree(p));
+      acc = colsum64(sv, c, acc);
     }
     const float a = acc.x + acc.y;
     if (e > 0) ctl->xchg[e - 1][0][rr] = a;
@@ -691,7 +712,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
             (a + ctl->xchg[0][0][rr]) + (ctl->xchg[1][0][rr] + ctl->xchg[2][0][rr]);
     }
   }
-  pair_teardown(ctl, b_done, tmem, status, K_ATTN_COLSUM);
+  cta_quiesce(ctl, b_done, 0, status, K_ATTN_COLSUM);
+  cta_release_tmem(tmem);
 }
 
 // out[m] = sum over groups and the `merge` rows of token m of part[group][row].
@@ -749,14 +771,14 @@ struct AttnLayout {
   size_t L_off, part_off, ml_off, total;
 };
 
-// Key splits of pass 1: enough CTA pairs to cover the GPU about twice.
+// Key splits of pass 1: enough work items to cover the GPU about twice.
 int choose_splits(int B, const int32_t* cu_q, const int32_t* cu_k, int H) {
   int64_t items = 0;
   int max_kt = 1;
   for (int b = 0; b < B; ++b) {
     const int nq = cu_q[b + 1] - cu_q[b], nk = cu_k[b + 1] - cu_k[b];
     items += static_cast<int64_t>(H) * ((nq + kPair - 1) / kPair);
-    max_kt = std::max(max_kt, (nk + kPair - 1) / kPair);
+    max_kt = std::max(max_kt, (nk + kStream - 1) / kStream);
   }
   if (items >= kTargetItems || items == 0) return 1;
   int s = static_cast<int>((kTargetItems + items - 1) / items);
@@ -773,7 +795,7 @@ AttnLayout attn_layout(int B, const int32_t* cu_q, const int32_t* cu_k, int H, i
   for (int b = 0; b < B; ++b) pr += static_cast<int64_t>((cu_q[b + 1] - cu_q[b] + kPair - 1) / kPair) * kPair;
   L.prows = pr;   // every image's L rows start on a 256-row (1 KB) boundary
   L.L_off = 0;
-  L.part_off = align_up(static_cast<size_t>(H) * L.prows * sizeof(float), 256);
+  L.part_off = align_up(static_cast<size_t>(H) * L.prows * kShiftCols * 2, 256);
   L.ml_off = L.part_off + align_up(static_cast<size_t>(groups) * L.ktot * sizeof(float), 256);
   L.total = L.ml_off;
   if (L.splits > 1) L.total += align_up(static_cast<size_t>(L.splits) * H * L.prows * sizeof(float2), 256);
@@ -794,8 +816,9 @@ pace_status_t check_segments(int B, const int32_t* cu, int multiple) {
 template <int D>
 pace_status_t set_smem_attrs(size_t* s1, size_t* s2) {
   using C = Cfg<D>;
-  *s1 = 1024 + C::TILE_BYTES + C::STAGES * C::TILE_BYTES + sizeof(SmemCtl);
-  *s2 = 1024 + C::TILE_BYTES + C::STAGES * C::TILE_BYTES + C::STAGES * kPair * 4 + sizeof(SmemCtl);
+  *s1 = 1024 + C::A::BYTES + C::STAGES * C::B::BYTES + sizeof(SmemCtl);
+  *s2 = 1024 + C::A::BYTES + kTile * kShiftCols * 2 + C::STAGES * (C::B::BYTES + kStream * kShiftCols * 2) +
+        sizeof(SmemCtl);
   static std::atomic<uint64_t> done{0};
   int dev = 0;
   PACE_CUDA(cudaGetDevice(&dev));
@@ -807,23 +830,11 @@ pace_status_t set_smem_attrs(size_t* s1, size_t* s2) {
   return PACE_OK;
 }
 
-// Launches `items` CTA pairs (clusters of two CTAs along x).
+// Launches `items` work items of two independent CTAs each.
 template <typename... Params, typename... Args>
 pace_status_t launch_pairs(void (*kernel)(Params...), int items, size_t smem, cudaStream_t stream, Args... args) {
   if (items <= 0) return PACE_OK;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(2 * static_cast<unsigned>(items));
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  PACE_CUDA(cudaLaunchKernelEx(&cfg, kernel, args...));
+  kernel<<<dim3(2 * static_cast<unsigned>(items)), dim3(kThreads), smem, stream>>>(args...);
   return check_launch();
 }
 
@@ -833,7 +844,7 @@ pace_status_t run_importance(const void* Q, const void* K, const int32_t* cu_q, 
   const int G = Hq / Hkv;
   const AttnLayout Lay = attn_layout(B, cu_q, cu_k, Hq, Hkv);
   uint8_t* w8 = static_cast<uint8_t*>(ws);
-  float* Lw = reinterpret_cast<float*>(w8 + Lay.L_off);
+  uint16_t* Lw = reinterpret_cast<uint16_t*>(w8 + Lay.L_off);
   float* part = reinterpret_cast<float*>(w8 + Lay.part_off);
   float2* ml = Lay.splits > 1 ? reinterpret_cast<float2*>(w8 + Lay.ml_off) : nullptr;
   int* status = device_status_word();
@@ -843,6 +854,11 @@ pace_status_t run_importance(const void* Q, const void* K, const int32_t* cu_q, 
   PACE_CHECK(make_map(&mk, K, krows, static_cast<int64_t>(Hkv) * D, true));
   PACE_CHECK(make_map(&mq32, Q, qrows, static_cast<int64_t>(Hq) * D, false));
   PACE_CHECK(make_map(&mk32, K, krows, static_cast<int64_t>(Hkv) * D, false));
+  CUtensorMap mshift, mones;
+  PACE_CHECK(make_map(&mshift, Lw, static_cast<int64_t>(Hq) * Lay.prows, kShiftCols, false));
+  const void* ones = nullptr;
+  PACE_CUDA(cudaGetSymbolAddress(const_cast<void**>(&ones), g_ones_slice));
+  PACE_CHECK(make_map(&mones, ones, kTile, kShiftCols, false));
   size_t s1 = 0, s2 = 0;
   PACE_CHECK(set_smem_attrs<D>(&s1, &s2));
   const float c = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634);
@@ -872,7 +888,7 @@ pace_status_t run_importance(const void* Q, const void* K, const int32_t* cu_q, 
     }
     PACE_CHECK(launch_pairs(attn_row_lse<D>, items1, s1, stream, mq, mq32, mk, mk32, t, c, Lw, ml, status));
     if (Lay.splits > 1) {
-      attn_lse_combine<<<dim3(ctiles, Hq), kTile, 0, stream>>>(t, ml, Lw);
+      attn_lse_combine<<<dim3(ctiles, Hq), kTile, 0, stream>>>(t, c, ml, Lw);
       PACE_CHECK(check_launch());
     }
     int items2 = 0;
@@ -880,8 +896,8 @@ pace_status_t run_importance(const void* Q, const void* K, const int32_t* cu_q, 
       items2 += Hkv * ((t.nk[i] + kPair - 1) / kPair);
       t.item_prefix[i + 1] = items2;
     }
-    PACE_CHECK(launch_pairs(attn_colsum<D>, items2, s2, stream, mq, mq32, mk, mk32, t, c,
-                            static_cast<const float*>(Lw), part, status));
+    PACE_CHECK(launch_pairs(attn_colsum<D>, items2, s2, stream, mq, mq32, mk, mk32, mshift, mones, t, c, part,
+                            status));
   }
   const int nout = static_cast<int>(Lay.ktot / merge);
   attn_reduce<<<(nout + 255) / 256, 256, 0, stream>>>(part, Hkv, static_cast<int>(Lay.ktot), merge, out);
