@@ -13,9 +13,9 @@
 //              the staged pixels (no 2 - 2cos cancellation).
 //   apc_tail   one CTA per image: radix select of the k_tail-th largest d_i (fp32 bits),
 //              tail mean, rho_d, rho, r and the target size.
-// Resize: apc_resample, one CTA per 32 x 64 output tile; for downscales up to 2.75x per side
-// the input window is staged in shared memory and filtered there with precomputed weights,
-// steeper downscales take a generic path with per-tap weights.
+// Resize: apc_resample, four CTAs per SM walking the 16 x 32 output tiles of the batch; for
+// downscales up to 2.75x per side the input window is staged in shared memory and filtered
+// there with precomputed weights, steeper downscales take a generic path with per-tap weights.
 #include <algorithm>
 #include <atomic>
 #include <cfloat>
@@ -332,9 +332,10 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
 // ------------------------------------------------------------------------------------------------
 // resample
 // ------------------------------------------------------------------------------------------------
-constexpr int kRsTH = 8;    // output rows per CTA
-constexpr int kRsTW = 32;   // output columns per CTA
-constexpr int kRsChunk = 8; // input rows filtered per step
+constexpr int kRsThreads = 128;  // threads of a resample CTA
+constexpr int kRsTH = 4;         // output rows of a generic tile (kRsTH x kRsTW = kRsThreads)
+constexpr int kRsTW = 32;        // output columns of a generic tile
+constexpr int kRsChunk = 8;      // input rows filtered per step of the generic path
 
 struct ResampleTable {
   int64_t src_off[kApcMaxB];
@@ -355,27 +356,49 @@ __device__ __forceinline__ float cubic_w(float t) {
   return 0.0f;
 }
 
-// Window [lo, lo + n) of taps for output index o, the tap offset of lo, 1/fs, 1/sum(weights).
-__device__ __forceinline__ void window_1d(int o, int n_in, int n_out, int& lo, int& n, float& off0, float& ifs,
-                                          float& inorm) {
-  const double scale = static_cast<double>(n_in) / n_out;
-  const double fs = scale > 1.0 ? scale : 1.0;
-  const double support = 2.0 * fs;
-  const double centre = (o + 0.5) * scale;
-  int a = static_cast<int>(floor(centre - support));
-  int e = static_cast<int>(ceil(centre + support));
+__device__ __forceinline__ int64_t floor_div(int64_t x, int64_t d) { return x >= 0 ? x / d : -((-x + d - 1) / d); }
+__device__ __forceinline__ int64_t ceil_div(int64_t x, int64_t d) { return x >= 0 ? (x + d - 1) / d : -((-x) / d); }
+
+// Window of output index o (reading R5) in exact integer arithmetic.  With s = n_in / n_out
+// and fs = max(s, 1), the centre is c = (2o + 1) n_in / (2 n_out), the taps are
+// lo .. lo + n - 1 with lo = max(0, floor(c - 2 fs)) and lo + n = min(n_in, ceil(c + 2 fs)),
+// and tap i sits at (lo + i + 0.5 - c) / fs = (num0 + i * step) * inv_den with integer
+// num0 = (2 lo + 1) n_out - (2o + 1) n_in, step = 2 n_out and den = 2 n_out fs.
+struct Win {
+  int lo, n, num0, step;
+  float inv_den;
+};
+__device__ __forceinline__ Win exact_window(int o, int n_in, int n_out) {
+  const bool down = n_in > n_out;
+  const int64_t cn = (2 * static_cast<int64_t>(o) + 1) * n_in;                   // c * 2 n_out
+  const int64_t sup = 4 * static_cast<int64_t>(down ? n_in : n_out);           // 2 fs * 2 n_out
+  const int64_t d = 2 * static_cast<int64_t>(n_out);
+  int64_t a = floor_div(cn - sup, d), e = ceil_div(cn + sup, d);
   if (a < 0) a = 0;
   if (e > n_in) e = n_in;
-  lo = a;
-  n = e - a;
-  off0 = static_cast<float>((a + 0.5 - centre) / fs);
-  ifs = static_cast<float>(1.0 / fs);
+  Win w;
+  w.lo = static_cast<int>(a);
+  w.n = static_cast<int>(e - a);
+  w.num0 = static_cast<int>((2 * a + 1) * n_out - cn);
+  w.step = 2 * n_out;
+  w.inv_den = 1.0f / static_cast<float>(down ? 2 * n_in : 2 * n_out);
+  return w;
+}
+
+// Window [lo, lo + n) of taps for output index o, the tap offset of lo, its step, 1/sum(weights).
+__device__ __forceinline__ void window_1d(int o, int n_in, int n_out, int& lo, int& n, float& off0, float& ifs,
+                                          float& inorm) {
+  const Win w = exact_window(o, n_in, n_out);
+  lo = w.lo;
+  n = w.n;
+  off0 = static_cast<float>(w.num0) * w.inv_den;
+  ifs = static_cast<float>(w.step) * w.inv_den;
   float s = 0.f;
-  for (int i = 0; i < n; ++i) s += cubic_w(fmaf(static_cast<float>(i), ifs, off0));
+  for (int i = 0; i < n; ++i) s += cubic_w(static_cast<float>(w.num0 + i * w.step) * w.inv_den);
   inorm = 1.0f / s;
 }
 
-// Any downscale: one 8 x 32 output tile, weights evaluated per tap, input read through L1.
+// Any downscale: one 4 x 32 output tile, weights evaluated per tap, input read through L1.
 __device__ void resample_tile_generic(const uint8_t* __restrict__ img, int H, int W, int Ho, int Wo, int ox0,
                                       int oy0, uint8_t* __restrict__ out) {
   __shared__ int xlo[kRsTW], xn[kRsTW];
@@ -403,7 +426,7 @@ __device__ void resample_tile_generic(const uint8_t* __restrict__ img, int H, in
   float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f;
   for (int r0 = iy_lo; r0 < iy_hi; r0 += kRsChunk) {
     // horizontal pass: kRsChunk rows x 32 columns x 3 channels
-    for (int v = tid; v < kRsChunk * kRsTW * 3; v += 256) {
+    for (int v = tid; v < kRsChunk * kRsTW * 3; v += kRsThreads) {
       const int rr = v / (kRsTW * 3), rem = v - rr * (kRsTW * 3);
       const int cc = rem / 3, ch = rem - cc * 3;
       const int iy = r0 + rr;
@@ -445,75 +468,56 @@ __device__ void resample_tile_generic(const uint8_t* __restrict__ img, int H, in
   __syncthreads();   // shared tile buffers are reused by the next call
 }
 
-// Downscale of at most kFMaxScale per side: one 32 x 64 output tile.  The CTA stages its whole
+// Downscale of at most 2.75 per side: one 16 x 32 output tile.  The CTA stages its whole
 // input window in shared memory with 4-byte loads (every image starts 16-byte aligned and
-// holds a multiple of 4 bytes, so the rounded loads stay inside it), precomputes the
-// normalised tap weights of its rows and columns once, then runs the horizontal pass into a
-// shared fp32 buffer and the vertical pass from there.
-constexpr int kFTH = 32, kFTW = 64, kFMaxTaps = 14;
-constexpr double kFMaxScale = 2.75;
-constexpr int kFRows = 102;                  // >= 32 * 2.75 + 14 staged input rows
-constexpr int kFCols = 190;                  // >= 64 * 2.75 + 14 staged input pixels per row
-constexpr int kFPitch = 576;                 // bytes per staged row: 3 * kFCols + 3 alignment slack, rounded
-static_assert(kFPitch >= 3 * kFCols + 6, "staged row pitch");
-static_assert(kFRows >= 32 * 2.75 + 14 && kFCols >= 64 * 2.75 + 14, "staged window");
-constexpr size_t kFSmem = static_cast<size_t>(kFRows) * kFPitch + static_cast<size_t>(kFRows) * kFTW * 3 * 4 +
+// holds a multiple of 4 bytes, so the rounded loads stay inside it) and precomputes the
+// normalised tap weights of its rows and columns; thread (column, channel) keeps its column's
+// weights in registers, filters every staged row horizontally into a shared fp32 buffer and
+// then its output column vertically.
+constexpr int kFTH = 16, kFTW = 32, kFMaxTaps = 14;
+// the fast path takes downscales of at most 2.75 = 11 / 4 per side (tested as 4 n_in <= 11 n_out)
+constexpr int kFRows = 58;                   // >= 16 * 2.75 + 14 staged input rows
+constexpr int kFCols = 118;                  // >= 32 * 2.75 + 14 window pixels + 14 read past it (weight 0)
+constexpr int kFPitch = 368;                 // bytes per staged row: 3 * kFCols + 3 alignment slack, rounded
+constexpr int kFLine = kFTW * 3;             // floats per row of the horizontal result
+static_assert(kFPitch >= 3 * kFCols + 6 && kFPitch % 16 == 0, "staged row pitch");
+static_assert(kFRows >= kFTH * 2.75 + 14 && kFCols >= kFTW * 2.75 + 14 + kFMaxTaps, "staged window");
+static_assert(3 * kFTW <= kRsThreads && 64 + kFTH <= kRsThreads, "thread roles of the fast tile");
+constexpr size_t kFSmem = static_cast<size_t>(kFRows) * kFPitch + static_cast<size_t>(kFRows) * kFLine * 4 +
                           (kFTW + kFTH) * kFMaxTaps * 4 + (2 * kFTW + 2 * kFTH + kFRows + 4) * 4;
+constexpr int kRsCtasPerSm = 4;
 
 // Normalised weights of the window of output index o (reading R5); returns the tap count.
 __device__ __forceinline__ int window_weights(int o, int n_in, int n_out, int& lo, float* w) {
-  const double scale = static_cast<double>(n_in) / n_out;
-  const double fs = scale > 1.0 ? scale : 1.0;
-  const double centre = (o + 0.5) * scale;
-  int a = static_cast<int>(floor(centre - 2.0 * fs));
-  int e = static_cast<int>(ceil(centre + 2.0 * fs));
-  if (a < 0) a = 0;
-  if (e > n_in) e = n_in;
-  const int n = e - a;
-  if (n > kFMaxTaps) return n;
-  const float off0 = static_cast<float>((a + 0.5 - centre) / fs), ifs = static_cast<float>(1.0 / fs);
+  const Win win = exact_window(o, n_in, n_out);
+  if (win.n > kFMaxTaps) return win.n;
   float sum = 0.f;
-  for (int i = 0; i < n; ++i) {
-    w[i] = cubic_w(fmaf(static_cast<float>(i), ifs, off0));
+  for (int i = 0; i < win.n; ++i) {
+    w[i] = cubic_w(static_cast<float>(win.num0 + i * win.step) * win.inv_den);
     sum += w[i];
   }
   const float inv = 1.0f / sum;
-  for (int i = 0; i < n; ++i) w[i] *= inv;
-  lo = a;
-  return n;
+  for (int i = 0; i < win.n; ++i) w[i] *= inv;
+  lo = win.lo;
+  return win.n;
 }
 
-__global__ void __launch_bounds__(256) apc_resample(const uint8_t* __restrict__ src,
-                                                    const __grid_constant__ ResampleTable t,
-                                                    const pace_apc_stats* __restrict__ stats,
-                                                    uint8_t* __restrict__ dst) {
+template <int MAXT>
+__device__ __forceinline__ void resample_tile_fast(const uint8_t* __restrict__ img, int H, int W, int Ho, int Wo,
+                                                   int ox0, int oy0, uint8_t* __restrict__ out) {
   extern __shared__ __align__(16) unsigned char rs_smem[];
-  const int b = blockIdx.z;
-  const int H = t.H[b], W = t.W[b];
-  const int Ho = stats ? stats[t.b_base + b].h_out : t.Ho[b];
-  const int Wo = stats ? stats[t.b_base + b].w_out : t.Wo[b];
-  const int ox0 = blockIdx.x * kFTW, oy0 = blockIdx.y * kFTH;
-  if (ox0 >= Wo || oy0 >= Ho || Ho < 1 || Wo < 1 || Ho > H || Wo > W) return;
-  const uint8_t* img = src + t.src_off[b];
-  uint8_t* out = dst + t.dst_off[b];
-  const int tid = threadIdx.x;
-  const bool fast = static_cast<double>(W) / Wo <= kFMaxScale && static_cast<double>(H) / Ho <= kFMaxScale;
-  if (!fast) {
-    for (int sy = 0; sy < kFTH; sy += kRsTH)
-      for (int sx = 0; sx < kFTW; sx += kRsTW) resample_tile_generic(img, H, W, Ho, Wo, ox0 + sx, oy0 + sy, out);
-    return;
-  }
   unsigned char* sin = rs_smem;                                           // [kFRows][kFPitch] bytes
-  float* sh = reinterpret_cast<float*>(sin + kFRows * kFPitch);            // [kFRows][kFTW][3]
-  float* wx = sh + kFRows * kFTW * 3;                                     // [kFTW][kFMaxTaps]
+  float* sh = reinterpret_cast<float*>(sin + kFRows * kFPitch);            // [kFRows][kFTW * 3]
+  float* wx = sh + kFRows * kFLine;                                        // [kFTW][kFMaxTaps]
   float* wy = wx + kFTW * kFMaxTaps;                                       // [kFTH][kFMaxTaps]
   int* xlo = reinterpret_cast<int*>(wy + kFTH * kFMaxTaps);
   int* xn = xlo + kFTW;
   int* ylo = xn + kFTW;
   int* yn = ylo + kFTH;
   int* shift = yn + kFTH;                                                  // [kFRows]
+  const int tid = threadIdx.x;
   const int ncol = min(kFTW, Wo - ox0), nrow = min(kFTH, Ho - oy0);
-  // with both scales <= kFMaxScale every window has <= 4 * 2.75 + 2 = 13 taps (min() is a guard)
+  // with both scales <= 2.75 every window has <= 4 * 2.75 + 2 = 13 taps (min() is a guard)
   if (tid < ncol) xn[tid] = min(kFMaxTaps, window_weights(ox0 + tid, W, Wo, xlo[tid], wx + tid * kFMaxTaps));
   if (tid >= 64 && tid < 64 + nrow)
     yn[tid - 64] =
@@ -525,7 +529,7 @@ __global__ void __launch_bounds__(256) apc_resample(const uint8_t* __restrict__ 
   // stage the input window (4-byte words covering each row segment)
   const int64_t pitch = static_cast<int64_t>(W) * 3;
   const int words = (nin_c * 3 + 3 + 3) >> 2;
-  for (int i = tid; i < nin_r * words; i += 256) {
+  for (int i = tid; i < nin_r * words; i += kRsThreads) {
     const int r = i / words, w = i - r * words;
     const int64_t start = (static_cast<int64_t>(y0 + r) * pitch + static_cast<int64_t>(x0) * 3);
     const int64_t a = start & ~int64_t{3};
@@ -535,27 +539,79 @@ __global__ void __launch_bounds__(256) apc_resample(const uint8_t* __restrict__ 
       *reinterpret_cast<uint32_t*>(sin + r * kFPitch + 4 * w) = __ldg(reinterpret_cast<const uint32_t*>(img + byte));
   }
   __syncthreads();
-  // horizontal pass: staged rows x output columns x channels
-  for (int i = tid; i < nin_r * ncol * 3; i += 256) {
-    const int ch = i % 3, rc = i / 3;
-    const int c = rc % ncol, r = rc / ncol;
-    const unsigned char* px = sin + r * kFPitch + shift[r] + (xlo[c] - x0) * 3 + ch;
-    const float* w = wx + c * kFMaxTaps;
-    float acc = 0.f;
-    for (int k = 0; k < xn[c]; ++k) acc = fmaf(w[k], static_cast<float>(px[3 * k]), acc);
-    sh[(r * kFTW + c) * 3 + ch] = acc;
+  if (tid < 3 * ncol) {
+    // horizontal pass: every staged row, this thread's (column, channel)
+    // (taps past the window have weight 0 and read staged bytes that exist: the staged row
+    // holds kFCols >= the window of the last column + MAXT pixels)
+    const int c = tid / 3, ch = tid - 3 * c;
+    const int n = xn[c];
+    float w[MAXT];
+#pragma unroll
+    for (int k = 0; k < MAXT; ++k) w[k] = k < n ? wx[c * kFMaxTaps + k] : 0.f;
+    const int base = (xlo[c] - x0) * 3 + ch;
+    for (int r = 0; r < nin_r; ++r) {
+      const unsigned char* px = sin + r * kFPitch + shift[r] + base;
+      float acc = 0.f;
+#pragma unroll
+      for (int k = 0; k < MAXT; ++k) acc = fmaf(w[k], byte_to_float(px[3 * k]), acc);
+      sh[r * kFLine + tid] = acc;
+    }
   }
   __syncthreads();
-  // vertical pass and the uint8 store
-  for (int i = tid; i < nrow * ncol * 3; i += 256) {
-    const int ch = i % 3, rc = i / 3;
-    const int c = rc % ncol, r = rc / ncol;
-    const float* w = wy + r * kFMaxTaps;
-    const float* col = sh + ((ylo[r] - y0) * kFTW + c) * 3 + ch;
-    float acc = 0.f;
-    for (int k = 0; k < yn[r]; ++k) acc = fmaf(w[k], col[k * kFTW * 3], acc);
-    out[(static_cast<int64_t>(oy0 + r) * Wo + ox0 + c) * 3 + ch] =
-        static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc))));
+  if (tid < 3 * ncol) {
+    // vertical pass and the uint8 store (a row of the tile is 3 * ncol consecutive bytes)
+    uint8_t* o = out + (static_cast<int64_t>(oy0) * Wo + ox0) * 3 + tid;
+    for (int r = 0; r < nrow; ++r) {
+      const float* w = wy + r * kFMaxTaps;
+      const float* col = sh + (ylo[r] - y0) * kFLine + tid;
+      const int n = yn[r];
+      float acc = 0.f;
+      for (int k = 0; k < n; ++k) acc = fmaf(w[k], col[k * kFLine], acc);
+      o[static_cast<int64_t>(r) * Wo * 3] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc))));
+    }
+  }
+  __syncthreads();   // the shared buffers are reused by the next tile
+}
+
+// Every CTA walks the output tiles of the whole batch (16 x 32 tiles; target sizes read from
+// the density statistics on the device, or given), so the grid never holds empty CTAs.
+__global__ void __launch_bounds__(kRsThreads) apc_resample(const uint8_t* __restrict__ src,
+                                                           const __grid_constant__ ResampleTable t,
+                                                           const pace_apc_stats* __restrict__ stats,
+                                                           uint8_t* __restrict__ dst) {
+  __shared__ int tile_prefix[kApcMaxB + 1];
+  __shared__ int sho[kApcMaxB], swo[kApcMaxB];
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int b = 0; b < t.nb; ++b) {
+      int Ho = stats ? stats[t.b_base + b].h_out : t.Ho[b];
+      int Wo = stats ? stats[t.b_base + b].w_out : t.Wo[b];
+      if (Ho < 1 || Wo < 1 || Ho > t.H[b] || Wo > t.W[b]) Ho = Wo = 0;   // nothing to write
+      sho[b] = Ho;
+      swo[b] = Wo;
+      tile_prefix[b] = acc;
+      acc += ((Ho + kFTH - 1) / kFTH) * ((Wo + kFTW - 1) / kFTW);
+    }
+    tile_prefix[t.nb] = acc;
+  }
+  __syncthreads();
+  const int total = tile_prefix[t.nb];
+  for (int g = blockIdx.x; g < total; g += gridDim.x) {
+    int b = 0;
+    while (b + 1 < t.nb && tile_prefix[b + 1] <= g) ++b;
+    const int Ho = sho[b], Wo = swo[b], H = t.H[b], W = t.W[b];
+    const int tw = (Wo + kFTW - 1) / kFTW;
+    const int l = g - tile_prefix[b];
+    const int oy0 = (l / tw) * kFTH, ox0 = (l - (l / tw) * tw) * kFTW;
+    const uint8_t* img = src + t.src_off[b];
+    uint8_t* out = dst + t.dst_off[b];
+    if (4 * W <= 11 * Wo && 4 * H <= 11 * Ho) {   // both scales <= 2.75 = 11 / 4
+      if (4 * W <= 9 * Wo && 4 * H <= 9 * Ho) resample_tile_fast<10>(img, H, W, Ho, Wo, ox0, oy0, out);   // <= 10 taps
+      else resample_tile_fast<kFMaxTaps>(img, H, W, Ho, Wo, ox0, oy0, out);
+    } else {
+        for (int sy = 0; sy < kFTH; sy += kRsTH)
+        for (int sx = 0; sx < kFTW; sx += kRsTW) resample_tile_generic(img, H, W, Ho, Wo, ox0 + sx, oy0 + sy, out);
+    }
   }
 }
 
@@ -697,16 +753,23 @@ static pace_status_t resample_impl(const uint8_t* src, const int64_t* src_off, c
   for (int b = 0; b < B; ++b)
     if (dst_off[b] < 0) return PACE_ERR_INVALID_ARG;
   PACE_CHECK(check_device());
+  int sms = 1;
   {
-    static std::atomic<uint64_t> done{0};   // opt in to the fast path's shared memory once per device
+    // opt in to the fast path's shared memory and read the SM count, once per device
+    static std::atomic<uint64_t> done{0};
+    static std::atomic<int> sm_count[64];
     int dev = 0;
     PACE_CUDA(cudaGetDevice(&dev));
     const uint64_t bit = uint64_t{1} << (dev & 63);
     if (!(done.load(std::memory_order_acquire) & bit)) {
+      int n = 0;
+      PACE_CUDA(cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev));
+      sm_count[dev & 63].store(n, std::memory_order_relaxed);
       PACE_CUDA(cudaFuncSetAttribute(apc_resample, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(kFSmem)));
       done.fetch_or(bit, std::memory_order_acq_rel);
     }
+    sms = std::max(sm_count[dev & 63].load(std::memory_order_relaxed), 1);
   }
   for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
     const int nb = (B - c0) < kApcMaxB ? (B - c0) : kApcMaxB;
@@ -725,8 +788,9 @@ static pace_status_t resample_impl(const uint8_t* src, const int64_t* src_off, c
       if (t.Ho[i] > hmax) hmax = t.Ho[i];
       if (t.Wo[i] > wmax) wmax = t.Wo[i];
     }
-    dim3 grid((wmax + kFTW - 1) / kFTW, (hmax + kFTH - 1) / kFTH, nb);
-    apc_resample<<<grid, 256, kFSmem, stream>>>(src, t, stats, dst);
+    const int64_t tiles = static_cast<int64_t>((wmax + kFTW - 1) / kFTW) * ((hmax + kFTH - 1) / kFTH) * nb;
+    const int grid = static_cast<int>(std::min<int64_t>(tiles, static_cast<int64_t>(kRsCtasPerSm) * sms));
+    apc_resample<<<grid, kRsThreads, kFSmem, stream>>>(src, t, stats, dst);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;
