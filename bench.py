@@ -272,6 +272,7 @@ def algorithmic_counts(wl, keep, r_ratio):
     wo = min(W, max(28, 28 * int(math.floor(W * s / 28 + 0.5))))
     return {
         "vit_flops": 2 * 2 * n * n * 80 * 16,            # two passes of 2 N^2 d H
+        "vit_ex2": 2 * n * n * 16,                          # one exp2 per score and pass
         "llm_flops": 2 * 2 * tq * 28 * nv * 128,
         "density_bytes": img_bytes + 4 * n,                # image once + d_i
         "resample_bytes": img_bytes + ho * wo * 3,
@@ -393,6 +394,9 @@ def run_gpu(args):
         cnt = algorithmic_counts(wl, KEEP, stats["r"])
         vit_ms = statistics.mean(part_ms["vit"])
         achieved = cnt["vit_flops"] / (vit_ms * 1e-3) / 1e12
+        # MUFU ceiling: 32 ex2 per clock per SM (measured on GB300) at the median SM clock seen
+        sm_mhz = (clocks or {}).get("sm_mhz") or float(peaks.get("sm_max_mhz", 0) or 0)
+        mufu_peak = 32.0 * torch.cuda.get_device_properties(0).multi_processor_count * sm_mhz * 1e6 if sm_mhz else None
         peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
         hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
         mean = {k: statistics.mean(v) for k, v in part_ms.items()}
@@ -421,6 +425,13 @@ def run_gpu(args):
                          "kernel": "ViT received attention (attn_row_lse + attn_colsum + attn_reduce), one launch "
                                    "of pace_vit_attn_importance",
                          "algorithmic_flops": cnt["vit_flops"], "us": round(vit_ms * 1e3, 1),
+                         # one pass of QK^T is the "useful" work; the second pass recomputes it
+                         "useful_one_pass_frac": round(achieved / 2 / peak, 4),
+                         # every score costs one exp2 per pass (N^2 H per pass)
+                         "mufu_ex2_per_s": round(cnt["vit_ex2"] / (vit_ms * 1e-3), 1),
+                         "mufu_frac": round(cnt["vit_ex2"] / (vit_ms * 1e-3) / mufu_peak, 4)
+                         if mufu_peak else None,
+                         "mufu_peak_ex2_per_s": mufu_peak,
                          "peak_source": f"{peak_src} bf16 dense burst (MEASURED_PEAKS.json)"
                          if peak_src == "measured" else "fallback 1.9 PFLOP/s bf16"},
             "rooflines_other": other,

@@ -154,6 +154,28 @@ PACE_API pace_status_t pace_apc_density_static(const uint8_t* img, const int64_t
                                                float* d_out, pace_apc_stats* stats, pace_stream_t stream);
 
 /*
+ * APC density on preview tokens (Sec. 3.2 "Shallow Feature Preview", Eq. 1-6): the paper's
+ * own input, the token embeddings T_v of the first ViT block, instead of the pixel stand-in.
+ * Per image b with tokens T_i (rows cu_tokens[b] .. cu_tokens[b+1]-1): t_hat_i = T_i / |T_i|
+ * (a zero token counts as t_hat = 0), c = mean t_hat, phi = |c|^2 (= Eq. 1), rho_g = 1 - phi,
+ * c_hat = c / |c| (0 when c = 0), d_i = |t_hat_i - c_hat|, then the same tail mean, rho_d,
+ * rho, r and target size as pace_apc_density (the target size from the image's H, W).
+ *
+ *  T          device  bf16 [cu_tokens[B], D] row-major, 4-byte aligned; D even, 2 <= D <= 4096
+ *  cu_tokens  host    int32 [B+1] prefix, cu_tokens[0] = 0, at least one token per image
+ *  H, W       host    int32 [B] size of each image in pixels (for h_out, w_out)
+ *  params     host    NULL for the paper's defaults
+ *  d_out      device  float [cu_tokens[B]], one distance per token
+ *  stats      device  pace_apc_stats [B] (n_patches = the token count)
+ *  ws         device  >= pace_apc_density_tokens_workspace_size(B, cu_tokens, D) bytes, 16-B aligned
+ */
+PACE_API size_t pace_apc_density_tokens_workspace_size(int B, const int32_t* cu_tokens, int D);
+PACE_API pace_status_t pace_apc_density_tokens(const void* T, const int32_t* cu_tokens, int B, int D,
+                                               const int32_t* H, const int32_t* W, const pace_apc_params* params,
+                                               float* d_out, pace_apc_stats* stats, void* ws, size_t ws_bytes,
+                                               pace_stream_t stream);
+
+/*
  * APC resize (Sec. 3.2 "Adaptive Condensation"; App. B.3: width and height scaled by
  * sqrt(r), bicubic).  Separable cubic convolution (a = -0.5) with centre-aligned
  * sampling, support widened by the downscale factor (antialias), the window clipped
@@ -223,11 +245,24 @@ PACE_API pace_status_t pace_llm_text_visual_importance(const void* Q, const void
                                               int head_dim, float scale, float* s_llm_raw, void* ws,
                                               size_t ws_bytes, pace_stream_t stream);
 
+/* Fusion of the two maps.  ADAPTIVE is Eq. 7; the other three are the fusion ablations of
+ * Sec. 4 ("Effect of Attention Fusion in DDAE"): Only LLM-Attn (alpha_w = 1, beta_w = 0), Only
+ * ViT-Attn (alpha_w = 0, beta_w = 1) and Fixed Fusion (0.5 / 0.5). */
+typedef enum pace_ddae_fusion {
+  PACE_DDAE_ADAPTIVE = 0,
+  PACE_DDAE_ONLY_LLM = 1,
+  PACE_DDAE_ONLY_VIT = 2,
+  PACE_DDAE_FIXED = 3
+} pace_ddae_fusion;
+
 typedef struct pace_ddae_params {
-  float tau; /* temperature of Eq. 7; 0.5 */
+  float tau;   /* temperature of Eq. 7; 0.5 */
+  int32_t fusion; /* pace_ddae_fusion; PACE_DDAE_ADAPTIVE */
 } pace_ddae_params;
 
-/* Fills the paper's default tau = 0.5. */
+/* Fills the paper's defaults: tau = 0.5, adaptive fusion.  (The static-resolution baselines
+ * of Sec. 4 "Adaptive Resolution vs. Static Resolution" need no mode: pace_apc_params with
+ * r_min = r_max = the fixed ratio.) */
 PACE_API void pace_ddae_params_default(pace_ddae_params* params);
 
 /* Token budget K = floor(frac * n_vis + 0.5), clamped to [0, n_vis]. */
@@ -239,7 +274,8 @@ PACE_API int32_t pace_budget(int32_t n_vis, double frac);
 /*
  * DDAE fusion and top-K (Sec. 3.3, Eq. 7).  Per image b: S_llm, S_vis = min-max
  * normalised maps (a constant map becomes 0); sigma = population standard deviation;
- * [alpha_w, beta_w] = softmax([sigma_llm, sigma_vis] / tau);
+ * [alpha_w, beta_w] = softmax([sigma_llm, sigma_vis] / tau) (or the fixed weights of the
+ * params' fusion mode);
  * S_final = alpha_w S_llm + beta_w S_vis; keep the K_b = cu_keep[b+1] - cu_keep[b]
  * highest S_final (ties: lower index first), written in ascending index order.
  *

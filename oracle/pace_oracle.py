@@ -32,6 +32,9 @@ Readings taken where the paper is silent or cannot be followed literally
   R8  min-max of a constant map gives 0; sigma is the population deviation.
   R9  top-K ties: the lower index wins; the kept indices are returned in
       ascending order.  K = floor(p * N_vis + 0.5) clamped to [0, N_vis].
+  R10 preview tokens given by the caller (apc_density_preview): a token of zero
+      norm counts as t_hat = 0 (cosine 0 with every token, Eq. 1 undefined
+      otherwise); if every token is zero, c_hat = 0.
 """
 from __future__ import annotations
 
@@ -62,9 +65,15 @@ def patch_tokens(img: np.ndarray) -> np.ndarray:
     return np.concatenate([x, np.ones((gh * gw, 1))], axis=1)
 
 
+def unit_rows(T: np.ndarray) -> np.ndarray:
+    """l2-normalised rows; a zero row stays zero (reading R10: its cosine with any token is 0)."""
+    nrm = np.linalg.norm(T, axis=1, keepdims=True)
+    return np.divide(T, nrm, out=np.zeros_like(T, dtype=np.float64), where=nrm > 0)
+
+
 def global_redundancy(T: np.ndarray, rows_per_block: int = 512) -> float:
     """Eq. 1: phi = (1/N^2) sum_i sum_j cos(T_i, T_j), summed literally over all N^2 pairs."""
-    Tn = T / np.linalg.norm(T, axis=1, keepdims=True)
+    Tn = unit_rows(T)
     N = Tn.shape[0]
     total = 0.0
     for i0 in range(0, N, rows_per_block):
@@ -76,11 +85,12 @@ def apc_density_tokens(T: np.ndarray, alpha: float = ALPHA, gamma: float = GAMMA
                        tail_frac: float = TAIL_FRAC) -> Dict[str, object]:
     """Eq. 1-6 on preview tokens T [N, D] (any N >= 1, any D)."""
     N = T.shape[0]
-    Tn = T / np.linalg.norm(T, axis=1, keepdims=True)          # l2-normalised tokens
+    Tn = unit_rows(T)                                           # l2-normalised tokens
     phi = global_redundancy(T)                                  # Eq. 1
     rho_g = 1.0 - phi                                           # Eq. 2
     c = Tn.mean(axis=0)                                         # Eq. 3
-    c_hat = c / np.linalg.norm(c)
+    cn = np.linalg.norm(c)
+    c_hat = c / cn if cn > 0 else np.zeros_like(c)              # reading R10
     d = np.linalg.norm(Tn - c_hat[None, :], axis=1)             # Eq. 4
     k_tail = max(1, int(math.floor(tail_frac * N + 0.5)))       # reading R2
     d_top = float(np.sort(d)[::-1][:k_tail].mean())
@@ -88,6 +98,15 @@ def apc_density_tokens(T: np.ndarray, alpha: float = ALPHA, gamma: float = GAMMA
     rho = alpha * rho_g + (1.0 - alpha) * rho_d                 # Eq. 6
     return dict(N=N, phi=phi, rho_g=rho_g, c=c, c_hat=c_hat, d=d, k_tail=k_tail,
                 d_top=d_top, rho_d=rho_d, rho=rho)
+
+
+def apc_density_preview(T: np.ndarray, H: int, W: int, alpha: float = ALPHA, gamma: float = GAMMA,
+                        tail_frac: float = TAIL_FRAC, r_min: float = 0.0, r_max: float = 1.0):
+    """Sec. 3.2 on the paper's own input: preview tokens T [N, D] of an H x W image."""
+    st = apc_density_tokens(np.asarray(T, dtype=np.float64), alpha, gamma, tail_frac)
+    st["r"] = retention_ratio(st["rho"], r_min, r_max)
+    st["H_out"], st["W_out"] = target_size(H, W, st["r"])
+    return st
 
 
 def retention_ratio(rho: float, r_min: float = 0.0, r_max: float = 1.0) -> float:
@@ -211,15 +230,24 @@ def min_max(x: np.ndarray) -> np.ndarray:
     return (x - lo) / (hi - lo)
 
 
-def ddae_fuse(s_llm_raw: np.ndarray, s_vis_raw: np.ndarray, tau: float = TAU) -> Dict[str, object]:
+# Fusion modes: Eq. 7, and the fusion ablations of Sec. 4 "Effect of Attention Fusion in DDAE"
+# (Only LLM-Attn, Only ViT-Attn, Fixed Fusion with 0.5 on each signal).
+FUSION_WEIGHTS = {"only_llm": (1.0, 0.0), "only_vit": (0.0, 1.0), "fixed": (0.5, 0.5)}
+
+
+def ddae_fuse(s_llm_raw: np.ndarray, s_vis_raw: np.ndarray, tau: float = TAU,
+              fusion: str = "adaptive") -> Dict[str, object]:
     """Eq. 7 and S_final = alpha_w * S_llm + beta_w * S_vis for one image."""
     S_llm = min_max(np.asarray(s_llm_raw, dtype=np.float64))
     S_vis = min_max(np.asarray(s_vis_raw, dtype=np.float64))
     sigma_llm = float(S_llm.std())      # population deviation (R8)
     sigma_vis = float(S_vis.std())
-    z = np.array([sigma_llm, sigma_vis]) / tau
-    e = np.exp(z - z.max())
-    w = e / e.sum()
+    if fusion == "adaptive":
+        z = np.array([sigma_llm, sigma_vis]) / tau
+        e = np.exp(z - z.max())
+        w = e / e.sum()
+    else:
+        w = np.array(FUSION_WEIGHTS[fusion])
     S_final = w[0] * S_llm + w[1] * S_vis
     return dict(S_llm=S_llm, S_vis=S_vis, sigma_llm=sigma_llm, sigma_vis=sigma_vis,
                 alpha_w=float(w[0]), beta_w=float(w[1]), S_final=S_final)
@@ -238,12 +266,12 @@ def top_k_ascending(S_final: np.ndarray, K: int) -> np.ndarray:
 
 
 def ddae_select(s_llm_raw: np.ndarray, s_vis_raw: np.ndarray, cu_v: Sequence[int],
-                keep: Sequence[int], tau: float = TAU) -> Dict[str, np.ndarray]:
+                keep: Sequence[int], tau: float = TAU, fusion: str = "adaptive") -> Dict[str, np.ndarray]:
     """Per image: fuse, then keep the top K_b tokens.  Kept rows are global (cu_v-offset) indices."""
     S_final, weights, kept = [], [], []
     for b in range(len(cu_v) - 1):
         v0, v1 = int(cu_v[b]), int(cu_v[b + 1])
-        f = ddae_fuse(s_llm_raw[v0:v1], s_vis_raw[v0:v1], tau)
+        f = ddae_fuse(s_llm_raw[v0:v1], s_vis_raw[v0:v1], tau, fusion)
         S_final.append(f["S_final"])
         weights.append([f["alpha_w"], f["beta_w"]])
         kept.append(top_k_ascending(f["S_final"], int(keep[b])) + v0)

@@ -43,7 +43,8 @@ struct ApcTable {
   int W[kApcMaxB];
   int gw[kApcMaxB];         // patches per row
   int chunks[kApcMaxB];     // strips per patch row
-  int patch0[kApcMaxB];     // first global patch of image b
+  int patch0[kApcMaxB];     // first global patch (or token) of image b
+  int n[kApcMaxB];          // patches (or tokens) of image b
   int ktail[kApcMaxB];
   int unit_prefix[kApcMaxB + 1];
   int nb;
@@ -236,6 +237,133 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
   }
 }
 
+// ------------------------------------------------------------------------------------------------
+// density on preview tokens (Sec. 3.2 "Shallow Feature Preview": T_v from the first ViT block)
+// ------------------------------------------------------------------------------------------------
+// Same Eq. 1-6 as the pixel path, on caller-supplied bf16 tokens [sum N, D].  A token of zero
+// norm counts as t_hat = 0 (its cosine with any token is taken as 0); if every token of an
+// image is zero, c_hat = 0.
+constexpr int kTokChunk = 32;    // tokens per CTA
+constexpr int kTokMaxD = 4096;   // longest token accepted (c_hat is staged in shared memory)
+
+struct TokTable {
+  int64_t tok0[kApcMaxB];        // first token of image b
+  int n[kApcMaxB];               // tokens of image b
+  int unit_prefix[kApcMaxB + 1]; // chunks of kTokChunk tokens
+  int ktail[kApcMaxB];
+  int nb;
+  int b_base;
+  int D;
+};
+
+__device__ __forceinline__ int find_tok_image(const TokTable& t, int unit) {
+  int b = 0;
+  while (b + 1 < t.nb && t.unit_prefix[b + 1] <= unit) ++b;
+  return b;
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+// Pass 1: 1/|T_i| per token (warp per token) and the chunk's column sums of t_hat = T_i / |T_i|,
+// added to the image's D-vector as signed 2^-32 fixed point (exact, order-independent).
+__global__ void __launch_bounds__(kApcThreads) apc_tok_pass1(const uint32_t* __restrict__ T,
+                                                             const __grid_constant__ TokTable t,
+                                                             float* __restrict__ inv_norm,
+                                                             unsigned long long* __restrict__ sums) {
+  __shared__ float inv[kTokChunk];
+  const int unit = blockIdx.x;
+  const int b = find_tok_image(t, unit);
+  const int c0 = (unit - t.unit_prefix[b]) * kTokChunk;
+  const int nt = min(kTokChunk, t.n[b] - c0);
+  const int words = t.D >> 1;   // bf16 pairs per token
+  const uint32_t* base = T + (t.tok0[b] + c0) * words;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int p = warp; p < nt; p += kApcThreads / 32) {
+    const uint32_t* row = base + static_cast<int64_t>(p) * words;
+    float ss = 0.f;
+    for (int w = lane; w < words; w += 32) {
+      const uint32_t v = row[w];
+      const float lo = bf16_lo(v), hi = bf16_hi(v);
+      ss = fmaf(lo, lo, fmaf(hi, hi, ss));
+    }
+    ss = warp_sum_f(ss);
+    if (lane == 0) {
+      const float iv = ss > 0.f ? 1.0f / sqrtf(ss) : 0.f;
+      inv[p] = iv;
+      inv_norm[t.tok0[b] + c0 + p] = iv;
+    }
+  }
+  __syncthreads();
+  unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * t.D;
+  for (int w = threadIdx.x; w < words; w += kApcThreads) {
+    float a0 = 0.f, a1 = 0.f;
+    for (int p = 0; p < nt; ++p) {   // the chunk's rows were just read: L1 hits
+      const uint32_t v = base[static_cast<int64_t>(p) * words + w];
+      a0 = fmaf(inv[p], bf16_lo(v), a0);
+      a1 = fmaf(inv[p], bf16_hi(v), a1);
+    }
+    atomicAdd(sb + 2 * w, static_cast<unsigned long long>(__float2ll_rn(a0 * 4294967296.0f)));
+    atomicAdd(sb + 2 * w + 1, static_cast<unsigned long long>(__float2ll_rn(a1 * 4294967296.0f)));
+  }
+}
+
+// Pass 2: c = sums / N, phi = |c|^2, c_hat = c / |c|, then d_i = |t_hat_i - c_hat| directly
+// (warp per token).
+__global__ void __launch_bounds__(kApcThreads) apc_tok_pass2(const uint32_t* __restrict__ T,
+                                                             const __grid_constant__ TokTable t,
+                                                             const float* __restrict__ inv_norm,
+                                                             const unsigned long long* __restrict__ sums,
+                                                             float* __restrict__ d_out,
+                                                             pace_apc_stats* __restrict__ stats) {
+  __shared__ __align__(16) float chat[kTokMaxD];
+  __shared__ float red[kApcThreads / 32];
+  const int unit = blockIdx.x;
+  const int b = find_tok_image(t, unit);
+  const int c0 = (unit - t.unit_prefix[b]) * kTokChunk;
+  const int nt = min(kTokChunk, t.n[b] - c0);
+  const int N = t.n[b], D = t.D, words = D >> 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * D;
+  float part = 0.f;
+  for (int k = threadIdx.x; k < D; k += kApcThreads) {
+    const float cv = static_cast<float>(static_cast<double>(static_cast<long long>(sb[k])) * (1.0 / kFix) / N);
+    chat[k] = cv;
+    part = fmaf(cv, cv, part);
+  }
+  part = warp_sum_f(part);
+  if (lane == 0) red[warp] = part;
+  __syncthreads();
+  float phi = 0.f;
+#pragma unroll
+  for (int w = 0; w < kApcThreads / 32; ++w) phi += red[w];
+  const float inv_c = phi > 0.f ? 1.0f / sqrtf(phi) : 0.f;
+  for (int k = threadIdx.x; k < D; k += kApcThreads) chat[k] *= inv_c;
+  if (c0 == 0 && threadIdx.x == 0) {
+    stats[t.b_base + b].phi = phi;
+    stats[t.b_base + b].rho_g = 1.0f - phi;
+    stats[t.b_base + b].n_patches = N;
+    stats[t.b_base + b].k_tail = t.ktail[b];
+  }
+  __syncthreads();
+  const uint32_t* base = T + (t.tok0[b] + c0) * words;
+  const float2* chat2 = reinterpret_cast<const float2*>(chat);
+  for (int p = warp; p < nt; p += kApcThreads / 32) {
+    const uint32_t* row = base + static_cast<int64_t>(p) * words;
+    const float iv = inv_norm[t.tok0[b] + c0 + p];
+    float acc0 = 0.f, acc1 = 0.f;
+    for (int w = lane; w < words; w += 32) {
+      const uint32_t v = row[w];
+      const float2 ch = chat2[w];
+      const float e0 = fmaf(bf16_lo(v), iv, -ch.x), e1 = fmaf(bf16_hi(v), iv, -ch.y);
+      acc0 = fmaf(e0, e0, acc0);
+      acc1 = fmaf(e1, e1, acc1);
+    }
+    const float acc = warp_sum_f(acc0 + acc1);
+    if (lane == 0) d_out[t.tok0[b] + c0 + p] = sqrtf(acc);
+  }
+}
+
 struct TailParams {
   float alpha, gamma, r_min, r_max;
   int align;
@@ -251,7 +379,7 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
   __shared__ float red[32];
   __shared__ unsigned cred[32];
   const int b = blockIdx.x;
-  const int N = (t.H[b] / kPatch) * t.gw[b];
+  const int N = t.n[b];
   const float* db = d + t.patch0[b];
   if (N <= kTailSmemMax) {   // one coalesced read of the distances, then work from shared memory
     for (int i = threadIdx.x; i < N; i += blockDim.x) sd[i] = db[i];
@@ -638,7 +766,7 @@ DensityLayout density_layout(int B, const int32_t* H, const int32_t* W) {
 // Dynamic shared memory of apc_tail: the largest image's distances when they fit.
 size_t tail_smem(const ApcTable& t) {
   int n = 0;
-  for (int i = 0; i < t.nb; ++i) n = std::max(n, (t.H[i] / kPatch) * t.gw[i]);
+  for (int i = 0; i < t.nb; ++i) n = std::max(n, t.n[i]);
   return n <= kTailSmemMax ? static_cast<size_t>(n) * sizeof(float) : 0;
 }
 
@@ -717,6 +845,7 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
       t.chunks[i] = (t.gw[i] + kStrip - 1) / kStrip;
       t.patch0[i] = patch0;
       const int N = (H[b] / kPatch) * t.gw[i];
+      t.n[i] = N;
       double kt = std::floor(static_cast<double>(p.tail_frac) * N + 0.5);
       if (kt < 1) kt = 1;
       if (kt > N) kt = N;
@@ -883,6 +1012,7 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
     t.chunks[b] = (t.gw[b] + kStrip - 1) / kStrip;
     t.patch0[b] = patch0;
     const int N = (H[b] / kPatch) * t.gw[b];
+    t.n[b] = N;
     double kt = std::floor(static_cast<double>(p.tail_frac) * N + 0.5);
     if (kt < 1) kt = 1;
     if (kt > N) kt = N;
@@ -901,4 +1031,88 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
   TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
   apc_tail<<<B, 1024, tail_smem(t), stream>>>(t, d_out, tp, stats);
   return check_launch();
+}
+
+// ------------------------------------------------------------------------------------------------
+// pace_apc_density_tokens: Eq. 1-6 on preview tokens
+// ------------------------------------------------------------------------------------------------
+namespace pace {
+namespace {
+struct TokLayout {
+  size_t sums_off, inv_off, total;
+};
+TokLayout tok_layout(int B, const int32_t* cu, int D) {
+  TokLayout L{};
+  L.sums_off = 0;
+  L.inv_off = align_up(static_cast<size_t>(B) * D * sizeof(unsigned long long), 256);
+  L.total = L.inv_off + align_up(static_cast<size_t>(cu[B]) * sizeof(float), 256);
+  return L;
+}
+}  // namespace
+}  // namespace pace
+
+extern "C" size_t pace_apc_density_tokens_workspace_size(int B, const int32_t* cu_tokens, int D) {
+  if (B <= 0 || cu_tokens == nullptr || D < 2) return 0;
+  return tok_layout(B, cu_tokens, D).total;
+}
+
+extern "C" pace_status_t pace_apc_density_tokens(const void* T, const int32_t* cu_tokens, int B, int D,
+                                                 const int32_t* H, const int32_t* W,
+                                                 const pace_apc_params* params, float* d_out,
+                                                 pace_apc_stats* stats, void* ws, size_t ws_bytes,
+                                                 pace_stream_t stream) {
+  if (B < 0) return PACE_ERR_INVALID_ARG;
+  if (B == 0) return PACE_OK;
+  if (T == nullptr || cu_tokens == nullptr || H == nullptr || W == nullptr || d_out == nullptr || stats == nullptr)
+    return PACE_ERR_INVALID_ARG;
+  if (D < 2 || D > kTokMaxD || D % 2 != 0 || reinterpret_cast<uintptr_t>(T) % 4 != 0) return PACE_ERR_INVALID_ARG;
+  if (cu_tokens[0] != 0) return PACE_ERR_INVALID_ARG;
+  for (int b = 0; b < B; ++b)
+    if (cu_tokens[b + 1] - cu_tokens[b] < 1 || H[b] < 1 || W[b] < 1) return PACE_ERR_INVALID_ARG;
+  pace_apc_params p;
+  if (params) p = *params; else pace_apc_params_default(&p);
+  if (!(p.tail_frac > 0.f && p.tail_frac <= 1.f) || !(p.gamma > 0.f) || !(p.alpha >= 0.f && p.alpha <= 1.f) ||
+      !(p.r_min <= p.r_max) || p.align < 1)
+    return PACE_ERR_INVALID_ARG;
+  const TokLayout L = tok_layout(B, cu_tokens, D);
+  if (ws == nullptr || ws_bytes < L.total || reinterpret_cast<uintptr_t>(ws) % 16) return PACE_ERR_WORKSPACE;
+  PACE_CHECK(check_device());
+  PACE_CHECK(tail_smem_attr());
+  uint8_t* w8 = static_cast<uint8_t*>(ws);
+  auto* sums = reinterpret_cast<unsigned long long*>(w8 + L.sums_off);
+  auto* inv = reinterpret_cast<float*>(w8 + L.inv_off);
+  PACE_CUDA(cudaMemsetAsync(sums, 0, static_cast<size_t>(B) * D * sizeof(unsigned long long), stream));
+  const uint32_t* T32 = static_cast<const uint32_t*>(T);
+  for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
+    const int nb = (B - c0) < kApcMaxB ? (B - c0) : kApcMaxB;
+    TokTable tt{};
+    ApcTable at{};   // what the shared tail kernel reads: sizes, token ranges, k_tail
+    tt.nb = at.nb = nb;
+    tt.b_base = at.b_base = c0;
+    tt.D = D;
+    tt.unit_prefix[0] = 0;
+    for (int i = 0; i < nb; ++i) {
+      const int b = c0 + i;
+      const int N = cu_tokens[b + 1] - cu_tokens[b];
+      tt.tok0[i] = cu_tokens[b];
+      tt.n[i] = at.n[i] = N;
+      double kt = std::floor(static_cast<double>(p.tail_frac) * N + 0.5);
+      if (kt < 1) kt = 1;
+      if (kt > N) kt = N;
+      tt.ktail[i] = at.ktail[i] = static_cast<int>(kt);
+      tt.unit_prefix[i + 1] = tt.unit_prefix[i] + (N + kTokChunk - 1) / kTokChunk;
+      at.H[i] = H[b];
+      at.W[i] = W[b];
+      at.patch0[i] = cu_tokens[b];
+    }
+    const int units = tt.unit_prefix[nb];
+    apc_tok_pass1<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums);
+    PACE_CHECK(check_launch());
+    apc_tok_pass2<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums, d_out, stats);
+    PACE_CHECK(check_launch());
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
+    apc_tail<<<nb, 1024, tail_smem(at), stream>>>(at, d_out, tp, stats);
+    PACE_CHECK(check_launch());
+  }
+  return PACE_OK;
 }

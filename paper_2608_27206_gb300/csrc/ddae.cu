@@ -69,7 +69,7 @@ __device__ __forceinline__ float2 block_reduce2(float a, float b, float* red) {
 __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* __restrict__ s_llm,
                                                                   const float* __restrict__ s_vis,
                                                                   const __grid_constant__ SelectTable tab,
-                                                                  float tau, float* __restrict__ s_final,
+                                                                  float tau, int fusion, float* __restrict__ s_final,
                                                                   float* __restrict__ weights,
                                                                   int32_t* __restrict__ kept, int b_base) {
   extern __shared__ float sm[];
@@ -117,10 +117,22 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
   const float2 sq = block_reduce2<0>(qa, qv, red);
   const float sig_a = sqrtf(sq.x / nv), sig_v = sqrtf(sq.y / nv);
 
-  // 3. Eq. 7: confidence-weighted softmax fusion
-  const float za = sig_a / tau, zv = sig_v / tau, zm = fmaxf(za, zv);
-  const float ea = expf(za - zm), ev = expf(zv - zm);
-  const float wa = ea / (ea + ev), wv = ev / (ea + ev);
+  // 3. Eq. 7: confidence-weighted softmax fusion (or a fixed-weight ablation)
+  float wa, wv;
+  if (fusion == PACE_DDAE_ONLY_LLM) {
+    wa = 1.f;
+    wv = 0.f;
+  } else if (fusion == PACE_DDAE_ONLY_VIT) {
+    wa = 0.f;
+    wv = 1.f;
+  } else if (fusion == PACE_DDAE_FIXED) {
+    wa = wv = 0.5f;
+  } else {
+    const float za = sig_a / tau, zv = sig_v / tau, zm = fmaxf(za, zv);
+    const float ea = expf(za - zm), ev = expf(zv - zm);
+    wa = ea / (ea + ev);
+    wv = ev / (ea + ev);
+  }
   if (tid == 0 && weights != nullptr) {
     weights[2 * (b_base + b)] = wa;
     weights[2 * (b_base + b) + 1] = wv;
@@ -275,7 +287,9 @@ extern "C" pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s
   }
   if (cu_keep[B] > 0 && kept == nullptr) return PACE_ERR_INVALID_ARG;
   const float tau = params ? params->tau : 0.5f;
+  const int fusion = params ? params->fusion : PACE_DDAE_ADAPTIVE;
   if (!(tau > 0.f) || !std::isfinite(tau)) return PACE_ERR_INVALID_ARG;
+  if (fusion < PACE_DDAE_ADAPTIVE || fusion > PACE_DDAE_FIXED) return PACE_ERR_INVALID_ARG;
   PACE_CHECK(check_device());
   const size_t smem = static_cast<size_t>(2 * max_nv) * sizeof(float);
   {
@@ -300,7 +314,7 @@ extern "C" pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s
       t.k0[i] = cu_keep[b];
       t.nk[i] = cu_keep[b + 1] - cu_keep[b];
     }
-    ddae_select_kernel<<<nb, kSelThreads, smem, stream>>>(s_llm_raw, s_vis_raw, t, tau, s_final, weights, kept,
+    ddae_select_kernel<<<nb, kSelThreads, smem, stream>>>(s_llm_raw, s_vis_raw, t, tau, fusion, s_final, weights, kept,
                                                            c0);
     PACE_CHECK(check_launch());
   }

@@ -155,6 +155,7 @@ void pace_apc_params_default(pace_apc_params* p) {
 void pace_ddae_params_default(pace_ddae_params* p) {
   if (!p) return;
   p->tau = 0.5f;
+  p->fusion = PACE_DDAE_ADAPTIVE;
 }
 
 }  // extern "C"

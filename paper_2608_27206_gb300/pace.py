@@ -36,7 +36,11 @@ class ApcParams(ctypes.Structure):
 
 
 class DdaeParams(ctypes.Structure):
-    _fields_ = [("tau", ctypes.c_float)]
+    _fields_ = [("tau", ctypes.c_float), ("fusion", ctypes.c_int32)]
+
+
+# fusion modes of DdaeParams (pace_ddae_fusion)
+DDAE_ADAPTIVE, DDAE_ONLY_LLM, DDAE_ONLY_VIT, DDAE_FIXED = 0, 1, 2, 3
 
 
 _P = ctypes.c_void_p
@@ -51,6 +55,9 @@ _SIGS = {
     "pace_device_status": (ctypes.c_int, [_I32P, _I32P, ctypes.c_int]),
     "pace_apc_params_default": (None, [ctypes.POINTER(ApcParams)]),
     "pace_apc_density_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, _I32P]),
+    "pace_apc_density_tokens_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, ctypes.c_int]),
+    "pace_apc_density_tokens": (ctypes.c_int, [_P, _I32P, ctypes.c_int, ctypes.c_int, _I32P, _I32P,
+                                               ctypes.POINTER(ApcParams), _P, _P, _P, ctypes.c_size_t, _P]),
     "pace_apc_density": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, ctypes.c_int, ctypes.POINTER(ApcParams), _P, _P,
                                         _P, ctypes.c_size_t, _P]),
     "pace_apc_density_static": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, ctypes.c_int, ctypes.POINTER(ApcParams),
@@ -239,6 +246,32 @@ def pace_apc_density_static(img: torch.Tensor, img_off, H, W, params: Optional[A
                                        ctypes.byref(params) if params is not None else None, _dev(d_out),
                                        _dev(stats), _stream(stream))
     _check("pace_apc_density_static", st)
+    return d_out[:n], stats[:B]
+
+
+def pace_apc_density_tokens_workspace_size(cu_tokens, D: int) -> int:
+    cu = _i32(cu_tokens)
+    return int(lib().pace_apc_density_tokens_workspace_size(len(cu) - 1, _pi32(cu), D))
+
+
+def pace_apc_density_tokens(T: torch.Tensor, cu_tokens, H, W, params: Optional[ApcParams] = None,
+                            d_out: Optional[torch.Tensor] = None, stats: Optional[torch.Tensor] = None,
+                            ws: Optional[torch.Tensor] = None, stream=None):
+    """APC density of B images' preview tokens T (bf16 [sum N, D]).  Returns (d [sum N], stats)."""
+    cu, h, w = _i32(cu_tokens), _i32(H), _i32(W)
+    B = len(cu) - 1
+    n, D = int(cu[-1]), int(T.shape[-1])
+    dev = T.device
+    if d_out is None:
+        d_out = torch.empty(max(n, 1), dtype=torch.float32, device=dev)
+    if stats is None:
+        stats = torch.zeros((max(B, 1), 10), dtype=torch.int32, device=dev)
+    if ws is None:
+        ws = torch.empty(max(pace_apc_density_tokens_workspace_size(cu, D), 16), dtype=torch.uint8, device=dev)
+    st = lib().pace_apc_density_tokens(_dev(T), _pi32(cu), B, D, _pi32(h), _pi32(w),
+                                       ctypes.byref(params) if params is not None else None, _dev(d_out),
+                                       _dev(stats), _dev(ws), ws.numel(), _stream(stream))
+    _check("pace_apc_density_tokens", st)
     return d_out[:n], stats[:B]
 
 

@@ -63,6 +63,7 @@ def test_param_defaults_match_paper(libpace, golden):
     assert p.tail_frac == pytest.approx(g["tail_frac"]) and p.align == g["merge_unit"]
     assert p.r_min == 0.0 and p.r_max == 1.0
     assert libpace.ddae_params().tau == pytest.approx(g["tau"])
+    assert libpace.ddae_params().fusion == libpace.DDAE_ADAPTIVE
 
 
 def test_budget_matches_oracle(libpace):

@@ -111,7 +111,61 @@ def test_density_batch_and_params(pace):
     p = pace.apc_params(alpha=0.3, gamma=0.8, tail_frac=0.05, r_min=0.1, r_max=0.4)
     d, st = _density(pace, imgs, params=p)
     _check_density(d, st, imgs, alpha=0.3, gamma=0.8, tail=0.05, r_min=0.1, r_max=0.4)
+    # the static-resolution baselines (a fixed ratio for every image): r_min = r_max = 0.5
+    p = pace.apc_params(r_min=0.5, r_max=0.5)
+    d, st = _density(pace, imgs, params=p)
+    _check_density(d, st, imgs, r_min=0.5, r_max=0.5)
+    for s, img in zip(st, imgs):
+        assert s["r"] == 0.5 and (s["h_out"], s["w_out"]) == O.target_size(img.shape[0], img.shape[1], 0.5)
     _no_device_error(pace)
+
+
+def _tokens_case(pace, lens, D, seed, zero_rows=(), params=None, sizes=None):
+    rng = np.random.default_rng(seed)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    # preview-like tokens: a shared direction plus per-token detail of varying strength
+    base = rng.normal(size=D)
+    T = base[None, :] * rng.uniform(0.5, 2.0, (cu[-1], 1)) + rng.normal(size=(cu[-1], D)) * rng.uniform(
+        0.05, 1.5, (cu[-1], 1))
+    T[list(zero_rows)] = 0.0
+    Tb = synth.f32_to_bf16_bits(T.astype(np.float32))
+    sizes = sizes or [(28 * (8 + 3 * b), 28 * (10 + 2 * b)) for b in range(len(lens))]
+    H = [h for h, _ in sizes]
+    W = [w for _, w in sizes]
+    d, st = pace.pace_apc_density_tokens(bf16_tensor(Tb).view(-1, D), cu, H, W, params=params)
+    return f64(Tb).reshape(-1, D), cu, H, W, d.cpu().numpy(), pace.stats_dict(st)
+
+
+@pytest.mark.parametrize("lens,D", [([1024], 1280), ([37], 64), ([5000, 3, 200], 1152), ([700], 4096)])
+def test_density_tokens(pace, lens, D):
+    """Eq. 1-6 on preview tokens (the paper's own input) against the oracle."""
+    T, cu, H, W, d, st = _tokens_case(pace, lens, D, seed=D + len(lens), zero_rows=[1] if lens[0] > 1 else [])
+    for b in range(len(lens)):
+        ref = O.apc_density_preview(T[cu[b]:cu[b + 1]], H[b], W[b])
+        s = st[b]
+        assert s["n_patches"] == lens[b] and s["k_tail"] == ref["k_tail"]
+        assert_scores_close(d[cu[b]:cu[b + 1]], ref["d"], atol_frac=2e-3, atol=1e-5, what="token d_i")
+        for k in ("phi", "d_top", "rho_d", "r"):
+            assert abs(s[k] - ref[k]) <= 2e-3 * max(abs(ref[k]), 1e-3), (k, s[k], ref[k])
+        assert abs(s["rho"] - ref["rho"]) <= 2e-3 * max(abs(ref["rho"]), 1e-3) + 2e-6
+        for side, key, exp in ((H[b], "h_out", ref["H_out"]), (W[b], "w_out", ref["W_out"])):
+            x = side * math.sqrt(max(ref["r"], 0.0)) / 28 + 0.5
+            assert s[key] == exp or (abs(x - round(x)) < 2e-3 * x and abs(s[key] - exp) == 28), (key, s[key], exp)
+    _no_device_error(pace)
+
+
+def test_density_tokens_params_and_rejects(pace):
+    p = pace.apc_params(alpha=0.2, gamma=0.9, tail_frac=0.2, r_min=0.3, r_max=0.6)
+    T, cu, H, W, d, st = _tokens_case(pace, [300, 41], 256, seed=5, params=p)
+    for b in range(2):
+        ref = O.apc_density_preview(T[cu[b]:cu[b + 1]], H[b], W[b], 0.2, 0.9, 0.2, 0.3, 0.6)
+        assert abs(st[b]["r"] - ref["r"]) <= 2e-3 * ref["r"] and st[b]["k_tail"] == ref["k_tail"]
+    Tt = torch.zeros((10, 63), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(pace.PaceError):
+        pace.pace_apc_density_tokens(Tt, [0, 10], [28], [28])           # odd D
+    Tt = torch.zeros((10, 64), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(pace.PaceError):
+        pace.pace_apc_density_tokens(Tt, [0, 10, 10], [28, 28], [28, 28])   # an image without tokens
 
 
 def test_density_constant_images(pace):
@@ -325,11 +379,35 @@ def test_importance_rejects_bad_args(pace):
 # ----------------------------------------------------------------------------------------------
 # DDAE select
 # ----------------------------------------------------------------------------------------------
-def _select(pace, sl, sv, cu, keep, tau=0.5):
+def _select(pace, sl, sv, cu, keep, tau=0.5, fusion=0):
     r = pace.pace_ddae_select(torch.from_numpy(sl.astype(np.float32)).cuda(),
                               torch.from_numpy(sv.astype(np.float32)).cuda(), cu,
-                              np.concatenate([[0], np.cumsum(keep)]).astype(np.int32), pace.ddae_params(tau=tau))
+                              np.concatenate([[0], np.cumsum(keep)]).astype(np.int32),
+                              pace.ddae_params(tau=tau, fusion=fusion))
     return [x.cpu().numpy() for x in r]
+
+
+@pytest.mark.parametrize("mode,name", [(1, "only_llm"), (2, "only_vit"), (3, "fixed")])
+def test_ddae_fusion_ablations(pace, mode, name):
+    """The fusion ablations (Only LLM-Attn, Only ViT-Attn, Fixed Fusion) against the oracle."""
+    rng = np.random.default_rng(40 + mode)
+    lens = [300, 2584, 17]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    sl = rng.gamma(0.5, 2.0, size=cu[-1]).astype(np.float32)
+    sv = rng.lognormal(0, 1, size=cu[-1]).astype(np.float32)
+    keep = [O.budget(n, 0.1) for n in lens]
+    s_final, w, kept = _select(pace, sl, sv, cu, keep, fusion=mode)
+    k0 = 0
+    for b, n in enumerate(lens):
+        v0, v1 = cu[b], cu[b + 1]
+        f = O.ddae_fuse(sl[v0:v1].astype(np.float64), sv[v0:v1].astype(np.float64), fusion=name)
+        assert (w[b, 0], w[b, 1]) == O.FUSION_WEIGHTS[name]
+        assert_scores_close(s_final[v0:v1], f["S_final"], atol_frac=2e-3, what=f"S_final {name}")
+        assert_kept_matches(kept[k0:k0 + keep[b]], f["S_final"], keep[b], offset=v0)
+        k0 += keep[b]
+    with pytest.raises(pace.PaceError):
+        _select(pace, sl, sv, cu, keep, fusion=4)
+    _no_device_error(pace)
 
 
 @pytest.mark.parametrize("lens,fracs", [([256], [0.1]), ([2584], [0.1]), ([10549], [0.05]), ([1], [1.0]),

@@ -310,3 +310,44 @@ def test_ddae_select_ragged_offsets():
 def test_gather_rows():
     E = np.arange(40, dtype=np.uint16).reshape(10, 4)
     np.testing.assert_array_equal(O.gather_rows(E, [3, 0, 9]), E[[3, 0, 9]])
+
+
+def test_ddae_fusion_ablation_modes():
+    """Fusion ablations (Sec. 4): with one weight at 1 the kept set is the top of that map alone
+    (checked against a plain sort of the single map); fixed fusion is the mean of the two maps
+    and equals Eq. 7 when the two deviations are equal."""
+    rng = np.random.default_rng(12)
+    sl, sv = rng.gamma(0.5, 2.0, 500), rng.lognormal(0, 1, 500)
+    for mode, raw in (("only_llm", sl), ("only_vit", sv)):
+        f = O.ddae_fuse(sl, sv, fusion=mode)
+        z = (raw - raw.min()) / (raw.max() - raw.min())
+        np.testing.assert_allclose(f["S_final"], z, rtol=0, atol=1e-15)
+        K = 37
+        brute = np.sort(sorted(range(500), key=lambda i: (-z[i], i))[:K])
+        np.testing.assert_array_equal(O.top_k_ascending(f["S_final"], K), brute)
+    f = O.ddae_fuse(sl, sv, fusion="fixed")
+    assert (f["alpha_w"], f["beta_w"]) == (0.5, 0.5)
+    np.testing.assert_allclose(f["S_final"], 0.5 * (f["S_llm"] + f["S_vis"]), atol=1e-15)
+    a = rng.normal(size=64)
+    g_adapt = O.ddae_fuse(a, -a)                       # mirrored maps: equal deviations
+    g_fixed = O.ddae_fuse(a, -a, fusion="fixed")
+    np.testing.assert_allclose(g_adapt["S_final"], g_fixed["S_final"], atol=1e-12)
+
+
+def test_preview_tokens_zero_rows_and_identity():
+    """Reading R10 on preview tokens: zero rows are t_hat = 0; Eq. 1 (literal double sum) still
+    equals |c|^2; with every token equal, phi = 1, rho_g = 0, all d_i = 0."""
+    rng = np.random.default_rng(21)
+    T = rng.normal(size=(40, 24))
+    T[[3, 17]] = 0.0
+    st = O.apc_density_tokens(T)
+    Tn = [t / np.linalg.norm(t) if np.linalg.norm(t) > 0 else np.zeros_like(t) for t in T]
+    brute = sum(float(a @ b_) for a in Tn for b_ in Tn) / (40 * 40)
+    assert st["phi"] == pytest.approx(brute, rel=1e-12)
+    assert st["phi"] == pytest.approx(float(st["c"] @ st["c"]), rel=1e-12)
+    assert st["d"][3] == pytest.approx(1.0) and st["d"][17] == pytest.approx(1.0)   # |0 - c_hat| = 1
+    same = np.tile(rng.normal(size=(1, 24)), (30, 1))
+    st2 = O.apc_density_preview(same, 280, 420)
+    assert st2["phi"] == pytest.approx(1.0) and st2["rho_g"] == pytest.approx(0.0, abs=1e-12)
+    assert np.all(np.abs(st2["d"]) < 1e-7)
+    assert (st2["H_out"], st2["W_out"]) == (28, 28)                                # r = 0
