@@ -301,6 +301,62 @@ PACE_API pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s_v
 PACE_API pace_status_t pace_gather(const void* src, int64_t n_src_rows, int64_t row_bytes, const int32_t* idx,
                           int64_t n_idx, void* dst, pace_stream_t stream);
 
+/*
+ * Token budget relative to Vanilla (App. C, "B = p1 p2"): K = floor(frac * n_vis_vanilla + 0.5)
+ * (the count the uncondensed image would have), capped at the n_vis_condensed tokens that
+ * remain after APC.  frac is the final ratio B; pace_budget is the same rule on one count.
+ */
+PACE_API int32_t pace_budget_vanilla(int32_t n_vis_vanilla, int32_t n_vis_condensed, double frac);
+
+/*
+ * Row list of the pruned LLM sequences (Sec. 3.3: the kept tokens "formulate the final LLM
+ * context sequence"; App. C: S_post = T + N_keep).  Sequence b occupies rows
+ * cu_seq[b] .. cu_seq[b+1]-1 of a packed pre-prune batch and holds its image's visual tokens
+ * at rows vis_start[b] .. vis_start[b] + n_vis_b - 1 of the sequence.  Its output keeps every
+ * position outside the visual span and the visual positions of its kept tokens, in sequence
+ * order, as global pre-prune row numbers:
+ *   out rows of sequence b start at sum_{c<b} (n_pre_c - n_vis_c + K_c).
+ * The list feeds pace_gather_multi (hidden states, KV-cache rows, position ids).  A kept
+ * entry outside image b's tokens writes -1 and records PACE_ERR_INVALID_ARG on the device.
+ *
+ *  cu_seq     host    int32 [B+1] pre-prune sequence prefix
+ *  vis_start  host    int32 [B] start of the visual span within each sequence
+ *  cu_vis     host    int32 [B+1] visual tokens per image (as passed to pace_ddae_select)
+ *  cu_keep    host    int32 [B+1] kept tokens per image (as passed to pace_ddae_select)
+ *  kept       device  int32 [cu_keep[B]] pace_ddae_select's kept list (global visual index,
+ *                     ascending within each image)
+ *  out_idx    device  int32 [sum_b n_pre_b - n_vis_b + K_b]
+ */
+PACE_API pace_status_t pace_prune_index(int B, const int32_t* cu_seq, const int32_t* vis_start,
+                                        const int32_t* cu_vis, const int32_t* cu_keep, const int32_t* kept,
+                                        int32_t* out_idx, pace_stream_t stream);
+
+/* One tensor of pace_gather_multi: n_slabs independent slabs (e.g. layer x KV head) of rows;
+ * output row r of slab s copies row_bytes from src row idx[r] of the same slab.  All strides
+ * in bytes.  16-byte copies are used when every pointer, stride and row_bytes allows. */
+typedef struct pace_gather_tensor {
+  const void* src;
+  void* dst;
+  int64_t row_bytes;
+  int64_t src_row_stride;   /* >= row_bytes */
+  int64_t dst_row_stride;   /* >= row_bytes */
+  int64_t n_slabs;
+  int64_t src_slab_stride;
+  int64_t dst_slab_stride;
+  int64_t n_src_rows;       /* rows per source slab; an index outside [0, n_src_rows) writes a zero
+                               row and records PACE_ERR_INVALID_ARG on the device */
+} pace_gather_tensor;
+
+#define PACE_GATHER_MAX_TENSORS 16
+
+/*
+ * The prune step's gathers in one launch (App. C): every tensor gathered with the same row
+ * list idx (device int32 [n_idx]); tensors host [n_tensors] descriptors, n_tensors <= 16.
+ * Byte-exact.
+ */
+PACE_API pace_status_t pace_gather_multi(const pace_gather_tensor* tensors, int n_tensors, const int32_t* idx,
+                                         int64_t n_idx, pace_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -282,3 +282,18 @@ def ddae_select(s_llm_raw: np.ndarray, s_vis_raw: np.ndarray, cu_v: Sequence[int
 def gather_rows(E: np.ndarray, idx: np.ndarray) -> np.ndarray:
     """Sec. 3.3: the kept visual rows form the pruned LLM context."""
     return E[np.asarray(idx, dtype=np.int64)]
+
+
+def budget_vanilla(n_vis_vanilla: int, n_vis_condensed: int, frac: float) -> int:
+    """App. C: the final ratio B = p1 p2 is relative to Vanilla, so K = round(B * N_vis_vanilla)
+    (reading R9's rounding), capped at the tokens left after condensation."""
+    return min(budget(n_vis_vanilla, frac), max(n_vis_condensed, 0))
+
+
+def prune_rows(n_pre: int, vis_start: int, n_vis: int, kept_local: Sequence[int]) -> np.ndarray:
+    """Sec. 3.3 / App. C: rows of the pruned LLM sequence, S_post = T + N_keep positions: every
+    position outside the visual span, and the kept visual positions, in sequence order."""
+    keep = np.ones(n_pre, dtype=bool)
+    keep[vis_start:vis_start + n_vis] = False
+    keep[vis_start + np.asarray(kept_local, dtype=np.int64)] = True
+    return np.nonzero(keep)[0]

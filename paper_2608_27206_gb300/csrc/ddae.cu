@@ -267,6 +267,99 @@ __global__ void __launch_bounds__(256) gather_rows_bytes(const uint8_t* __restri
   }
 }
 
+// Row list of the pruned LLM sequences (Sec. 3.3; App. C): sequence b (rows seq0 .. seq0 +
+// n_pre - 1 of the packed pre-prune batch) keeps every position outside its visual span
+// [vis, vis + n_vis) and the visual positions of its kept tokens, in sequence order.
+constexpr int kPruneMaxB = 256;
+struct PruneTable {
+  int seq0[kPruneMaxB];   // first pre-prune row of sequence b
+  int n_pre[kPruneMaxB];  // pre-prune length
+  int vis[kPruneMaxB];    // start of the visual span within the sequence
+  int v0[kPruneMaxB];     // first global visual index of image b (as in the kept list)
+  int nv[kPruneMaxB];     // visual tokens of image b
+  int k0[kPruneMaxB];     // first kept entry of image b
+  int nk[kPruneMaxB];     // kept tokens of image b
+  int post0[kPruneMaxB];  // first output row of sequence b
+  int nb;
+};
+
+__global__ void __launch_bounds__(256) prune_index_kernel(const __grid_constant__ PruneTable t,
+                                                          const int32_t* __restrict__ kept,
+                                                          int32_t* __restrict__ out, int* status) {
+  const int b = blockIdx.y;
+  const int n_post = t.n_pre[b] - t.nv[b] + t.nk[b];
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_post; i += gridDim.x * blockDim.x) {
+    int row;
+    if (i < t.vis[b]) {
+      row = i;                                                    // before the visual span
+    } else if (i < t.vis[b] + t.nk[b]) {
+      const int k = kept[t.k0[b] + i - t.vis[b]] - t.v0[b];       // kept visual token (local)
+      if (k < 0 || k >= t.nv[b]) {
+        record_error(status, PACE_ERR_INVALID_ARG, K_PRUNE_INDEX);
+        row = -1;
+        out[t.post0[b] + i] = row;
+        continue;
+      }
+      row = t.vis[b] + k;
+    } else {
+      row = i - t.nk[b] + t.nv[b];                                // after the visual span
+    }
+    out[t.post0[b] + i] = t.seq0[b] + row;
+  }
+}
+
+// One launch over several tensors gathered with the same row list (hidden states, KV-cache
+// rows, position ids ...): work item = (tensor, slab, output row), one warp each.
+struct GatherMultiTable {
+  pace_gather_tensor g[PACE_GATHER_MAX_TENSORS];
+  int64_t item_prefix[PACE_GATHER_MAX_TENSORS + 1];   // slabs x rows per tensor
+  int width[PACE_GATHER_MAX_TENSORS];                  // copy width in bytes: 16, 4 or 1
+  int n;
+};
+
+template <typename V>
+__device__ __forceinline__ void copy_row(const uint8_t* sp, uint8_t* dp, int64_t bytes, int lane) {
+  const V* s = reinterpret_cast<const V*>(sp);
+  V* d = reinterpret_cast<V*>(dp);
+  const int64_t n = bytes / static_cast<int64_t>(sizeof(V));
+  for (int64_t c = lane; c < n; c += 32) d[c] = s[c];
+}
+template <typename V>
+__device__ __forceinline__ void zero_row(uint8_t* dp, int64_t bytes, int lane) {
+  V* d = reinterpret_cast<V*>(dp);
+  const int64_t n = bytes / static_cast<int64_t>(sizeof(V));
+  for (int64_t c = lane; c < n; c += 32) d[c] = V{};
+}
+
+__global__ void __launch_bounds__(256) gather_multi_kernel(const __grid_constant__ GatherMultiTable t,
+                                                           const int32_t* __restrict__ idx, int64_t n_idx,
+                                                           int* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  const int64_t total = t.item_prefix[t.n];
+  for (int64_t w = warp0; w < total; w += nwarps) {
+    int k = 0;
+    while (k + 1 < t.n && t.item_prefix[k + 1] <= w) ++k;
+    const pace_gather_tensor& g = t.g[k];
+    const int64_t local = w - t.item_prefix[k];
+    const int64_t slab = local / n_idx, r = local - slab * n_idx;
+    const int64_t s = idx[r];
+    uint8_t* dp = static_cast<uint8_t*>(g.dst) + slab * g.dst_slab_stride + r * g.dst_row_stride;
+    if (s < 0 || s >= g.n_src_rows) {
+      if (t.width[k] == 16) zero_row<uint4>(dp, g.row_bytes, lane);
+      else if (t.width[k] == 4) zero_row<uint32_t>(dp, g.row_bytes, lane);
+      else zero_row<uint8_t>(dp, g.row_bytes, lane);
+      if (lane == 0) record_error(status, PACE_ERR_INVALID_ARG, K_GATHER_MULTI);
+      continue;
+    }
+    const uint8_t* sp = static_cast<const uint8_t*>(g.src) + slab * g.src_slab_stride + s * g.src_row_stride;
+    if (t.width[k] == 16) copy_row<uint4>(sp, dp, g.row_bytes, lane);
+    else if (t.width[k] == 4) copy_row<uint32_t>(sp, dp, g.row_bytes, lane);
+    else copy_row<uint8_t>(sp, dp, g.row_bytes, lane);
+  }
+}
+
 }  // namespace
 }  // namespace pace
 
@@ -344,5 +437,83 @@ extern "C" pace_status_t pace_gather(const void* src, int64_t n_src_rows, int64_
     gather_rows_bytes<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
         static_cast<const uint8_t*>(src), n_src_rows, row_bytes, idx, n_idx, static_cast<uint8_t*>(dst), status);
   }
+  return check_launch();
+}
+
+extern "C" pace_status_t pace_prune_index(int B, const int32_t* cu_seq, const int32_t* vis_start,
+                                          const int32_t* cu_vis, const int32_t* cu_keep, const int32_t* kept,
+                                          int32_t* out_idx, pace_stream_t stream) {
+  if (B < 0) return PACE_ERR_INVALID_ARG;
+  if (B == 0) return PACE_OK;
+  if (cu_seq == nullptr || vis_start == nullptr || cu_vis == nullptr || cu_keep == nullptr) return PACE_ERR_INVALID_ARG;
+  if (cu_seq[0] != 0 || cu_vis[0] != 0 || cu_keep[0] != 0) return PACE_ERR_INVALID_ARG;
+  int64_t n_out = 0;
+  for (int b = 0; b < B; ++b) {
+    const int n_pre = cu_seq[b + 1] - cu_seq[b], nv = cu_vis[b + 1] - cu_vis[b], nk = cu_keep[b + 1] - cu_keep[b];
+    if (n_pre < 0 || nv < 0 || nk < 0 || nk > nv || vis_start[b] < 0 || vis_start[b] + nv > n_pre)
+      return PACE_ERR_INVALID_ARG;
+    n_out += n_pre - nv + nk;
+  }
+  if (n_out == 0) return PACE_OK;
+  if (out_idx == nullptr || (cu_keep[B] > 0 && kept == nullptr)) return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(check_device());
+  int* status = device_status_word();
+  int post = 0;
+  for (int c0 = 0; c0 < B; c0 += kPruneMaxB) {
+    const int nb = (B - c0) < kPruneMaxB ? (B - c0) : kPruneMaxB;
+    PruneTable t{};
+    t.nb = nb;
+    int max_post = 1;
+    for (int i = 0; i < nb; ++i) {
+      const int b = c0 + i;
+      t.seq0[i] = cu_seq[b];
+      t.n_pre[i] = cu_seq[b + 1] - cu_seq[b];
+      t.vis[i] = vis_start[b];
+      t.v0[i] = cu_vis[b];
+      t.nv[i] = cu_vis[b + 1] - cu_vis[b];
+      t.k0[i] = cu_keep[b];
+      t.nk[i] = cu_keep[b + 1] - cu_keep[b];
+      t.post0[i] = post;
+      const int np = t.n_pre[i] - t.nv[i] + t.nk[i];
+      post += np;
+      if (np > max_post) max_post = np;
+    }
+    const dim3 grid(static_cast<unsigned>(std::min((max_post + 255) / 256, 64)), static_cast<unsigned>(nb));
+    prune_index_kernel<<<grid, 256, 0, stream>>>(t, kept, out_idx, status);
+    PACE_CHECK(check_launch());
+  }
+  return PACE_OK;
+}
+
+extern "C" pace_status_t pace_gather_multi(const pace_gather_tensor* tensors, int n_tensors, const int32_t* idx,
+                                           int64_t n_idx, pace_stream_t stream) {
+  if (n_tensors < 0 || n_tensors > PACE_GATHER_MAX_TENSORS || n_idx < 0) return PACE_ERR_INVALID_ARG;
+  if (n_tensors == 0 || n_idx == 0) return PACE_OK;
+  if (tensors == nullptr || idx == nullptr) return PACE_ERR_INVALID_ARG;
+  GatherMultiTable t{};
+  t.n = n_tensors;
+  t.item_prefix[0] = 0;
+  for (int k = 0; k < n_tensors; ++k) {
+    const pace_gather_tensor& g = tensors[k];
+    if (g.src == nullptr || g.dst == nullptr || g.row_bytes <= 0 || g.n_slabs < 0 || g.n_src_rows < 0 ||
+        g.src_row_stride < g.row_bytes || g.dst_row_stride < g.row_bytes)
+      return PACE_ERR_INVALID_ARG;
+    t.g[k] = g;
+    const uintptr_t a = reinterpret_cast<uintptr_t>(g.src) | reinterpret_cast<uintptr_t>(g.dst) |
+                        static_cast<uintptr_t>(g.row_bytes) | static_cast<uintptr_t>(g.src_row_stride) |
+                        static_cast<uintptr_t>(g.dst_row_stride) | static_cast<uintptr_t>(g.src_slab_stride) |
+                        static_cast<uintptr_t>(g.dst_slab_stride);
+    t.width[k] = (a % 16 == 0) ? 16 : (a % 4 == 0) ? 4 : 1;
+    t.item_prefix[k + 1] = t.item_prefix[k] + g.n_slabs * n_idx;
+  }
+  if (t.item_prefix[n_tensors] == 0) return PACE_OK;
+  PACE_CHECK(check_device());
+  int* status = device_status_word();
+  int sms = 152, dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int64_t blocks = (t.item_prefix[n_tensors] + 7) / 8;
+  const int64_t cap = static_cast<int64_t>(sms) * 16;
+  if (blocks > cap) blocks = cap;
+  gather_multi_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(t, idx, n_idx, status);
   return check_launch();
 }

@@ -135,6 +135,12 @@ pace_status_t pace_selftest_wait_timeout(uint32_t limit_us, pace_stream_t stream
   return pace::check_launch();
 }
 
+int32_t pace_budget_vanilla(int32_t n_vis_vanilla, int32_t n_vis_condensed, double frac) {
+  if (n_vis_condensed <= 0) return 0;
+  const int32_t k = pace_budget(n_vis_vanilla, frac);
+  return k < n_vis_condensed ? k : n_vis_condensed;
+}
+
 int32_t pace_budget(int32_t n_vis, double frac) {
   if (n_vis <= 0 || !(frac > 0.0)) return 0;
   double k = std::floor(frac * static_cast<double>(n_vis) + 0.5);

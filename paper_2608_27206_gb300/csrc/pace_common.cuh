@@ -22,6 +22,8 @@ enum KernelId : int {
   K_DDAE_SELECT = 9,
   K_GATHER = 10,
   K_SELFTEST = 11,
+  K_PRUNE_INDEX = 12,
+  K_GATHER_MULTI = 13,
 };
 
 // Device status word layout: [0] = code (pace_status_t), [1] = kernel id.

@@ -43,6 +43,16 @@ class DdaeParams(ctypes.Structure):
 DDAE_ADAPTIVE, DDAE_ONLY_LLM, DDAE_ONLY_VIT, DDAE_FIXED = 0, 1, 2, 3
 
 
+class GatherTensor(ctypes.Structure):
+    _fields_ = [("src", ctypes.c_void_p), ("dst", ctypes.c_void_p), ("row_bytes", ctypes.c_int64),
+                ("src_row_stride", ctypes.c_int64), ("dst_row_stride", ctypes.c_int64), ("n_slabs", ctypes.c_int64),
+                ("src_slab_stride", ctypes.c_int64), ("dst_slab_stride", ctypes.c_int64),
+                ("n_src_rows", ctypes.c_int64)]
+
+
+GATHER_MAX_TENSORS = 16
+
+
 _P = ctypes.c_void_p
 _I32P = ctypes.POINTER(ctypes.c_int32)
 _I64P = ctypes.POINTER(ctypes.c_int64)
@@ -55,6 +65,9 @@ _SIGS = {
     "pace_device_status": (ctypes.c_int, [_I32P, _I32P, ctypes.c_int]),
     "pace_apc_params_default": (None, [ctypes.POINTER(ApcParams)]),
     "pace_apc_density_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, _I32P]),
+    "pace_budget_vanilla": (ctypes.c_int32, [ctypes.c_int32, ctypes.c_int32, ctypes.c_double]),
+    "pace_prune_index": (ctypes.c_int, [ctypes.c_int, _I32P, _I32P, _I32P, _I32P, _P, _P, _P]),
+    "pace_gather_multi": (ctypes.c_int, [ctypes.POINTER(GatherTensor), ctypes.c_int, _P, ctypes.c_int64, _P]),
     "pace_apc_density_tokens_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, ctypes.c_int]),
     "pace_apc_density_tokens": (ctypes.c_int, [_P, _I32P, ctypes.c_int, ctypes.c_int, _I32P, _I32P,
                                                ctypes.POINTER(ApcParams), _P, _P, _P, ctypes.c_size_t, _P]),
@@ -273,6 +286,44 @@ def pace_apc_density_tokens(T: torch.Tensor, cu_tokens, H, W, params: Optional[A
                                        _dev(stats), _dev(ws), ws.numel(), _stream(stream))
     _check("pace_apc_density_tokens", st)
     return d_out[:n], stats[:B]
+
+
+def pace_budget_vanilla(n_vis_vanilla: int, n_vis_condensed: int, frac: float) -> int:
+    return int(lib().pace_budget_vanilla(int(n_vis_vanilla), int(n_vis_condensed), float(frac)))
+
+
+def pace_prune_index(cu_seq, vis_start, cu_vis, cu_keep, kept: torch.Tensor, out: Optional[torch.Tensor] = None,
+                     stream=None):
+    """Row list of the pruned sequences (global pre-prune rows), int32 on kept's device."""
+    sq, vs, v, kp = _i32(cu_seq), _i32(vis_start), _i32(cu_vis), _i32(cu_keep)
+    B = len(sq) - 1
+    n_out = int((sq[1:] - sq[:-1]).sum() - v[-1] + kp[-1]) if B > 0 else 0
+    if out is None:
+        out = torch.empty(max(n_out, 1), dtype=torch.int32, device=kept.device)
+    st = lib().pace_prune_index(B, _pi32(sq), _pi32(vs), _pi32(v), _pi32(kp), _dev(kept), _dev(out), _stream(stream))
+    _check("pace_prune_index", st)
+    return out[:n_out]
+
+
+def gather_spec(src: torch.Tensor, dst: torch.Tensor, dim: int) -> GatherTensor:
+    """Descriptor for gathering contiguous src along `dim` into contiguous dst: the dimensions
+    before `dim` are slabs, the ones after it form a row."""
+    if not (src.is_contiguous() and dst.is_contiguous()) or src.dtype != dst.dtype:
+        raise ValueError("gather_spec needs contiguous src and dst of one dtype")
+    if src.shape[:dim] != dst.shape[:dim] or src.shape[dim + 1:] != dst.shape[dim + 1:]:
+        raise ValueError("src and dst may differ only along the gathered dimension")
+    es = src.element_size()
+    row = es * int(np.prod(src.shape[dim + 1:], dtype=np.int64))
+    slabs = int(np.prod(src.shape[:dim], dtype=np.int64))
+    return GatherTensor(src.data_ptr(), dst.data_ptr(), row, row, row, slabs, row * src.shape[dim],
+                        row * dst.shape[dim], src.shape[dim])
+
+
+def pace_gather_multi(specs, idx: torch.Tensor, stream=None):
+    """Gathers every GatherTensor in `specs` with the same row list idx (device int32)."""
+    arr = (GatherTensor * max(len(specs), 1))(*specs)
+    st = lib().pace_gather_multi(arr, len(specs), _dev(idx), idx.numel(), _stream(stream))
+    _check("pace_gather_multi", st)
 
 
 def stats_dict(stats: torch.Tensor):

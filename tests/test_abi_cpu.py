@@ -85,3 +85,15 @@ def test_workspace_queries(libpace):
     l = libpace.pace_llm_text_visual_importance_workspace_size([0, 64], [0, 256], 28, 4)
     assert l >= 28 * 128 * 4 + 4 * 256 * 4
     assert libpace.pace_vit_attn_importance_workspace_size([0], 16) == 0
+
+
+def test_budget_vanilla_matches_oracle(libpace):
+    """B = p1 p2 relative to Vanilla, capped at the condensed token count (host helper)."""
+    from oracle import pace_oracle as O
+    rng = np.random.default_rng(9)
+    for _ in range(2000):
+        nv = int(rng.integers(0, 50000))
+        nc = int(rng.integers(0, nv + 1))
+        f = float(rng.choice([0.05, 0.1, 0.25, rng.uniform(0, 1.2)]))
+        assert libpace.pace_budget_vanilla(nv, nc, f) == O.budget_vanilla(nv, nc, f)
+    assert libpace.pace_budget_vanilla(10549, 2660, 0.10) == 1055 and libpace.pace_budget_vanilla(10549, 900, 0.10) == 900

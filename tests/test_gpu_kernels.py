@@ -460,3 +460,48 @@ def test_ddae_select_rejects(pace):
     with pytest.raises(pace.PaceError):
         n = pace.PACE_DDAE_MAX_TOKENS + 1
         _select(pace, np.zeros(n), np.zeros(n), np.array([0, n], np.int32), [1])
+
+
+# ----------------------------------------------------------------------------------------------
+# prune step: row list and multi-tensor gather
+# ----------------------------------------------------------------------------------------------
+def test_prune_index_and_gather_multi(pace):
+    """Pruned LLM context of a batch: row list from the kept tokens, then hidden states,
+    KV-cache rows of two layers and M-RoPE position ids gathered in one launch (byte-exact)."""
+    rng = np.random.default_rng(77)
+    n_vis, pre, post = [300, 17, 1024], [40, 5, 0], [12, 0, 33]
+    cu_vis = np.concatenate([[0], np.cumsum(n_vis)]).astype(np.int32)
+    K = [O.budget(n, 0.1) for n in n_vis]
+    cu_keep = np.concatenate([[0], np.cumsum(K)]).astype(np.int32)
+    sl = rng.gamma(0.5, 2.0, cu_vis[-1]).astype(np.float32)
+    sv = rng.lognormal(0, 1, cu_vis[-1]).astype(np.float32)
+    _, _, kept = pace.pace_ddae_select(torch.from_numpy(sl).cuda(), torch.from_numpy(sv).cuda(), cu_vis, cu_keep)
+    n_pre = [a + b + c for a, b, c in zip(pre, n_vis, post)]
+    cu_seq = np.concatenate([[0], np.cumsum(n_pre)]).astype(np.int32)
+    idx = pace.pace_prune_index(cu_seq, pre, cu_vis, cu_keep, kept)
+    kept_h = kept.cpu().numpy()
+    ref = np.concatenate([O.prune_rows(n_pre[b], pre[b], n_vis[b], kept_h[cu_keep[b]:cu_keep[b + 1]] - cu_vis[b])
+                          + cu_seq[b] for b in range(3)])
+    np.testing.assert_array_equal(idx.cpu().numpy(), ref)
+    S, n = int(cu_seq[-1]), len(ref)
+    hid = torch.randn(S, 896, device="cuda").to(torch.bfloat16)               # hidden states [S, D]
+    kv = torch.randn(2, 2, 4, S, 128, device="cuda").to(torch.bfloat16)       # [layer, K/V, head, S, d]
+    pos = torch.randint(0, 1 << 20, (3, S), device="cuda", dtype=torch.int64)  # M-RoPE ids [3, S]
+    odd = torch.randint(0, 255, (S, 7), device="cuda", dtype=torch.uint8)     # 7-byte rows: byte path
+    outs = [torch.empty(n, 896, dtype=torch.bfloat16, device="cuda"),
+            torch.empty(2, 2, 4, n, 128, dtype=torch.bfloat16, device="cuda"),
+            torch.empty(3, n, dtype=torch.int64, device="cuda"), torch.empty(n, 7, dtype=torch.uint8, device="cuda")]
+    specs = [pace.gather_spec(hid, outs[0], 0), pace.gather_spec(kv, outs[1], 3), pace.gather_spec(pos, outs[2], 1),
+             pace.gather_spec(odd, outs[3], 0)]
+    pace.pace_gather_multi(specs, idx)
+    r = torch.from_numpy(ref).cuda().long()
+    assert torch.equal(outs[0], hid[r]) and torch.equal(outs[1], kv[:, :, :, r]) and torch.equal(outs[2], pos[:, r])
+    assert torch.equal(outs[3], odd[r])
+    _no_device_error(pace)
+    bad = torch.tensor([0, S + 5], dtype=torch.int32, device="cuda")           # out of range: zero row + status
+    o2 = torch.full((2, 896), 7, dtype=torch.bfloat16, device="cuda")
+    pace.pace_gather_multi([pace.gather_spec(hid, o2, 0)], bad)
+    torch.cuda.synchronize()
+    code, where = pace.pace_device_status(clear=True)
+    assert code == 1 and where == 13
+    assert torch.equal(o2[0], hid[0]) and bool((o2[1] == 0).all())

@@ -351,3 +351,18 @@ def test_preview_tokens_zero_rows_and_identity():
     assert st2["phi"] == pytest.approx(1.0) and st2["rho_g"] == pytest.approx(0.0, abs=1e-12)
     assert np.all(np.abs(st2["d"]) < 1e-7)
     assert (st2["H_out"], st2["W_out"]) == (28, 28)                                # r = 0
+
+
+def test_prune_rows_against_position_loop():
+    """The pruned sequence keeps text positions and the kept visual positions, in order
+    (checked against a plain loop over positions)."""
+    rng = np.random.default_rng(3)
+    for _ in range(50):
+        n_vis = int(rng.integers(0, 60))
+        pre, post = int(rng.integers(0, 20)), int(rng.integers(0, 20))
+        kept = np.sort(rng.choice(n_vis, size=int(rng.integers(0, n_vis + 1)), replace=False)) if n_vis else []
+        rows = O.prune_rows(pre + n_vis + post, pre, n_vis, kept)
+        ks = set(int(k) for k in kept)
+        expect = [p for p in range(pre + n_vis + post) if not (pre <= p < pre + n_vis) or (p - pre) in ks]
+        np.testing.assert_array_equal(rows, expect)
+        assert len(rows) == pre + post + len(kept)       # S_post = T + N_keep
