@@ -245,6 +245,45 @@ PACE_API pace_status_t pace_llm_text_visual_importance(const void* Q, const void
                                               int head_dim, float scale, float* s_llm_raw, void* ws,
                                               size_t ws_bytes, pace_stream_t stream);
 
+/* Query sets of the full-sequence S_llm (App. "Impact of Attention Token Sources"): every
+ * position from the first visual token on (Vision + Text, the paper's default), the text
+ * positions after the visual span, or the last position only. */
+typedef enum pace_query_set {
+  PACE_QUERY_VISION_TEXT = 0,
+  PACE_QUERY_TEXT = 1,
+  PACE_QUERY_LAST = 2
+} pace_query_set;
+
+/* Scratch bytes for pace_llm_sequence_importance (host arrays as there); 0 if they are invalid. */
+PACE_API size_t pace_llm_sequence_importance_workspace_size(int B, const int32_t* cu_seq, const int32_t* vis_start,
+                                                  const int32_t* n_vis, int n_q_heads, int n_kv_heads,
+                                                  int query_set);
+
+/*
+ * Full-sequence S_llm (Sec. 3.3; App. B.3, layer L_ext = 2; App. "Impact of Attention Token
+ * Sources").  Sequence b is positions 0 .. S_b - 1 of a causal LLM prefill (system, visual
+ * and text tokens), its visual tokens at positions v_b .. v_b + N_b - 1.  For query head h
+ * (KV head g = h / (n_q_heads / n_kv_heads)) and query position q in the query set P_b:
+ * u_j = sum_h sum_{q in P_b} softmax_{k <= q}(scale q_qh . k_kg)[v_b + j],
+ * the softmax over every position up to q.  P_b = {v_b .. S_b - 1} (VISION_TEXT),
+ * {v_b + N_b .. S_b - 1} (TEXT; empty when the visual span ends the sequence, giving zeros)
+ * or {S_b - 1} (LAST).
+ *
+ *  Q           device  bf16 [sum S, n_q_heads, head_dim]  (queries of every position)
+ *  K           device  bf16 [sum S, n_kv_heads, head_dim]
+ *  cu_seq      host    int32 [B+1] prefix sums of S_b >= 1
+ *  vis_start   host    int32 [B]   v_b >= 0
+ *  n_vis       host    int32 [B]   N_b >= 1, v_b + N_b <= S_b
+ *  query_set   pace_query_set
+ *  s_llm_raw   device  float [sum N_b]
+ *  sum S + 128 B <= 2^30.  Invalid arguments: PACE_ERR_INVALID_ARG before any launch.
+ */
+PACE_API pace_status_t pace_llm_sequence_importance(const void* Q, const void* K, const int32_t* cu_seq,
+                                          const int32_t* vis_start, const int32_t* n_vis, int B,
+                                          int n_q_heads, int n_kv_heads, int head_dim, float scale,
+                                          int query_set, float* s_llm_raw, void* ws, size_t ws_bytes,
+                                          pace_stream_t stream);
+
 /* Fusion of the two maps.  ADAPTIVE is Eq. 7; the other three are the fusion ablations of
  * Sec. 4 ("Effect of Attention Fusion in DDAE"): Only LLM-Attn (alpha_w = 1, beta_w = 0), Only
  * ViT-Attn (alpha_w = 0, beta_w = 1) and Fixed Fusion (0.5 / 0.5). */

@@ -222,6 +222,58 @@ def llm_text_visual_importance(Q: np.ndarray, K: np.ndarray, cu_q: Sequence[int]
     return np.concatenate(out) if out else np.zeros(0)
 
 
+# Query sets of the full-sequence S_llm (App. "Impact of Attention Token Sources"): all sequence
+# tokens (Vision + Text, the paper's default, App. B.3 "averaged uniformly across all valid
+# tokens"), the text tokens only, or the last token only.
+QUERY_SETS = ("vision_text", "text", "last")
+
+
+def query_start(n_seq: int, vis_start: int, n_vis: int, query_set: str) -> int:
+    """First query position; the query set is positions query_start .. n_seq - 1.  Positions
+    before the visual span cannot attend to it (causal mask), so they are left out."""
+    if query_set == "vision_text":
+        return vis_start
+    if query_set == "text":
+        return vis_start + n_vis
+    if query_set == "last":
+        return n_seq - 1
+    raise ValueError(query_set)
+
+
+def llm_sequence_importance(Q: np.ndarray, K: np.ndarray, cu_seq: Sequence[int], vis_start: Sequence[int],
+                            n_vis: Sequence[int], scale: float, query_set: str = "vision_text",
+                            rows_per_block: int = 256) -> np.ndarray:
+    """Full-sequence S_llm (Sec. 3.3; App. B.3; App. "Impact of Attention Token Sources").
+
+    Q float64 [sum S, Hq, d], K float64 [sum S, Hkv, d]: queries and keys of every position of
+    each causal LLM sequence at the extraction layer.  For sequence b with its visual tokens at
+    positions v .. v + N_vis - 1 and query set P: S_llm[j] = sum_h sum_{q in P}
+    softmax_{k <= q}(scale q_q . k_k)[v + j], the softmax over every earlier position (system,
+    visual and text tokens).  GQA head h reads KV head h // (Hq / Hkv).  Returns [sum N_vis].
+    """
+    Hq, Hkv = Q.shape[1], K.shape[1]
+    group = Hq // Hkv
+    out: List[np.ndarray] = []
+    for b in range(len(cu_seq) - 1):
+        s0, s1 = int(cu_seq[b]), int(cu_seq[b + 1])
+        S, v, nv = s1 - s0, int(vis_start[b]), int(n_vis[b])
+        q_lo = query_start(S, v, nv, query_set)
+        u = np.zeros(nv)
+        for h in range(Hq):
+            Kh = K[s0:s1, h // group]
+            for i0 in range(q_lo, S, rows_per_block):
+                i1 = min(S, i0 + rows_per_block)
+                logits = (Q[s0 + i0:s0 + i1, h] @ Kh.T) * scale           # [rows, S]
+                pos_q = np.arange(i0, i1)[:, None]
+                logits = np.where(np.arange(S)[None, :] <= pos_q, logits, -np.inf)   # causal
+                logits -= logits.max(axis=1, keepdims=True)
+                p = np.exp(logits)
+                p /= p.sum(axis=1, keepdims=True)
+                u += p[:, v:v + nv].sum(axis=0)
+        out.append(u)
+    return np.concatenate(out) if out else np.zeros(0)
+
+
 def min_max(x: np.ndarray) -> np.ndarray:
     """Sec. 3.3: min-max normalisation to [0, 1]; a constant map becomes 0 (R8)."""
     lo, hi = float(x.min()), float(x.max())

@@ -41,6 +41,7 @@
 #include <atomic>
 #include <cmath>
 #include <mutex>
+#include <vector>
 
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
@@ -60,6 +61,7 @@ constexpr int kEpiWarps = 16;
 constexpr int kThreads = 64 + 32 * kEpiWarps;   // 576
 constexpr int kAttnMaxB = 64;
 constexpr uint32_t kTmemCols = 512;
+constexpr int kNoMask = 1 << 29;          // diag of a non-causal image: every key is seen
 constexpr int kTargetItems = 152;         // work items (two CTAs each): two waves over the SMs
 
 // An operand tile of ROWS rows and head dimension D is stored as NB blocks of 64 columns
@@ -121,6 +123,8 @@ __device__ __forceinline__ void store_shift_row(uint16_t* row, float v) {
 struct AttnTable {
   int q0[kAttnMaxB], nq[kAttnMaxB];   // query rows of image b
   int k0[kAttnMaxB], nk[kAttnMaxB];   // key rows of image b
+  int diag[kAttnMaxB];                // causal mask: local key k is seen by local query i iff k <= i + diag
+  int out0[kAttnMaxB];                // first part-map row of image b (pass 2)
   int lpad[kAttnMaxB];                // first padded L row of image b (multiple of 256)
   int item_prefix[kAttnMaxB + 1];
   int nb;
@@ -311,6 +315,14 @@ __device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], float c, flo
   return fadd2(acc, a1);
 }
 
+// colsum64 over the columns e >= lo only (the causal mask of pass 2).
+__device__ __forceinline__ float2 colsum64_from(const uint32_t (&v)[64], int lo, float c, float2 acc) {
+  uint32_t w[64];
+#pragma unroll
+  for (int e = 0; e < 64; ++e) w[e] = e < lo ? 0xFF800000u : v[e];   // -inf: 2^(c * -inf) = 0
+  return colsum64(w, c, acc);
+}
+
 // Brings the CTA to a quiet point: waits for its MMAs (phase `done_phase` of b_done) and lets
 // in-flight copies land after an abort; TMEM stays allocated.
 __device__ __forceinline__ void cta_quiesce(SmemCtl* ctl, uint32_t b_done, uint32_t done_phase, int* status,
@@ -339,7 +351,7 @@ __device__ __forceinline__ void cta_release_tmem(uint32_t tmem) {
 // ------------------------------------------------------------------------------------------------
 // pass 1: row log-sum-exp
 // ------------------------------------------------------------------------------------------------
-template <int D>
+template <int D, bool CAUSAL>
 __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constant__ CUtensorMap tmq,
                                                             const __grid_constant__ CUtensorMap tmq32,
                                                             const __grid_constant__ CUtensorMap tmk,
@@ -369,14 +381,18 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
   const int split = r % t.splits;
   r /= t.splits;
   const int npair = (t.nq[b] + kPair - 1) / kPair;
-  const int pair = r % npair;
+  const int diag = t.diag[b];
+  // causal images: the last query rows see the most keys, so they are scheduled first
+  const int pair = CAUSAL ? npair - 1 - r % npair : r % npair;
   const int h = r / npair;
   const int g = h / t.G;
   const int qrow0 = pair * kPair + kTile * static_cast<int>(rank);     // this CTA's first local query row
   const int nkt_all = (t.nk[b] + kStream - 1) / kStream;
   const int kt0 = static_cast<int>((static_cast<int64_t>(split) * nkt_all) / t.splits);
-  const int kt1 = static_cast<int>((static_cast<int64_t>(split + 1) * nkt_all) / t.splits);
-  const int nj = kt1 - kt0;
+  // causal: key tiles past the one holding key qrow0 + 127 + diag are masked for every row (diag >= 0)
+  const int kt1_all = static_cast<int>((static_cast<int64_t>(split + 1) * nkt_all) / t.splits);
+  const int kt1 = CAUSAL ? min(kt1_all, (diag + qrow0 + kTile - 1) / kStream + 1) : kt1_all;
+  const int nj = max(kt1 - kt0, 0);
 
   if (threadIdx.x == 0) {
     mbar_init(b_qfull, 1);
@@ -473,7 +489,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
           break;
         }
         tc_fence_after_sync();
-        const int valid = t.nk[b] - ((kt0 + j) * kStream + hh * 128);   // keys of these columns in the image
+        // keys of these columns that the row sees: inside the image and, if causal, k <= row + diag
+        const int cs = (kt0 + j) * kStream + hh * 128;
+        const int valid = CAUSAL ? min(t.nk[b] - cs, diag + qrow0 + rr - cs + 1) : t.nk[b] - cs;
         uint32_t sv[64];
         load_cols64(tbuf, sv);
         if (round == 0) lse_fixed(sv, valid, c, m_run, l_run);
@@ -559,7 +577,7 @@ __global__ void __launch_bounds__(128) attn_lse_combine(const __grid_constant__ 
 // ------------------------------------------------------------------------------------------------
 // pass 2: column sums of 2^(c s - L)
 // ------------------------------------------------------------------------------------------------
-template <int D>
+template <int D, bool CAUSAL>
 __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant__ CUtensorMap tmq,
                                                            const __grid_constant__ CUtensorMap tmq32,
                                                            const __grid_constant__ CUtensorMap tmk,
@@ -593,8 +611,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
   const int kp = r % nkp;
   const int g = r / nkp;
   const int krow0 = kp * kPair + kTile * static_cast<int>(rank);     // this CTA's first local key row
+  const int diag = t.diag[b];
   const int nqt = (t.nq[b] + kStream - 1) / kStream;
-  const int nj = t.G * nqt;                                           // stream: (head in group, query tile)
+  // causal images: query tiles that end before row krow0 - diag see none of this CTA's keys
+  const int qt_min = CAUSAL && krow0 > diag ? (krow0 - diag) / kStream : 0;
+  const int nspan = max(nqt - qt_min, 0);
+  const int nj = t.G * nspan;                                         // stream: (head in group, query tile)
 
   if (threadIdx.x == 0) {
     mbar_init(b_afull, 1);
@@ -638,7 +660,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
           break;
         }
         if (aborted(ctl)) break;
-        const int hq = j / nqt, qt = j - hq * nqt;
+        const int hq = j / nspan, qt = qt_min + j - hq * nspan;
         const int h = g * t.G + hq;
         uint8_t* st = sQ + s * B2;
         mbar_arrive_expect_tx(b_qfull(s), B2);
@@ -685,6 +707,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
     const int rr = quad * 32 + lane;
     float2 acc = make_float2(0.f, 0.f);
     const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
+    const int key = krow0 + rr;
     for (int j = p; j < nj; j += 2) {
       const int v = j >> 1;
       const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs));
@@ -693,22 +716,28 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
         break;
       }
       tc_fence_after_sync();
+      // causal mask: query columns before `lo` do not see this thread's key
+      int lo = 0;
+      bool masked = false;
+      if (CAUSAL) {
+        lo = key - diag - ((qt_min + j % nspan) * kStream + hh * 128);
+        masked = __any_sync(0xffffffffu, lo > 0);
+      }
       uint32_t sv[64];
       load_cols64(tbuf, sv);
-      acc = colsum64(sv, c, acc);
+      acc = masked ? colsum64_from(sv, lo, c, acc) : colsum64(sv, c, acc);
       load_cols64(tbuf + 64, sv);
       tc_fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(b_sfree(p));
-      acc = colsum64(sv, c, acc);
+      acc = masked ? colsum64_from(sv, lo - 64, c, acc) : colsum64(sv, c, acc);
     }
     const float a = acc.x + acc.y;
     if (e > 0) ctl->xchg[e - 1][0][rr] = a;
     named_barrier_sync(1, 32 * kEpiWarps);
     if (e == 0) {
-      const int key = krow0 + rr;
       if (key < t.nk[b])
-        part[static_cast<int64_t>(g) * t.ktot + t.k0[b] + key] =
+        part[static_cast<int64_t>(g) * t.ktot + t.out0[b] + key] =
             (a + ctl->xchg[0][0][rr]) + (ctl->xchg[1][0][rr] + ctl->xchg[2][0][rr]);
     }
   }
@@ -765,20 +794,28 @@ pace_status_t make_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t co
   return PACE_OK;
 }
 
+// One image of a call.  Pass 1: queries q0 .. q0 + nq - 1 of Q against keys k0 .. k0 + nk - 1
+// of K, key k seen by query i iff k <= i + diag (diag >= 0).  Pass 2: the same queries against
+// the scored keys v0 .. v0 + nv - 1 (rows of K), key j seen by query i iff j <= i + vdiag;
+// scores go to output rows out0 .. out0 + nv - 1.
+struct Seg {
+  int q0, nq, k0, nk, diag;
+  int v0, nv, vdiag, out0;
+};
+
 struct AttnLayout {
   int splits;
-  int64_t prows, ktot, qtot;
+  int64_t prows, ktot;
   size_t L_off, part_off, ml_off, total;
 };
 
 // Key splits of pass 1: enough work items to cover the GPU about twice.
-int choose_splits(int B, const int32_t* cu_q, const int32_t* cu_k, int H) {
+int choose_splits(const std::vector<Seg>& segs, int H) {
   int64_t items = 0;
   int max_kt = 1;
-  for (int b = 0; b < B; ++b) {
-    const int nq = cu_q[b + 1] - cu_q[b], nk = cu_k[b + 1] - cu_k[b];
-    items += static_cast<int64_t>(H) * ((nq + kPair - 1) / kPair);
-    max_kt = std::max(max_kt, (nk + kStream - 1) / kStream);
+  for (const Seg& sg : segs) {
+    items += static_cast<int64_t>(H) * ((sg.nq + kPair - 1) / kPair);
+    max_kt = std::max(max_kt, (sg.nk + kStream - 1) / kStream);
   }
   if (items >= kTargetItems || items == 0) return 1;
   int s = static_cast<int>((kTargetItems + items - 1) / items);
@@ -786,20 +823,48 @@ int choose_splits(int B, const int32_t* cu_q, const int32_t* cu_k, int H) {
   return std::max(s, 1);
 }
 
-AttnLayout attn_layout(int B, const int32_t* cu_q, const int32_t* cu_k, int H, int groups) {
+AttnLayout attn_layout(const std::vector<Seg>& segs, int H, int groups) {
   AttnLayout L{};
-  L.splits = choose_splits(B, cu_q, cu_k, H);
-  L.qtot = cu_q[B];
-  L.ktot = cu_k[B];
-  int64_t pr = 0;
-  for (int b = 0; b < B; ++b) pr += static_cast<int64_t>((cu_q[b + 1] - cu_q[b] + kPair - 1) / kPair) * kPair;
+  L.splits = choose_splits(segs, H);
+  int64_t pr = 0, kt = 0;
+  for (const Seg& sg : segs) {
+    pr += static_cast<int64_t>((sg.nq + kPair - 1) / kPair) * kPair;
+    kt += sg.nv;
+  }
   L.prows = pr;   // every image's L rows start on a 256-row (1 KB) boundary
+  L.ktot = kt;
   L.L_off = 0;
   L.part_off = align_up(static_cast<size_t>(H) * L.prows * kShiftCols * 2, 256);
   L.ml_off = L.part_off + align_up(static_cast<size_t>(groups) * L.ktot * sizeof(float), 256);
   L.total = L.ml_off;
   if (L.splits > 1) L.total += align_up(static_cast<size_t>(L.splits) * H * L.prows * sizeof(float2), 256);
   return L;
+}
+
+// Non-causal images: queries cu_q[b] .. against keys cu_k[b] .. in both passes.
+std::vector<Seg> cross_segs(int B, const int32_t* cu_q, const int32_t* cu_k) {
+  std::vector<Seg> segs(static_cast<size_t>(std::max(B, 0)));
+  for (int b = 0; b < B; ++b) {
+    const int nq = cu_q[b + 1] - cu_q[b], nk = cu_k[b + 1] - cu_k[b];
+    segs[b] = Seg{cu_q[b], nq, cu_k[b], nk, kNoMask, cu_k[b], nk, kNoMask, cu_k[b]};
+  }
+  return segs;
+}
+
+// Causal sequences (full-sequence S_llm): image b is positions cu_seq[b] .. cu_seq[b+1] - 1 of Q
+// and K, its visual tokens at local positions v .. v + nv - 1, queries from local position q_lo
+// (the query set) to the end.
+std::vector<Seg> sequence_segs(int B, const int32_t* cu_seq, const int32_t* vis_start, const int32_t* n_vis,
+                               int query_set) {
+  std::vector<Seg> segs(static_cast<size_t>(std::max(B, 0)));
+  int out0 = 0;
+  for (int b = 0; b < B; ++b) {
+    const int S = cu_seq[b + 1] - cu_seq[b], v = vis_start[b], nv = n_vis[b];
+    const int q_lo = query_set == PACE_QUERY_VISION_TEXT ? v : query_set == PACE_QUERY_TEXT ? v + nv : S - 1;
+    segs[b] = Seg{cu_seq[b] + q_lo, S - q_lo, cu_seq[b], S, q_lo, cu_seq[b] + v, nv, q_lo - v, out0};
+    out0 += nv;
+  }
+  return segs;
 }
 
 pace_status_t check_segments(int B, const int32_t* cu, int multiple) {
@@ -813,7 +878,7 @@ pace_status_t check_segments(int B, const int32_t* cu, int multiple) {
 
 // Opts the two passes into their shared-memory size, once per device (so that later
 // calls, including ones made during stream capture, only launch).
-template <int D>
+template <int D, bool CAUSAL>
 pace_status_t set_smem_attrs(size_t* s1, size_t* s2) {
   using C = Cfg<D>;
   *s1 = 1024 + C::A::BYTES + C::STAGES * C::B::BYTES + sizeof(SmemCtl);
@@ -824,8 +889,10 @@ pace_status_t set_smem_attrs(size_t* s1, size_t* s2) {
   PACE_CUDA(cudaGetDevice(&dev));
   const uint64_t bit = uint64_t{1} << (dev & 63);
   if (done.load(std::memory_order_acquire) & bit) return PACE_OK;
-  PACE_CUDA(cudaFuncSetAttribute(attn_row_lse<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(*s1)));
-  PACE_CUDA(cudaFuncSetAttribute(attn_colsum<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(*s2)));
+  PACE_CUDA(cudaFuncSetAttribute(attn_row_lse<D, CAUSAL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(*s1)));
+  PACE_CUDA(cudaFuncSetAttribute(attn_colsum<D, CAUSAL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(*s2)));
   done.fetch_or(bit, std::memory_order_acq_rel);
   return PACE_OK;
 }
@@ -838,29 +905,32 @@ pace_status_t launch_pairs(void (*kernel)(Params...), int items, size_t smem, cu
   return check_launch();
 }
 
-template <int D>
-pace_status_t run_importance(const void* Q, const void* K, const int32_t* cu_q, const int32_t* cu_k, int B, int Hq,
-                             int Hkv, float scale, int merge, float* out, void* ws, cudaStream_t stream) {
+template <int D, bool CAUSAL>
+pace_status_t run_importance(const void* Q, const void* K, int64_t qrows, int64_t krows,
+                             const std::vector<Seg>& segs, int Hq, int Hkv, float scale, int merge, float* out,
+                             void* ws, cudaStream_t stream) {
+  const int B = static_cast<int>(segs.size());
   const int G = Hq / Hkv;
-  const AttnLayout Lay = attn_layout(B, cu_q, cu_k, Hq, Hkv);
+  const AttnLayout Lay = attn_layout(segs, Hq, Hkv);
   uint8_t* w8 = static_cast<uint8_t*>(ws);
   uint16_t* Lw = reinterpret_cast<uint16_t*>(w8 + Lay.L_off);
   float* part = reinterpret_cast<float*>(w8 + Lay.part_off);
   float2* ml = Lay.splits > 1 ? reinterpret_cast<float2*>(w8 + Lay.ml_off) : nullptr;
   int* status = device_status_word();
   CUtensorMap mq, mq32, mk, mk32;
-  const int64_t qrows = std::max<int64_t>(Lay.qtot, 1), krows = std::max<int64_t>(Lay.ktot, 1);
+  qrows = std::max<int64_t>(qrows, 1);
+  krows = std::max<int64_t>(krows, 1);
   PACE_CHECK(make_map(&mq, Q, qrows, static_cast<int64_t>(Hq) * D, true));
   PACE_CHECK(make_map(&mk, K, krows, static_cast<int64_t>(Hkv) * D, true));
   PACE_CHECK(make_map(&mq32, Q, qrows, static_cast<int64_t>(Hq) * D, false));
   PACE_CHECK(make_map(&mk32, K, krows, static_cast<int64_t>(Hkv) * D, false));
   CUtensorMap mshift, mones;
-  PACE_CHECK(make_map(&mshift, Lw, static_cast<int64_t>(Hq) * Lay.prows, kShiftCols, false));
+  PACE_CHECK(make_map(&mshift, Lw, std::max<int64_t>(static_cast<int64_t>(Hq) * Lay.prows, 1), kShiftCols, false));
   const void* ones = nullptr;
   PACE_CUDA(cudaGetSymbolAddress(const_cast<void**>(&ones), g_ones_slice));
   PACE_CHECK(make_map(&mones, ones, kTile, kShiftCols, false));
   size_t s1 = 0, s2 = 0;
-  PACE_CHECK(set_smem_attrs<D>(&s1, &s2));
+  PACE_CHECK((set_smem_attrs<D, CAUSAL>(&s1, &s2)));
   const float c = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634);
   int lpad = 0;
   for (int c0 = 0; c0 < B; c0 += kAttnMaxB) {
@@ -875,33 +945,66 @@ pace_status_t run_importance(const void* Q, const void* K, const int32_t* cu_q, 
     int items1 = 0, ctiles = 0;
     t.item_prefix[0] = 0;
     for (int i = 0; i < nb; ++i) {
-      const int b = c0 + i;
-      t.q0[i] = cu_q[b];
-      t.nq[i] = cu_q[b + 1] - cu_q[b];
-      t.k0[i] = cu_k[b];
-      t.nk[i] = cu_k[b + 1] - cu_k[b];
+      const Seg& sg = segs[c0 + i];
+      t.q0[i] = sg.q0;
+      t.nq[i] = sg.nq;
+      t.k0[i] = sg.k0;
+      t.nk[i] = sg.nk;
+      t.diag[i] = sg.diag;
       t.lpad[i] = lpad;
-      lpad += (t.nq[i] + kPair - 1) / kPair * kPair;
-      items1 += Hq * ((t.nq[i] + kPair - 1) / kPair) * Lay.splits;
+      lpad += (sg.nq + kPair - 1) / kPair * kPair;
+      items1 += Hq * ((sg.nq + kPair - 1) / kPair) * Lay.splits;
       t.item_prefix[i + 1] = items1;
-      ctiles += (t.nq[i] + kPair - 1) / kPair * 2;
+      ctiles += (sg.nq + kPair - 1) / kPair * 2;
     }
-    PACE_CHECK(launch_pairs(attn_row_lse<D>, items1, s1, stream, mq, mq32, mk, mk32, t, c, Lw, ml, status));
-    if (Lay.splits > 1) {
+    PACE_CHECK(launch_pairs(attn_row_lse<D, CAUSAL>, items1, s1, stream, mq, mq32, mk, mk32, t, c, Lw, ml, status));
+    if (Lay.splits > 1 && ctiles > 0) {
       attn_lse_combine<<<dim3(ctiles, Hq), kTile, 0, stream>>>(t, c, ml, Lw);
       PACE_CHECK(check_launch());
     }
+    // pass 2 streams the same query rows (and L rows) against the scored keys
     int items2 = 0;
     for (int i = 0; i < nb; ++i) {
-      items2 += Hkv * ((t.nk[i] + kPair - 1) / kPair);
+      const Seg& sg = segs[c0 + i];
+      t.k0[i] = sg.v0;
+      t.nk[i] = sg.nv;
+      t.diag[i] = sg.vdiag;
+      t.out0[i] = sg.out0;
+      items2 += Hkv * ((sg.nv + kPair - 1) / kPair);
       t.item_prefix[i + 1] = items2;
     }
-    PACE_CHECK(launch_pairs(attn_colsum<D>, items2, s2, stream, mq, mq32, mk, mk32, mshift, mones, t, c, part,
+    PACE_CHECK(launch_pairs(attn_colsum<D, CAUSAL>, items2, s2, stream, mq, mq32, mk, mk32, mshift, mones, t, c, part,
                             status));
   }
   const int nout = static_cast<int>(Lay.ktot / merge);
-  attn_reduce<<<(nout + 255) / 256, 256, 0, stream>>>(part, Hkv, static_cast<int>(Lay.ktot), merge, out);
-  return check_launch();
+  if (nout > 0) {
+    attn_reduce<<<(nout + 255) / 256, 256, 0, stream>>>(part, Hkv, static_cast<int>(Lay.ktot), merge, out);
+    PACE_CHECK(check_launch());
+  }
+  return PACE_OK;
+}
+
+pace_status_t check_heads(int Hq, int Hkv, int D, float scale, const void* Q, const void* K) {
+  if (Q == nullptr || K == nullptr) return PACE_ERR_INVALID_ARG;
+  if (Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || Hq > 256) return PACE_ERR_INVALID_ARG;
+  if (D != 64 && D != 80 && D != 128) return PACE_ERR_INVALID_ARG;
+  if (!(scale > 0.f) || !std::isfinite(scale)) return PACE_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(Q) | reinterpret_cast<uintptr_t>(K)) % 16) return PACE_ERR_INVALID_ARG;
+  return PACE_OK;
+}
+
+template <bool CAUSAL>
+pace_status_t dispatch(const void* Q, const void* K, int64_t qrows, int64_t krows, const std::vector<Seg>& segs,
+                       int Hq, int Hkv, int D, float scale, int merge, float* out, void* ws, size_t ws_bytes,
+                       cudaStream_t stream) {
+  const AttnLayout Lay = attn_layout(segs, Hq, Hkv);
+  if (ws == nullptr || ws_bytes < Lay.total || reinterpret_cast<uintptr_t>(ws) % 16) return PACE_ERR_WORKSPACE;
+  PACE_CHECK(check_device());
+  switch (D) {
+    case 64: return run_importance<64, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream);
+    case 80: return run_importance<80, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream);
+    default: return run_importance<128, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream);
+  }
 }
 
 pace_status_t importance(const void* Q, const void* K, const int32_t* cu_q, const int32_t* cu_k, int B, int Hq,
@@ -909,22 +1012,28 @@ pace_status_t importance(const void* Q, const void* K, const int32_t* cu_q, cons
                          cudaStream_t stream) {
   if (B < 0) return PACE_ERR_INVALID_ARG;
   if (B == 0) return PACE_OK;
-  if (Q == nullptr || K == nullptr || out == nullptr) return PACE_ERR_INVALID_ARG;
-  if (Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || Hq > 256) return PACE_ERR_INVALID_ARG;
-  if (D != 64 && D != 80 && D != 128) return PACE_ERR_INVALID_ARG;
-  if (!(scale > 0.f) || !std::isfinite(scale)) return PACE_ERR_INVALID_ARG;
-  if ((reinterpret_cast<uintptr_t>(Q) | reinterpret_cast<uintptr_t>(K)) % 16) return PACE_ERR_INVALID_ARG;
+  if (out == nullptr) return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(check_heads(Hq, Hkv, D, scale, Q, K));
   PACE_CHECK(check_segments(B, cu_q, cu_q == cu_k ? merge : 1));
   if (cu_k != cu_q) PACE_CHECK(check_segments(B, cu_k, merge));
   if (static_cast<int64_t>(cu_q[B]) + static_cast<int64_t>(kTile) * B > (int64_t{1} << 30)) return PACE_ERR_INVALID_ARG;
-  const AttnLayout Lay = attn_layout(B, cu_q, cu_k, Hq, Hkv);
-  if (ws == nullptr || ws_bytes < Lay.total || reinterpret_cast<uintptr_t>(ws) % 16) return PACE_ERR_WORKSPACE;
-  PACE_CHECK(check_device());
-  switch (D) {
-    case 64: return run_importance<64>(Q, K, cu_q, cu_k, B, Hq, Hkv, scale, merge, out, ws, stream);
-    case 80: return run_importance<80>(Q, K, cu_q, cu_k, B, Hq, Hkv, scale, merge, out, ws, stream);
-    default: return run_importance<128>(Q, K, cu_q, cu_k, B, Hq, Hkv, scale, merge, out, ws, stream);
+  return dispatch<false>(Q, K, cu_q[B], cu_k[B], cross_segs(B, cu_q, cu_k), Hq, Hkv, D, scale, merge, out, ws, ws_bytes,
+                  stream);
+}
+
+// Checks the sequence layout of the full-sequence S_llm.
+pace_status_t check_sequences(int B, const int32_t* cu_seq, const int32_t* vis_start, const int32_t* n_vis,
+                              int query_set) {
+  if (cu_seq == nullptr || vis_start == nullptr || n_vis == nullptr || cu_seq[0] != 0) return PACE_ERR_INVALID_ARG;
+  if (query_set != PACE_QUERY_VISION_TEXT && query_set != PACE_QUERY_TEXT && query_set != PACE_QUERY_LAST)
+    return PACE_ERR_INVALID_ARG;
+  for (int b = 0; b < B; ++b) {
+    const int64_t S = static_cast<int64_t>(cu_seq[b + 1]) - cu_seq[b];
+    if (S < 1 || vis_start[b] < 0 || n_vis[b] < 1 || static_cast<int64_t>(vis_start[b]) + n_vis[b] > S)
+      return PACE_ERR_INVALID_ARG;
   }
+  if (static_cast<int64_t>(cu_seq[B]) + static_cast<int64_t>(kTile) * B > (int64_t{1} << 30)) return PACE_ERR_INVALID_ARG;
+  return PACE_OK;
 }
 
 }  // namespace
@@ -934,7 +1043,7 @@ using namespace pace;
 
 extern "C" size_t pace_vit_attn_importance_workspace_size(int B, const int32_t* cu_seqlens, int n_heads) {
   if (B <= 0 || cu_seqlens == nullptr || n_heads < 1) return 0;
-  return attn_layout(B, cu_seqlens, cu_seqlens, n_heads, n_heads).total;
+  return attn_layout(cross_segs(B, cu_seqlens, cu_seqlens), n_heads, n_heads).total;
 }
 
 extern "C" pace_status_t pace_vit_attn_importance(const void* Q, const void* K, const int32_t* cu_seqlens, int B,
@@ -949,7 +1058,7 @@ extern "C" pace_status_t pace_vit_attn_importance(const void* Q, const void* K, 
 extern "C" size_t pace_llm_text_visual_importance_workspace_size(int B, const int32_t* cu_q, const int32_t* cu_k,
                                                                  int n_q_heads, int n_kv_heads) {
   if (B <= 0 || cu_q == nullptr || cu_k == nullptr || n_q_heads < 1 || n_kv_heads < 1) return 0;
-  return attn_layout(B, cu_q, cu_k, n_q_heads, n_kv_heads).total;
+  return attn_layout(cross_segs(B, cu_q, cu_k), n_q_heads, n_kv_heads).total;
 }
 
 extern "C" pace_status_t pace_llm_text_visual_importance(const void* Q, const void* K, const int32_t* cu_q,
@@ -959,4 +1068,26 @@ extern "C" pace_status_t pace_llm_text_visual_importance(const void* Q, const vo
                                                          pace_stream_t stream) {
   return importance(Q, K, cu_q, cu_k, B, n_q_heads, n_kv_heads, head_dim, scale, 1, s_llm_raw, ws, ws_bytes,
                     stream);
+}
+
+extern "C" size_t pace_llm_sequence_importance_workspace_size(int B, const int32_t* cu_seq, const int32_t* vis_start,
+                                                              const int32_t* n_vis, int n_q_heads, int n_kv_heads,
+                                                              int query_set) {
+  if (B <= 0 || n_q_heads < 1 || n_kv_heads < 1) return 0;
+  if (check_sequences(B, cu_seq, vis_start, n_vis, query_set) != PACE_OK) return 0;
+  return attn_layout(sequence_segs(B, cu_seq, vis_start, n_vis, query_set), n_q_heads, n_kv_heads).total;
+}
+
+extern "C" pace_status_t pace_llm_sequence_importance(const void* Q, const void* K, const int32_t* cu_seq,
+                                                      const int32_t* vis_start, const int32_t* n_vis, int B,
+                                                      int n_q_heads, int n_kv_heads, int head_dim, float scale,
+                                                      int query_set, float* s_llm_raw, void* ws, size_t ws_bytes,
+                                                      pace_stream_t stream) {
+  if (B < 0) return PACE_ERR_INVALID_ARG;
+  if (B == 0) return PACE_OK;
+  if (s_llm_raw == nullptr) return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(check_heads(n_q_heads, n_kv_heads, head_dim, scale, Q, K));
+  PACE_CHECK(check_sequences(B, cu_seq, vis_start, n_vis, query_set));
+  return dispatch<true>(Q, K, cu_seq[B], cu_seq[B], sequence_segs(B, cu_seq, vis_start, n_vis, query_set), n_q_heads,
+                  n_kv_heads, head_dim, scale, 1, s_llm_raw, ws, ws_bytes, stream);
 }

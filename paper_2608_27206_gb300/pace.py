@@ -41,6 +41,8 @@ class DdaeParams(ctypes.Structure):
 
 # fusion modes of DdaeParams (pace_ddae_fusion)
 DDAE_ADAPTIVE, DDAE_ONLY_LLM, DDAE_ONLY_VIT, DDAE_FIXED = 0, 1, 2, 3
+QUERY_VISION_TEXT, QUERY_TEXT, QUERY_LAST = 0, 1, 2
+QUERY_SETS = {"vision_text": QUERY_VISION_TEXT, "text": QUERY_TEXT, "last": QUERY_LAST}
 
 
 class GatherTensor(ctypes.Structure):
@@ -85,6 +87,11 @@ _SIGS = {
     "pace_llm_text_visual_importance": (ctypes.c_int, [_P, _P, _I32P, _I32P, ctypes.c_int, ctypes.c_int,
                                                        ctypes.c_int, ctypes.c_int, ctypes.c_float, _P, _P,
                                                        ctypes.c_size_t, _P]),
+    "pace_llm_sequence_importance_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, _I32P, _I32P,
+                                                                      ctypes.c_int, ctypes.c_int, ctypes.c_int]),
+    "pace_llm_sequence_importance": (ctypes.c_int, [_P, _P, _I32P, _I32P, _I32P, ctypes.c_int, ctypes.c_int,
+                                                    ctypes.c_int, ctypes.c_int, ctypes.c_float, ctypes.c_int, _P,
+                                                    _P, ctypes.c_size_t, _P]),
     "pace_ddae_params_default": (None, [ctypes.POINTER(DdaeParams)]),
     "pace_budget": (ctypes.c_int32, [ctypes.c_int32, ctypes.c_double]),
     "pace_ddae_select": (ctypes.c_int, [_P, _P, _I32P, _I32P, ctypes.c_int, ctypes.POINTER(DdaeParams), _P, _P,
@@ -403,6 +410,42 @@ def pace_llm_text_visual_importance(Q: torch.Tensor, K: torch.Tensor, cu_q, cu_k
                                                _dev(out), _dev(ws), ws.numel() * ws.element_size(), _stream(stream))
     _check("pace_llm_text_visual_importance", st)
     return out[: int(k[-1])]
+
+
+def _query_set(query_set) -> int:
+    return QUERY_SETS[query_set] if isinstance(query_set, str) else int(query_set)
+
+
+def pace_llm_sequence_importance_workspace_size(cu_seq, vis_start, n_vis, n_q_heads: int, n_kv_heads: int,
+                                                query_set="vision_text") -> int:
+    c, v, n = _i32(cu_seq), _i32(vis_start), _i32(n_vis)
+    return int(lib().pace_llm_sequence_importance_workspace_size(len(c) - 1, _pi32(c), _pi32(v), _pi32(n),
+                                                                 int(n_q_heads), int(n_kv_heads),
+                                                                 _query_set(query_set)))
+
+
+def pace_llm_sequence_importance(Q: torch.Tensor, K: torch.Tensor, cu_seq, vis_start, n_vis,
+                                 query_set="vision_text", scale: Optional[float] = None,
+                                 out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                                 stream=None) -> torch.Tensor:
+    """Full-sequence S_llm_raw [sum n_vis] from bf16 Q [sum S, Hq, D] and K [sum S, Hkv, D] of causal
+    sequences; query_set is "vision_text", "text" or "last" (or a QUERY_* code)."""
+    c, v, n = _i32(cu_seq), _i32(vis_start), _i32(n_vis)
+    B = len(c) - 1
+    _, Hq, D = Q.shape
+    Hkv = K.shape[1]
+    qs = _query_set(query_set)
+    if scale is None:
+        scale = float(D) ** -0.5
+    total = int(n.sum()) if B > 0 else 0
+    if out is None:
+        out = torch.empty(max(total, 1), dtype=torch.float32, device=Q.device)
+    ws = _workspace(pace_llm_sequence_importance_workspace_size(c, v, n, Hq, Hkv, qs), ws, Q.device)
+    st = lib().pace_llm_sequence_importance(_dev(Q), _dev(K), _pi32(c), _pi32(v), _pi32(n), B, Hq, Hkv, D,
+                                            float(scale), qs, _dev(out), _dev(ws), ws.numel() * ws.element_size(),
+                                            _stream(stream))
+    _check("pace_llm_sequence_importance", st)
+    return out[:total]
 
 
 def pace_ddae_select(s_llm_raw: torch.Tensor, s_vis_raw: torch.Tensor, cu_v, cu_keep,

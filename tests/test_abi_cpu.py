@@ -85,6 +85,12 @@ def test_workspace_queries(libpace):
     l = libpace.pace_llm_text_visual_importance_workspace_size([0, 64], [0, 256], 28, 4)
     assert l >= 28 * 128 * 4 + 4 * 256 * 4
     assert libpace.pace_vit_attn_importance_workspace_size([0], 16) == 0
+    # full-sequence S_llm: L rows cover the query set (padded to 256 rows), the part map the visual tokens
+    for qs, nq in (("vision_text", 1000 - 14), ("text", 1000 - 14 - 576), ("last", 1)):
+        s = libpace.pace_llm_sequence_importance_workspace_size([0, 1000], [14], [576], 28, 4, qs)
+        assert s >= 28 * ((nq + 255) // 256 * 256) * 32 + 4 * 576 * 4, qs
+    assert libpace.pace_llm_sequence_importance_workspace_size([0, 10], [8], [4], 28, 4, "text") == 0   # past the end
+    assert libpace.pace_llm_sequence_importance_workspace_size([0, 10], [0], [4], 28, 4, 3) == 0        # bad query set
 
 
 def test_budget_vanilla_matches_oracle(libpace):

@@ -365,6 +365,57 @@ def test_llm_importance_gqa_shapes(pace):
         assert_scores_close(out, ref, what=f"S_llm_raw Hq={Hq} Hkv={Hkv}")
 
 
+def _seq_case(pace, S, vis, nvis, query_set, Hq=28, Hkv=4, D=128, seed=0):
+    cu = np.concatenate([[0], np.cumsum(S)]).astype(np.int32)
+    Qb = synth.random_small_qk(seed, int(cu[-1]), Hq, D)
+    Kb = synth.random_small_qk(seed + 1, int(cu[-1]), Hkv, D)
+    scale = 1.0 / math.sqrt(D)
+    out = pace.pace_llm_sequence_importance(bf16_tensor(Qb), bf16_tensor(Kb), cu, vis, nvis, query_set,
+                                            scale).cpu().numpy()
+    ref = O.llm_sequence_importance(f64(Qb), f64(Kb), cu, vis, nvis, scale, query_set)
+    return out, ref
+
+
+@pytest.mark.parametrize("query_set", ["vision_text", "text", "last"])
+@pytest.mark.parametrize("S,vis,nvis", [([700], [30], [400]), ([1300], [3], [1024]), ([9], [2], [4])])
+def test_llm_sequence_importance(pace, S, vis, nvis, query_set):
+    out, ref = _seq_case(pace, S, vis, nvis, query_set)
+    assert_scores_close(out, ref, what=f"full-sequence S_llm_raw ({query_set})")
+    _no_device_error(pace)
+
+
+@pytest.mark.parametrize("query_set", ["vision_text", "text", "last"])
+def test_llm_sequence_importance_ragged_gqa(pace, query_set):
+    # the first sequence ends with its visual span, so its text query set is empty
+    S, vis, nvis = [300, 1100, 77, 520], [0, 14, 5, 200], [300, 900, 60, 1]
+    for Hq, Hkv, D in ((8, 2, 80), (12, 12, 64)):
+        out, ref = _seq_case(pace, S, vis, nvis, query_set, Hq=Hq, Hkv=Hkv, D=D, seed=Hq)
+        assert_scores_close(out, ref, what=f"full-sequence S_llm_raw ({query_set}, Hq={Hq}, Hkv={Hkv})")
+        if query_set == "text":
+            assert np.all(out[:300] == 0.0)
+    _no_device_error(pace)
+
+
+def test_llm_sequence_importance_all_visual_mass(pace):
+    # an all-visual sequence: every query row's causal softmax lies on visual keys
+    out, _ = _seq_case(pace, [640, 257], [0, 0], [640, 257], "vision_text", Hq=4, Hkv=1, D=64, seed=5)
+    assert out[:640].sum() == pytest.approx(640 * 4, rel=1e-4)
+    assert out[640:].sum() == pytest.approx(257 * 4, rel=1e-4)
+    # key 0 is seen by every row; the last key only by the last row (weight of its own softmax)
+    assert out[639] < out[0]
+
+
+def test_llm_sequence_importance_rejects(pace):
+    Q = torch.zeros((16, 2, 64), dtype=torch.bfloat16, device="cuda")
+    for cu, vis, nvis, qs in (([0, 16], [10], [7], "vision_text"),     # visual span past the end
+                              ([0, 16], [-1], [4], "text"),            # negative start
+                              ([0, 16], [0], [0], "last"),             # no visual tokens
+                              ([0, 16], [0], [4], 7)):                  # unknown query set
+        with pytest.raises(pace.PaceError):
+            pace.pace_llm_sequence_importance(Q, Q, cu, vis, nvis, qs)
+    _no_device_error(pace)
+
+
 def test_importance_rejects_bad_args(pace):
     Q = torch.zeros((8, 2, 80), dtype=torch.bfloat16, device="cuda")
     with pytest.raises(pace.PaceError):

@@ -366,3 +366,35 @@ def test_prune_rows_against_position_loop():
         expect = [p for p in range(pre + n_vis + post) if not (pre <= p < pre + n_vis) or (p - pre) in ks]
         np.testing.assert_array_equal(rows, expect)
         assert len(rows) == pre + post + len(kept)       # S_post = T + N_keep
+
+
+def test_llm_sequence_importance_brute_force_and_mass():
+    """Full-sequence S_llm: a materialised causal softmax written as plain loops (tiny sizes),
+    and the attention mass: each query's softmax sums to 1 over its keys, so the visual mass is
+    at most |P| * Hq, with equality when the visual span is the whole prefix of every query."""
+    rng = np.random.default_rng(8)
+    S, v, nv, Hq, Hkv, d = 23, 5, 9, 4, 2, 6
+    Q = rng.normal(size=(S, Hq, d))
+    K = rng.normal(size=(S, Hkv, d))
+    scale = 0.4
+    for qs in O.QUERY_SETS:
+        got = O.llm_sequence_importance(Q, K, [0, S], [v], [nv], scale, qs)
+        q_lo = {"vision_text": v, "text": v + nv, "last": S - 1}[qs]
+        want = np.zeros(nv)
+        for h in range(Hq):
+            for q in range(q_lo, S):
+                w = [math.exp(scale * float(Q[q, h] @ K[k, h // 2])) for k in range(q + 1)]
+                z = sum(w)
+                for j in range(nv):
+                    if v + j <= q:
+                        want[j] += w[v + j] / z
+        np.testing.assert_allclose(got, want, rtol=1e-12, atol=1e-15)
+        assert got.sum() <= (S - q_lo) * Hq + 1e-9
+    # image at the start of the sequence, text queries only, keys = visual + earlier text:
+    # with text keys scored -inf-like (huge negative), all mass goes to the visual keys
+    K2 = K.copy()
+    K2[nv:] = 0.0
+    Q2 = Q.copy()
+    got = O.llm_sequence_importance(Q2 * 0 + 1.0, K2 * 0 + np.r_[np.ones(nv), np.zeros(S - nv)][:, None, None],
+                                    [0, S], [0], [nv], 50.0, "text")
+    assert got.sum() == pytest.approx((S - nv) * Hq, rel=1e-9)
