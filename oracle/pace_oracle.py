@@ -35,6 +35,11 @@ Readings taken where the paper is silent or cannot be followed literally
   R10 preview tokens given by the caller (apc_density_preview): a token of zero
       norm counts as t_hat = 0 (cosine 0 with every token, Eq. 1 undefined
       otherwise); if every token is zero, c_hat = 0.
+  R11 full-sequence S_llm (llm_sequence_importance): the query set starts at
+      the first visual position (Vision + Text; earlier positions cannot see
+      the visual span under the causal mask), after the visual span (Text) or
+      at the last position (Last); each query's softmax runs over every
+      position up to and including itself.
 """
 from __future__ import annotations
 
