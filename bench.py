@@ -363,14 +363,10 @@ def run_gpu(args):
     h2d = sum(v.numel() * v.element_size() for v in pinned.values())
     d2h = sum(v.numel() * v.element_size() for v in out_host.values())
 
+    copy_stream = torch.cuda.Stream(device)
+
     def e2e_step():
-        for kname, v in pinned.items():
-            pipe.d[kname].copy_(v, non_blocking=True)
-        pipe.step()
-        out_host["kept"].copy_(pipe.kept, non_blocking=True)
-        out_host["rows"].copy_(pipe.rows, non_blocking=True)
-        out_host["stats"].copy_(pipe.stats, non_blocking=True)
-        out_host["s_final"].copy_(pipe.s_final, non_blocking=True)
+        pipe.step_from_host(pinned, out_host, copy_stream)
 
     for _ in range(max(1, args.warmup)):
         e2e_step()

@@ -97,6 +97,37 @@ class HotPath:
         for _, f in self.parts:
             f()
 
+    # -- one step from host memory ---------------------------------------------------------------
+    # Input tensors in the order the calls need them; each group is copied on a side stream and
+    # the compute stream waits only for the group its next call reads.
+    COPY_GROUPS = (("img",), ("vit_q", "vit_k"), ("llm_q", "llm_k"), ("embed",))
+    CALL_NEEDS = {"density": 0, "vit": 1, "llm": 2, "gather": 3}
+
+    def step_from_host(self, pinned: dict, out_host: dict, copy_stream: Optional[torch.cuda.Stream] = None):
+        """Copies this step's inputs from pinned host tensors (keys as in `self.host`), runs the six
+        calls, and copies the results named in `out_host` back to (pinned) host tensors.
+
+        The host-to-device copies run on `copy_stream` in call order, so the ViT Q/K copy overlaps
+        density and resampling; each call waits only for the inputs it reads.  The next step's copies
+        wait for this step's calls to finish (the device input buffers are reused)."""
+        main = torch.cuda.current_stream(self.dev)
+        cs = copy_stream if copy_stream is not None else torch.cuda.Stream(self.dev)
+        cs.wait_stream(main)        # the previous step's calls have read their inputs
+        ready = []
+        with torch.cuda.stream(cs):
+            for group in self.COPY_GROUPS:
+                for k in group:
+                    self.d[k].copy_(pinned[k], non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(cs)
+                ready.append(ev)
+        for name, f in self.parts:
+            if name in self.CALL_NEEDS:
+                main.wait_event(ready[self.CALL_NEEDS[name]])
+            f()
+        for k, v in out_host.items():      # attribute name -> host tensor of the same shape
+            v.copy_(getattr(self, k), non_blocking=True)
+
     # -- results on the host ---------------------------------------------------------------------
     def resized_images(self):
         st = P.stats_dict(self.stats[: self.B])
