@@ -61,6 +61,7 @@ constexpr int kEpiWarps = 16;
 constexpr int kThreads = 64 + 32 * kEpiWarps;   // 576
 constexpr int kAttnMaxB = 64;
 constexpr uint32_t kTmemCols = 512;
+constexpr float kShiftMargin = 90.f;      // pass 1: fixed shift = first chunk maximum + this (base 2)
 constexpr int kNoMask = 1 << 29;          // diag of a non-causal image: every key is seen
 constexpr int kTargetItems = 152;         // work items (two CTAs each): two waves over the SMs
 
@@ -251,10 +252,12 @@ __device__ __forceinline__ void lse_update64(const uint32_t (&v)[64], int valid,
 }
 
 // Fixed-shift row update with 64 new scores: the shift m is the base-2 maximum of the row's
-// first chunk and then never moves, so there is no maximum in the common path.  Every term
-// 2^(c s - m) is computed to full relative precision whatever its size, and the largest term
-// of the row is >= 1, so nothing underflows; the only failure is overflow (a score more than
-// about 127 - log2(N) above m), which leaves l = inf or NaN and is caught by the caller.
+// first chunk plus a margin of kShiftMargin, and then never moves, so there is no maximum in the
+// common path.  Every term 2^(c s - m) above 2^-126 is computed to full relative precision, and
+// the largest term of the row is >= 2^-kShiftMargin, so the terms flushed to zero weigh at most
+// N 2^(kShiftMargin - 126) of the sum (2^-16 for N = 2^20).  The only failure is overflow (a
+// score more than about 127 + kShiftMargin - log2(N) above the first chunk's maximum), which
+// leaves l = inf or NaN and is caught by the caller.
 template <bool FIRST>
 __device__ __forceinline__ void lse_fixed64(const uint32_t (&v)[64], int valid, float c, float& m_run,
                                             float& l_run) {
@@ -275,7 +278,7 @@ __device__ __forceinline__ void lse_fixed64(const uint32_t (&v)[64], int valid, 
       mx2 = max3(mx2, s[e + 4], s[e + 5]);
       mx3 = max3(mx3, s[e + 6], s[e + 7]);
     }
-    m_run = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * c;
+    m_run = fmaf(fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)), c, kShiftMargin);
   }
   const float2 cc = make_float2(c, c);
   const float2 nm = make_float2(-m_run, -m_run);

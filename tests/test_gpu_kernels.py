@@ -299,8 +299,8 @@ def _spiked_qk(n, H, D, seed, spikes):
 
 def test_vit_importance_wide_score_range(pace):
     """Rows whose maximum lies 88 and 244 (base 2) above the scores of their first keys: the
-    first stays finite in a fixed-shift sum, the second overflows exp2 and must be redone
-    with an exact running maximum."""
+    first stays finite in the fixed-shift sum (shift = first maximum + 90), the second overflows
+    it and the CTA streams its keys again with an exact running maximum."""
     n, H, D = 1024, 2, 80
     Qb, Kb = _spiked_qk(n, H, D, seed=5, spikes=[(700, np.arange(0, 200), 25.0),
                                                  (900, np.arange(300, 340), 40.0)])
@@ -313,10 +313,31 @@ def test_vit_importance_wide_score_range(pace):
     _no_device_error(pace)
 
 
+def test_vit_importance_high_run_below_margin(pace):
+    """Rows whose 7936 last keys all score about 91 (base 2) above their first keys: the warps
+    that start on the low keys hold the high terms just below the fixed shift's margin (no
+    overflow, no redo) while the first keys' terms sit near 2^-90."""
+    n, H, D, a = 8192, 1, 80, 24.6
+    rng = np.random.default_rng(11)
+    Q = f64(synth.random_small_qk(11, n, H, D))
+    K = f64(synth.random_small_qk(1011, n, H, D))
+    u = rng.standard_normal((H, D))
+    u /= np.linalg.norm(u, axis=1, keepdims=True)
+    K[256:] = a * u
+    Q[:64] = a * u + 0.05 * rng.standard_normal((64, H, D))
+    Qb, Kb = synth.f32_to_bf16_bits(Q.astype(np.float32)), synth.f32_to_bf16_bits(K.astype(np.float32))
+    cu = np.array([0, n], np.int32)
+    scale = 1.0 / math.sqrt(D)
+    out = pace.pace_vit_attn_importance(bf16_tensor(Qb), bf16_tensor(Kb), cu, scale, 1).cpu().numpy()
+    ref = O.vit_attn_importance(f64(Qb), f64(Kb), cu, scale, 1)
+    assert_scores_close(out, ref, what="S_vis_raw with a long run of high scores")
+    _no_device_error(pace)
+
+
 def test_llm_importance_wide_score_range(pace):
-    """A spike 200 (base 2) above the other scores through the GQA path with key splits (few
-    query tiles, many key tiles): exp2 overflows in the first round of every split that holds
-    the spike key."""
+    """A spike about 245 (base 2) above the other scores through the GQA path with key splits
+    (few query tiles, many key tiles): the fixed-shift sum overflows in every split that holds
+    the spike key, which redoes its keys with an exact running maximum."""
     nq, nk, Hq, Hkv, D = 64, 2304, 4, 2, 128
     Qs, _ = _spiked_qk(nq, Hq, D, seed=6, spikes=[])
     rng = np.random.default_rng(6)
@@ -325,9 +346,9 @@ def test_llm_importance_wide_score_range(pace):
     for g in range(Hkv):
         u = rng.standard_normal(D)
         u /= np.linalg.norm(u)
-        K[2000, g] = 40.0 * u
+        K[2000, g] = 44.0 * u
         for h in range(g * (Hq // Hkv), (g + 1) * (Hq // Hkv)):
-            Q[:32, h] = 40.0 * u
+            Q[:32, h] = 44.0 * u
     Qb, Kb = synth.f32_to_bf16_bits(Q.astype(np.float32)), synth.f32_to_bf16_bits(K.astype(np.float32))
     cq, ck = np.array([0, nq], np.int32), np.array([0, nk], np.int32)
     scale = 1.0 / math.sqrt(D)
