@@ -35,7 +35,26 @@ constexpr int kStrip = 32;                           // patches per strip
 constexpr int kStripRowBytes = kStrip * kPatch * 3;  // 1344 bytes of one image row per strip
 constexpr int kApcThreads = 256;
 constexpr int kApcMaxB = 64;
-constexpr double kFix = 4294967296.0;                // 2^32 fixed-point scale
+// Column sums are 2^-32 fixed point in 64-bit integers.  The conversions below use only 32-bit
+// conversions and fp32 (no fp64, which is a slow pipe on this GPU); fix32 rounds exactly like
+// rounding v * 2^32 to the nearest integer (ties to even).
+__device__ __forceinline__ unsigned long long fix32(float v) {   // 0 <= v < 2^31
+  const float h = floorf(v);
+  return (static_cast<unsigned long long>(static_cast<uint32_t>(h)) << 32) +
+         __float2uint_rn((v - h) * 4294967296.0f);   // v - h is exact; the product is an exact scaling
+}
+__device__ __forceinline__ unsigned long long fix32_signed(float v) {   // |v| < 2^31, two's complement
+  return v >= 0.f ? fix32(v) : 0ull - fix32(-v);
+}
+// sum * 2^-32 * inv_n for a non-negative (or, with SIGNED, two's-complement) fixed-point sum.
+template <bool SIGNED>
+__device__ __forceinline__ float unfix32(unsigned long long sum, float inv_n) {
+  const bool neg = SIGNED && static_cast<long long>(sum) < 0;
+  const unsigned long long m = neg ? 0ull - sum : sum;
+  const float hi = static_cast<float>(static_cast<uint32_t>(m >> 32));   // < 2^24 for every use here
+  const float v = fmaf(static_cast<float>(static_cast<uint32_t>(m)), 0x1p-32f, hi) * inv_n;
+  return neg ? -v : v;
+}
 
 struct ApcTable {
   int64_t off[kApcMaxB];    // byte offset of image b
@@ -159,13 +178,12 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restri
         a0 = fmaf(inv[p], byte_to_float(v & 255u), a0);
         a1 = fmaf(inv[p], byte_to_float(v >> 8), a1);
       }
-      atomicAdd(sb + k, static_cast<unsigned long long>(llrint(static_cast<double>(a0 * (1.0f / 255.0f)) * kFix)));
-      atomicAdd(sb + k + 1,
-                static_cast<unsigned long long>(llrint(static_cast<double>(a1 * (1.0f / 255.0f)) * kFix)));
+      atomicAdd(sb + k, fix32(a0 * (1.0f / 255.0f)));
+      atomicAdd(sb + k + 1, fix32(a1 * (1.0f / 255.0f)));
     } else {
       float a = 0.f;
       for (int p = 0; p < np; ++p) a += inv[p];
-      atomicAdd(sb + kPatchBytes, static_cast<unsigned long long>(llrint(static_cast<double>(a) * kFix)));
+      atomicAdd(sb + kPatchBytes, fix32(a));
     }
   }
 }
@@ -187,13 +205,14 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
   const int px0 = cx * kStrip;
   const int np = min(kStrip, t.gw[b] - px0);
   const int N = (t.H[b] / kPatch) * t.gw[b];
+  const float inv_n = 1.0f / static_cast<float>(N);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   // c = sums / N, |c|^2 (fixed summation order)
   const unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * kTokDim;
   float part = 0.f;
   for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) {
-    const float c = static_cast<float>(static_cast<double>(sb[k]) * (1.0 / kFix) / N);
+    const float c = unfix32<false>(sb[k], inv_n);
     chat[k] = c;
     part = fmaf(c, c, part);
   }
@@ -303,8 +322,8 @@ __global__ void __launch_bounds__(kApcThreads) apc_tok_pass1(const uint32_t* __r
       a0 = fmaf(inv[p], bf16_lo(v), a0);
       a1 = fmaf(inv[p], bf16_hi(v), a1);
     }
-    atomicAdd(sb + 2 * w, static_cast<unsigned long long>(__float2ll_rn(a0 * 4294967296.0f)));
-    atomicAdd(sb + 2 * w + 1, static_cast<unsigned long long>(__float2ll_rn(a1 * 4294967296.0f)));
+    atomicAdd(sb + 2 * w, fix32_signed(a0));
+    atomicAdd(sb + 2 * w + 1, fix32_signed(a1));
   }
 }
 
@@ -323,11 +342,12 @@ __global__ void __launch_bounds__(kApcThreads) apc_tok_pass2(const uint32_t* __r
   const int c0 = (unit - t.unit_prefix[b]) * kTokChunk;
   const int nt = min(kTokChunk, t.n[b] - c0);
   const int N = t.n[b], D = t.D, words = D >> 1;
+  const float inv_n = 1.0f / static_cast<float>(N);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * D;
   float part = 0.f;
   for (int k = threadIdx.x; k < D; k += kApcThreads) {
-    const float cv = static_cast<float>(static_cast<double>(static_cast<long long>(sb[k])) * (1.0 / kFix) / N);
+    const float cv = unfix32<true>(sb[k], inv_n);
     chat[k] = cv;
     part = fmaf(cv, cv, part);
   }
@@ -370,10 +390,15 @@ struct TailParams {
 };
 
 constexpr int kTailSmemMax = 48 * 1024;   // d values staged in shared memory (floats)
+constexpr int kTailBins = 4096;            // level-1 buckets of the tail select
+
+// Bucket of a distance d >= 0: floor(2048 d), capped at the top bucket (monotone in d).
+__device__ __forceinline__ int tail_bucket(float v) { return min(static_cast<int>(v * 2048.0f), kTailBins - 1); }
 
 __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTable t, const float* __restrict__ d,
                                                  TailParams prm, pace_apc_stats* __restrict__ stats) {
   extern __shared__ float sd[];
+  __shared__ unsigned bins[kTailBins];
   __shared__ unsigned hist[256];
   __shared__ unsigned sel[2];
   __shared__ float red[32];
@@ -387,19 +412,67 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
     db = sd;
   }
   const unsigned k = static_cast<unsigned>(t.ktail[b]);
-  unsigned prefix = 0u, mask = 0u, remaining = k;
-  const int lane_id = threadIdx.x & 31;
+  const int lane_id = threadIdx.x & 31, warp_id = threadIdx.x >> 5;
+  // Level 1: the k-th largest distance's bucket among 4096 buckets of width 1/2048 (d <= 2 for
+  // unit vectors; the top bucket also takes anything above).  Value-domain buckets spread the
+  // shared-memory atomics, which the float's top bits (a few exponents) would not.
+  for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
+  __syncthreads();
+  for (int i = threadIdx.x; i < N; i += blockDim.x) atomicAdd(&bins[tail_bucket(db[i])], 1u);
+  __syncthreads();
+  // counts from the top: thread j owns buckets 4095 - 4j .. 4092 - 4j
+  unsigned c4[4], s4 = 0u;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    c4[q] = bins[kTailBins - 1 - 4 * static_cast<int>(threadIdx.x) - q];
+    s4 += c4[q];
+  }
+  unsigned incl = s4;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane_id >= o) incl += n;
+  }
+  if (lane_id == 31) cred[warp_id] = incl;
+  __syncthreads();
+  if (warp_id == 0) {
+    unsigned w = cred[lane_id];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned n = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane_id >= o) w += n;
+    }
+    cred[lane_id] = w;   // inclusive totals of warps 0 .. lane
+  }
+  __syncthreads();
+  incl += warp_id > 0 ? cred[warp_id - 1] : 0u;   // inclusive count down to this thread's last bucket
+  const unsigned excl = incl - s4;
+  if (excl < k && incl >= k) {                     // exactly one thread holds the k-th largest
+    unsigned above = excl;
+    int q = 0;
+#pragma unroll
+    for (int qq = 0; qq < 3; ++qq)
+      if (q == qq && above + c4[qq] < k) {
+        above += c4[qq];
+        q = qq + 1;
+      }
+    sel[0] = static_cast<unsigned>(kTailBins - 1 - 4 * static_cast<int>(threadIdx.x) - q);
+    sel[1] = above;
+  }
+  __syncthreads();
+  const int tb = static_cast<int>(sel[0]);
+  // Level 2: radix select (8-bit digits of the float bits) among the bucket's members only
+  const unsigned lo_key = __float_as_uint(static_cast<float>(tb) * (1.0f / 2048.0f));
+  const unsigned hi_key = tb == kTailBins - 1 ? 0xFFFFFFFFu : __float_as_uint(static_cast<float>(tb + 1) * (1.0f / 2048.0f));
+  unsigned prefix = 0u, mask = 0u, remaining = k - sel[1];
+  __syncthreads();
   for (int shift = 24; shift >= 0; shift -= 8) {
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0u;
     __syncthreads();
-    // lanes holding the same digit are combined before the shared atomic
-    for (int base = 0; base < N; base += blockDim.x) {
-      const int i = base + threadIdx.x;
-      const unsigned key = i < N ? __float_as_uint(db[i]) : 0u;
-      const bool in = i < N && (key & mask) == prefix;
-      const unsigned digit = in ? ((key >> shift) & 255u) : 256u;
-      const unsigned peers = __match_any_sync(0xffffffffu, digit);
-      if (in && lane_id == __ffs(peers) - 1) atomicAdd(&hist[digit], static_cast<unsigned>(__popc(peers)));
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+      const unsigned key = __float_as_uint(db[i]);
+      if (key >= lo_key && (key < hi_key || tb == kTailBins - 1) && (key & mask) == prefix)
+        atomicAdd(&hist[(key >> shift) & 255u], 1u);
     }
     __syncthreads();
     if (threadIdx.x < 32) warp_digit_search(hist, remaining, sel);
