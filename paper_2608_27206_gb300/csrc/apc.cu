@@ -23,6 +23,7 @@
 #include <mutex>
 
 #include "pace_common.cuh"
+#include "pace_ptx.cuh"
 #include "pace_select.cuh"
 
 namespace pace {
@@ -34,6 +35,7 @@ constexpr int kTokDim = kPatchBytes + 1;             // 589: pixels + constant c
 constexpr int kStrip = 32;                           // patches per strip
 constexpr int kStripRowBytes = kStrip * kPatch * 3;  // 1344 bytes of one image row per strip
 constexpr int kApcThreads = 256;
+constexpr int kPairIters = (kPatchBytes / 2 + 31) / 32;   // 10: coordinate pairs per lane
 constexpr int kApcMaxB = 64;
 // Column sums are 2^-32 fixed point in 64-bit integers.  The conversions below use only 32-bit
 // conversions and fp32 (no fp64, which is a slow pipe on this GPU); fix32 rounds exactly like
@@ -76,7 +78,20 @@ __device__ __forceinline__ int find_image(const ApcTable& t, int unit) {
   return b;
 }
 
-// Stages the 14 rows x (np * 42) bytes of one strip into s (row pitch kStripRowBytes).
+// Asynchronous 4-byte global -> shared copies (no register round trip, all in flight at once).
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+               "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Stages the 14 rows x (np * 42) bytes of one strip into s (row pitch kStripRowBytes).  WIDE:
+// asynchronous copies that the caller commits and waits for; otherwise plain loads and stores.
+// Either way the caller synchronises the block before reading s.
 template <bool WIDE>
 __device__ __forceinline__ void load_strip(const uint8_t* __restrict__ img, int W, int py, int px0, int np,
                                            uint8_t* s) {
@@ -87,8 +102,7 @@ __device__ __forceinline__ void load_strip(const uint8_t* __restrict__ img, int 
     const int words = seg >> 2;
     for (int i = threadIdx.x; i < kPatch * words; i += kApcThreads) {
       const int y = i / words, w = i - y * words;
-      const uint32_t v = __ldg(reinterpret_cast<const uint32_t*>(base + y * pitch) + w);
-      *reinterpret_cast<uint32_t*>(s + y * kStripRowBytes + 4 * w) = v;
+      cp_async4(s + y * kStripRowBytes + 4 * w, reinterpret_cast<const uint32_t*>(base + y * pitch) + w);
     }
   } else {
     const int halves = seg >> 1;
@@ -109,6 +123,21 @@ __device__ __forceinline__ float warp_sum_f(float v) {
 // Exact uint8 -> float without the conversion pipe: 2^23 + v has v in its low mantissa bits.
 __device__ __forceinline__ float byte_to_float(uint32_t v) { return __uint_as_float(0x4B000000u | v) - 8388608.0f; }
 
+// The two bytes of a 16-bit pair as floats: byte permutes build 2^23 + b in each word, one packed
+// subtract removes the 2^23.
+__device__ __forceinline__ float2 bytes2_to_float2(uint32_t v) {
+  const float2 w = make_float2(__uint_as_float(__byte_perm(v, 0x4B000000u, 0x7540)),
+                               __uint_as_float(__byte_perm(v, 0x4B000000u, 0x7541)));
+  return ptx::fadd2(w, make_float2(-8388608.0f, -8388608.0f));
+}
+
+// Shared-memory offset of token coordinates 2j, 2j + 1 of patch 0 in a staged strip (row y of the
+// patch, byte kk within its 42-byte row).
+__device__ __forceinline__ int pair_offset(int j) {
+  const int k = 2 * j, y = k / 42;
+  return y * kStripRowBytes + (k - y * 42);
+}
+
 // Sum of squares of the 42 bytes at s (2-byte aligned): 4-byte words with dp4a, the unaligned
 // ends as 16-bit loads.
 __device__ __forceinline__ uint32_t row_sumsq42(const uint8_t* s) {
@@ -128,131 +157,203 @@ __device__ __forceinline__ uint32_t row_sumsq42(const uint8_t* s) {
   return acc;
 }
 
+struct Strip {
+  int b, u, py, px0, np;
+};
+
+__device__ __forceinline__ Strip strip_of(const ApcTable& t, int unit) {
+  Strip q;
+  q.b = find_image(t, unit);
+  q.u = unit - t.unit_prefix[q.b];
+  q.py = q.u / t.chunks[q.b];
+  q.px0 = (q.u - q.py * t.chunks[q.b]) * kStrip;
+  q.np = min(kStrip, t.gw[q.b] - q.px0);
+  return q;
+}
+
+template <bool WIDE>
+__device__ __forceinline__ void issue_strip(const uint8_t* __restrict__ img, const ApcTable& t, int unit, uint8_t* s) {
+  const Strip q = strip_of(t, unit);
+  load_strip<WIDE>(img + t.off[q.b], t.W[q.b], q.py, q.px0, q.np, s);
+  cp_async_commit();
+}
+
+// Both passes run a grid of resident CTAs over the strips (unit = blockIdx.x, + gridDim.x, ...),
+// loading the next strip asynchronously while the current one is worked on.
 template <bool WIDE>
 __global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restrict__ img,
-                                                         const __grid_constant__ ApcTable t,
+                                                         const __grid_constant__ ApcTable t, int units,
                                                          float* __restrict__ inv_norm,
                                                          unsigned long long* __restrict__ sums) {
-  __shared__ __align__(16) uint8_t s[kPatch * kStripRowBytes];
+  __shared__ __align__(16) uint8_t s2[2][kPatch * kStripRowBytes];
   __shared__ uint32_t ssq[8][kStrip];
   __shared__ float inv[kStrip];
-  const int unit = blockIdx.x;
-  const int b = find_image(t, unit);
-  const int u = unit - t.unit_prefix[b];
-  const int py = u / t.chunks[b], cx = u - py * t.chunks[b];
-  const int px0 = cx * kStrip;
-  const int np = min(kStrip, t.gw[b] - px0);
-  load_strip<WIDE>(img + t.off[b], t.W[b], py, px0, np, s);
-  __syncthreads();
-  // |x|^2 of every patch: thread (p = tid % 32, rows yg and yg + 8)
-  {
-    const int p = threadIdx.x & 31, yg = threadIdx.x >> 5;
-    uint32_t a = 0u;
-    if (p < np) {
-      a = row_sumsq42(s + yg * kStripRowBytes + p * 42);
-      if (yg + 8 < kPatch) a += row_sumsq42(s + (yg + 8) * kStripRowBytes + p * 42);
-    }
-    ssq[yg][p] = a;
-  }
-  __syncthreads();
-  if (threadIdx.x < np) {
-    const int p = threadIdx.x;
-    uint32_t ss = 0u;
+  int unit = blockIdx.x;
+  if (unit >= units) return;
+  // weighted column sums: thread slot j (j = tid, tid + 256) owns columns 2j, 2j+1 (a pair never
+  // crosses a 42-byte row); slot 294 owns the constant coordinate.  Each strip's sums are rounded
+  // to 2^-32 fixed point and added exactly; one atomic per column when the image changes.
+  constexpr int kSlots = kPatchBytes / 2 + 1;   // 295
+  unsigned long long acc[2][2] = {{0ull, 0ull}, {0ull, 0ull}};
+  int cur_b = -1;
+  auto flush = [&]() {
+    if (cur_b < 0) return;
+    unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + cur_b) * kTokDim;
 #pragma unroll
-    for (int g = 0; g < 8; ++g) ss += ssq[g][p];
-    const float n2 = static_cast<float>(ss) * (1.0f / 65025.0f) + 1.0f;
-    const float iv = 1.0f / sqrtf(n2);
-    inv[p] = iv;
-    inv_norm[t.patch0[b] + py * t.gw[b] + px0 + p] = iv;
-  }
-  __syncthreads();
-  // weighted column sums: thread j owns columns 2j, 2j+1 (a pair never crosses a 42-byte row)
-  unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * kTokDim;
-  for (int j = threadIdx.x; j < kPatchBytes / 2 + 1; j += kApcThreads) {
-    if (j < kPatchBytes / 2) {
-      const int k = 2 * j, y = k / 42, kk = k - y * 42;
-      const uint16_t* col = reinterpret_cast<const uint16_t*>(s + y * kStripRowBytes + kk);
-      float a0 = 0.f, a1 = 0.f;
-      for (int p = 0; p < np; ++p) {
-        const uint32_t v = col[p * 21];
-        a0 = fmaf(inv[p], byte_to_float(v & 255u), a0);
-        a1 = fmaf(inv[p], byte_to_float(v >> 8), a1);
+    for (int q = 0; q < 2; ++q) {
+      const int j = threadIdx.x + q * kApcThreads;
+      if (j < kPatchBytes / 2) {
+        atomicAdd(sb + 2 * j, acc[q][0]);
+        atomicAdd(sb + 2 * j + 1, acc[q][1]);
+      } else if (j == kPatchBytes / 2) {
+        atomicAdd(sb + kPatchBytes, acc[q][0]);
       }
-      atomicAdd(sb + k, fix32(a0 * (1.0f / 255.0f)));
-      atomicAdd(sb + k + 1, fix32(a1 * (1.0f / 255.0f)));
-    } else {
-      float a = 0.f;
-      for (int p = 0; p < np; ++p) a += inv[p];
-      atomicAdd(sb + kPatchBytes, fix32(a));
+      acc[q][0] = acc[q][1] = 0ull;
     }
+  };
+  issue_strip<WIDE>(img, t, unit, s2[0]);
+  for (int i = 0; unit < units; ++i, unit += gridDim.x) {
+    const int next = unit + static_cast<int>(gridDim.x);
+    if (next < units) {
+      issue_strip<WIDE>(img, t, next, s2[(i + 1) & 1]);
+      cp_async_wait_group<1>();
+    } else {
+      cp_async_wait_group<0>();
+    }
+    __syncthreads();
+    const uint8_t* s = s2[i & 1];
+    const Strip q = strip_of(t, unit);
+    if (q.b != cur_b) {
+      flush();
+      cur_b = q.b;
+    }
+    // |x|^2 of every patch: thread (p = tid % 32, rows yg and yg + 8)
+    {
+      const int p = threadIdx.x & 31, yg = threadIdx.x >> 5;
+      uint32_t a = 0u;
+      if (p < q.np) {
+        a = row_sumsq42(s + yg * kStripRowBytes + p * 42);
+        if (yg + 8 < kPatch) a += row_sumsq42(s + (yg + 8) * kStripRowBytes + p * 42);
+      }
+      ssq[yg][p] = a;
+    }
+    __syncthreads();
+    if (threadIdx.x < q.np) {
+      const int p = threadIdx.x;
+      uint32_t ss = 0u;
+#pragma unroll
+      for (int g = 0; g < 8; ++g) ss += ssq[g][p];
+      const float n2 = static_cast<float>(ss) * (1.0f / 65025.0f) + 1.0f;
+      const float iv = 1.0f / sqrtf(n2);
+      inv[p] = iv;
+      inv_norm[t.patch0[q.b] + q.py * t.gw[q.b] + q.px0 + p] = iv;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int qs = 0; qs < 2; ++qs) {
+      const int j = threadIdx.x + qs * kApcThreads;
+      if (j < kPatchBytes / 2) {
+        const uint16_t* col = reinterpret_cast<const uint16_t*>(s + pair_offset(j));
+        float2 a = make_float2(0.f, 0.f);
+        for (int p = 0; p < q.np; ++p) {
+          const float iv = inv[p];
+          a = ptx::ffma2(make_float2(iv, iv), bytes2_to_float2(col[p * 21]), a);
+        }
+        acc[qs][0] += fix32(a.x * (1.0f / 255.0f));
+        acc[qs][1] += fix32(a.y * (1.0f / 255.0f));
+      } else if (j == kPatchBytes / 2) {
+        float a = 0.f;
+        for (int p = 0; p < q.np; ++p) a += inv[p];
+        acc[qs][0] += fix32(a);
+      }
+    }
+    __syncthreads();   // this buffer is refilled two strips on
   }
+  flush();
+  static_assert(kSlots <= 2 * kApcThreads, "column slots");
 }
 
 template <bool WIDE>
 __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restrict__ img,
-                                                         const __grid_constant__ ApcTable t,
+                                                         const __grid_constant__ ApcTable t, int units,
                                                          const float* __restrict__ inv_norm,
                                                          const unsigned long long* __restrict__ sums,
                                                          float* __restrict__ d_out,
                                                          pace_apc_stats* __restrict__ stats) {
-  __shared__ __align__(16) uint8_t s[kPatch * kStripRowBytes];
+  __shared__ __align__(16) uint8_t s2[2][kPatch * kStripRowBytes];
   __shared__ __align__(8) float chat[kTokDim + 3];
   __shared__ float red[kApcThreads / 32];
-  const int unit = blockIdx.x;
-  const int b = find_image(t, unit);
-  const int u = unit - t.unit_prefix[b];
-  const int py = u / t.chunks[b], cx = u - py * t.chunks[b];
-  const int px0 = cx * kStrip;
-  const int np = min(kStrip, t.gw[b] - px0);
-  const int N = (t.H[b] / kPatch) * t.gw[b];
-  const float inv_n = 1.0f / static_cast<float>(N);
+  int unit = blockIdx.x;
+  if (unit >= units) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  // c = sums / N, |c|^2 (fixed summation order)
-  const unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * kTokDim;
-  float part = 0.f;
-  for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) {
-    const float c = unfix32<false>(sb[k], inv_n);
-    chat[k] = c;
-    part = fmaf(c, c, part);
-  }
-  part = warp_sum_f(part);
-  if (lane == 0) red[warp] = part;
-  load_strip<WIDE>(img + t.off[b], t.W[b], py, px0, np, s);
-  __syncthreads();
-  float phi = 0.f;
+  int off[kPairIters];   // this lane's coordinate pairs j = lane + 32 it
 #pragma unroll
-  for (int w = 0; w < kApcThreads / 32; ++w) phi += red[w];
-  const float inv_c = 1.0f / sqrtf(phi);
-  for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) chat[k] *= inv_c;
-  if (u == 0 && threadIdx.x == 0) {
-    stats[t.b_base + b].phi = phi;
-    stats[t.b_base + b].rho_g = 1.0f - phi;
-    stats[t.b_base + b].n_patches = N;
-    stats[t.b_base + b].k_tail = t.ktail[b];
-  }
-  __syncthreads();
-  // d_i = |t_i - c_hat| computed directly: warp per patch, lanes over column pairs
-  const float* pinv = inv_norm + t.patch0[b] + py * t.gw[b] + px0;
-  const float2* chat2 = reinterpret_cast<const float2*>(chat);
-  for (int p = warp; p < np; p += kApcThreads / 32) {
-    const float iv = pinv[p];
-    const float sc = iv * (1.0f / 255.0f);
-    float acc0 = 0.f, acc1 = 0.f;
-    for (int j = lane; j < kPatchBytes / 2; j += 32) {
-      const int k = 2 * j, y = k / 42, kk = k - y * 42;
-      const uint32_t v = *reinterpret_cast<const uint16_t*>(s + y * kStripRowBytes + p * 42 + kk);
-      const float2 ch = chat2[j];
-      const float e0 = fmaf(byte_to_float(v & 255u), sc, -ch.x);
-      const float e1 = fmaf(byte_to_float(v >> 8), sc, -ch.y);
-      acc0 = fmaf(e0, e0, acc0);
-      acc1 = fmaf(e1, e1, acc1);
+  for (int it = 0; it < kPairIters; ++it) off[it] = pair_offset(min(lane + 32 * it, kPatchBytes / 2 - 1));
+  int cur_b = -1;
+  issue_strip<WIDE>(img, t, unit, s2[0]);
+  for (int i = 0; unit < units; ++i, unit += gridDim.x) {
+    const int next = unit + static_cast<int>(gridDim.x);
+    const Strip q = strip_of(t, unit);
+    if (q.b != cur_b) {   // c = sums / N, |c|^2 (fixed summation order), c_hat = c / |c|
+      cur_b = q.b;
+      const int N = (t.H[q.b] / kPatch) * t.gw[q.b];
+      const float inv_n = 1.0f / static_cast<float>(N);
+      const unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + q.b) * kTokDim;
+      float part = 0.f;
+      for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) {
+        const float c = unfix32<false>(sb[k], inv_n);
+        chat[k] = c;
+        part = fmaf(c, c, part);
+      }
+      part = warp_sum_f(part);
+      if (lane == 0) red[warp] = part;
+      __syncthreads();
+      float phi = 0.f;
+#pragma unroll
+      for (int w = 0; w < kApcThreads / 32; ++w) phi += red[w];
+      const float inv_c = 1.0f / sqrtf(phi);
+      __syncthreads();
+      for (int k = threadIdx.x; k < kTokDim; k += kApcThreads) chat[k] *= inv_c;
+      if (q.u == 0 && threadIdx.x == 0) {
+        stats[t.b_base + q.b].phi = phi;
+        stats[t.b_base + q.b].rho_g = 1.0f - phi;
+        stats[t.b_base + q.b].n_patches = N;
+        stats[t.b_base + q.b].k_tail = t.ktail[q.b];
+      }
     }
-    float acc = warp_sum_f(acc0 + acc1);
-    if (lane == 0) {
-      const float v = iv - chat[kPatchBytes];
-      d_out[t.patch0[b] + py * t.gw[b] + px0 + p] = sqrtf(fmaf(v, v, acc));
+    if (next < units) {
+      issue_strip<WIDE>(img, t, next, s2[(i + 1) & 1]);
+      cp_async_wait_group<1>();
+    } else {
+      cp_async_wait_group<0>();
     }
+    __syncthreads();
+    const uint8_t* s = s2[i & 1];
+    // d_i = |t_i - c_hat| computed directly: warp per patch, lanes over column pairs
+    const float* pinv = inv_norm + t.patch0[q.b] + q.py * t.gw[q.b] + q.px0;
+    const float2* chat2 = reinterpret_cast<const float2*>(chat);
+    for (int p = warp; p < q.np; p += kApcThreads / 32) {
+      const float sc = pinv[p] * (1.0f / 255.0f);
+      const float2 sc2 = make_float2(sc, sc);
+      float2 acc2 = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int it = 0; it < kPairIters; ++it) {   // lanes over the 294 coordinate pairs
+        const int j = lane + 32 * it;
+        if (it < kPairIters - 1 || j < kPatchBytes / 2) {
+          const uint32_t v = *reinterpret_cast<const uint16_t*>(s + off[it] + p * 42);
+          const float2 ch = chat2[j];
+          const float2 e = ptx::ffma2(bytes2_to_float2(v), sc2, make_float2(-ch.x, -ch.y));
+          acc2 = ptx::ffma2(e, e, acc2);
+        }
+      }
+      const float iv = pinv[p];
+      float acc = warp_sum_f(acc2.x + acc2.y);
+      if (lane == 0) {
+        const float v = iv - chat[kPatchBytes];
+        d_out[t.patch0[q.b] + q.py * t.gw[q.b] + q.px0 + p] = sqrtf(fmaf(v, v, acc));
+      }
+    }
+    __syncthreads();   // this buffer is refilled two strips on; chat may be rewritten
   }
 }
 
@@ -395,93 +496,114 @@ constexpr int kTailBins = 4096;            // level-1 buckets of the tail select
 // Bucket of a distance d >= 0: floor(2048 d), capped at the top bucket (monotone in d).
 __device__ __forceinline__ int tail_bucket(float v) { return min(static_cast<int>(v * 2048.0f), kTailBins - 1); }
 
-__global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTable t, const float* __restrict__ d,
-                                                 TailParams prm, pace_apc_stats* __restrict__ stats) {
-  extern __shared__ float sd[];
-  __shared__ unsigned bins[kTailBins];
-  __shared__ unsigned hist[256];
-  __shared__ unsigned sel[2];
-  __shared__ float red[32];
-  __shared__ unsigned cred[32];
-  const int b = blockIdx.x;
-  const int N = t.n[b];
-  const float* db = d + t.patch0[b];
-  if (N <= kTailSmemMax) {   // one coalesced read of the distances, then work from shared memory
-    for (int i = threadIdx.x; i < N; i += blockDim.x) sd[i] = db[i];
-    __syncthreads();
-    db = sd;
-  }
-  const unsigned k = static_cast<unsigned>(t.ktail[b]);
-  const int lane_id = threadIdx.x & 31, warp_id = threadIdx.x >> 5;
-  // Level 1: the k-th largest distance's bucket among 4096 buckets of width 1/2048 (d <= 2 for
-  // unit vectors; the top bucket also takes anything above).  Value-domain buckets spread the
-  // shared-memory atomics, which the float's top bits (a few exponents) would not.
-  for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
-  __syncthreads();
-  for (int i = threadIdx.x; i < N; i += blockDim.x) atomicAdd(&bins[tail_bucket(db[i])], 1u);
-  __syncthreads();
-  // counts from the top: thread j owns buckets 4095 - 4j .. 4092 - 4j
+// Called by all 1024 threads: the bin holding the r-th largest entry, counting from bin 4095 down
+// (1 <= r <= total): sel[0] = that bin, sel[1] = entries in the bins above it.  wsum: 32 words.
+__device__ __forceinline__ void select_from_top(const unsigned* bins, unsigned r, unsigned* sel, unsigned* wsum) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int top = kTailBins - 1 - 4 * static_cast<int>(threadIdx.x);   // this thread: bins top .. top - 3
   unsigned c4[4], s4 = 0u;
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
-    c4[q] = bins[kTailBins - 1 - 4 * static_cast<int>(threadIdx.x) - q];
+    c4[q] = bins[top - q];
     s4 += c4[q];
   }
   unsigned incl = s4;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     const unsigned n = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane_id >= o) incl += n;
+    if (lane >= o) incl += n;
   }
-  if (lane_id == 31) cred[warp_id] = incl;
+  if (lane == 31) wsum[warp] = incl;
   __syncthreads();
-  if (warp_id == 0) {
-    unsigned w = cred[lane_id];
+  if (warp == 0) {
+    unsigned w = wsum[lane];
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const unsigned n = __shfl_up_sync(0xffffffffu, w, o);
-      if (lane_id >= o) w += n;
+      if (lane >= o) w += n;
     }
-    cred[lane_id] = w;   // inclusive totals of warps 0 .. lane
+    wsum[lane] = w;   // entries in warps 0 .. lane
   }
   __syncthreads();
-  incl += warp_id > 0 ? cred[warp_id - 1] : 0u;   // inclusive count down to this thread's last bucket
+  incl += warp > 0 ? wsum[warp - 1] : 0u;
   const unsigned excl = incl - s4;
-  if (excl < k && incl >= k) {                     // exactly one thread holds the k-th largest
+  if (excl < r && incl >= r) {   // exactly one thread
     unsigned above = excl;
     int q = 0;
 #pragma unroll
     for (int qq = 0; qq < 3; ++qq)
-      if (q == qq && above + c4[qq] < k) {
+      if (q == qq && above + c4[qq] < r) {
         above += c4[qq];
         q = qq + 1;
       }
-    sel[0] = static_cast<unsigned>(kTailBins - 1 - 4 * static_cast<int>(threadIdx.x) - q);
+    sel[0] = static_cast<unsigned>(top - q);
     sel[1] = above;
   }
   __syncthreads();
-  const int tb = static_cast<int>(sel[0]);
-  // Level 2: radix select (8-bit digits of the float bits) among the bucket's members only
-  const unsigned lo_key = __float_as_uint(static_cast<float>(tb) * (1.0f / 2048.0f));
-  const unsigned hi_key = tb == kTailBins - 1 ? 0xFFFFFFFFu : __float_as_uint(static_cast<float>(tb + 1) * (1.0f / 2048.0f));
-  unsigned prefix = 0u, mask = 0u, remaining = k - sel[1];
+}
+
+__global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTable t, const float* __restrict__ d,
+                                                 TailParams prm, pace_apc_stats* __restrict__ stats) {
+  extern __shared__ float sd[];
+  __shared__ unsigned bins[kTailBins];
+  __shared__ unsigned sel[2];
+  __shared__ float red[32];
+  __shared__ unsigned cred[32];
+  const int b = blockIdx.x;
+  const int N = t.n[b];
+  const float* db = d + t.patch0[b];
+  const unsigned k = static_cast<unsigned>(t.ktail[b]);
+  const int lane_id = threadIdx.x & 31;
+  // Level 1: the k-th largest distance's bucket among 4096 buckets of width 1/2048 (d <= 2 for
+  // unit vectors; the top bucket also takes anything above).  Value-domain buckets spread the
+  // shared-memory atomics, which the float's top bits (a few exponents) would not.  The
+  // distances are staged in shared memory on the way, when they fit.
+  if (N <= kTailSmemMax) {
+    for (int i = threadIdx.x; i < N; i += blockDim.x) cp_async4(sd + i, db + i);
+    db = sd;
+  }
+  for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
+  cp_async_wait_all();
   __syncthreads();
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0u;
+#pragma unroll 4
+  for (int i = threadIdx.x; i < N; i += blockDim.x) atomicAdd(&bins[tail_bucket(db[i])], 1u);
+  __syncthreads();
+  select_from_top(bins, k, sel, cred);
+  const int tb = static_cast<int>(sel[0]);
+  // Level 2: the bucket's members by key offset from its first key, 4096 offsets (2^shift keys
+  // each) at a time, until one key is left: the k-th largest distance.
+  unsigned lo = __float_as_uint(static_cast<float>(tb) * (1.0f / 2048.0f));
+  unsigned span = (tb == kTailBins - 1 ? 0x7F800001u : __float_as_uint(static_cast<float>(tb + 1) * (1.0f / 2048.0f))) - lo;
+  unsigned remaining = k - sel[1];
+  while (true) {
+    const int bits = 32 - __clz(span - 1u);        // keys lo .. lo + span - 1 need `bits` bits
+    const int shift = bits > 12 ? bits - 12 : 0;
+    __syncthreads();                               // everyone has read sel and the bins
+    for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
     __syncthreads();
-    for (int i = threadIdx.x; i < N; i += blockDim.x) {
-      const unsigned key = __float_as_uint(db[i]);
-      if (key >= lo_key && (key < hi_key || tb == kTailBins - 1) && (key & mask) == prefix)
-        atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    for (int base = 0; base < N; base += blockDim.x) {   // uniform trip count: __match_any_sync below
+      const int i = base + static_cast<int>(threadIdx.x);
+      const unsigned off = i < N ? __float_as_uint(db[i]) - lo : span;   // wraps for keys below lo
+      const bool in = off < span;
+      const unsigned digit = in ? off >> shift : kTailBins;
+      const unsigned members = __ballot_sync(0xffffffffu, in);
+      if (__popc(members) > 4) {
+        // many members in this warp: lanes with the same digit add once (identical distances
+        // would otherwise serialise on one counter)
+        const unsigned peers = __match_any_sync(0xffffffffu, digit);
+        if (in && lane_id == __ffs(peers) - 1) atomicAdd(&bins[digit], static_cast<unsigned>(__popc(peers)));
+      } else if (in) {
+        atomicAdd(&bins[digit], 1u);
+      }
     }
     __syncthreads();
-    if (threadIdx.x < 32) warp_digit_search(hist, remaining, sel);
-    __syncthreads();
-    prefix |= sel[0] << shift;
-    mask |= 255u << shift;
+    select_from_top(bins, remaining, sel, cred);
+    lo += sel[0] << shift;
     remaining -= sel[1];
-    __syncthreads();
+    if (shift == 0) break;
+    span = min(span - (sel[0] << shift), 1u << shift);
   }
+  const unsigned prefix = lo;
   const float T = __uint_as_float(prefix);   // k-th largest d
   float s = 0.f;
   unsigned cnt = 0u;
@@ -837,6 +959,22 @@ DensityLayout density_layout(int B, const int32_t* H, const int32_t* W) {
 }
 
 // Dynamic shared memory of apc_tail: the largest image's distances when they fit.
+// Grid of the strip passes: the CTAs that are resident at once (capped by the strips).
+unsigned strip_grid(int units) {
+  static std::atomic<int> cap[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) dev = 0;
+  int c = cap[dev & 63].load(std::memory_order_relaxed);
+  if (c == 0) {
+    int nsm = 0, per = 0;
+    cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, apc_pass2<true>, kApcThreads, 0);
+    c = std::max(1, nsm * std::max(per, 1));
+    cap[dev & 63].store(c, std::memory_order_relaxed);
+  }
+  return static_cast<unsigned>(std::max(1, std::min(units, c)));
+}
+
 size_t tail_smem(const ApcTable& t) {
   int n = 0;
   for (int i = 0; i < t.nb; ++i) n = std::max(n, t.n[i]);
@@ -928,11 +1066,11 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
       if ((static_cast<int64_t>(W[b]) * 3) % 4 != 0 || (t.gw[i] % 2) != 0 || (img_off[b] % 4) != 0) wide = false;
     }
     const int units = t.unit_prefix[nb];
-    if (wide) apc_pass1<true><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums);
-    else apc_pass1<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums);
+    if (wide) apc_pass1<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums);
+    else apc_pass1<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums);
     PACE_CHECK(check_launch());
-    if (wide) apc_pass2<true><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d, stats);
-    else apc_pass2<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d, stats);
+    if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats);
+    else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats);
     PACE_CHECK(check_launch());
     TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
     apc_tail<<<nb, 1024, tail_smem(t), stream>>>(t, d, tp, stats);
@@ -1095,11 +1233,11 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
     if ((static_cast<int64_t>(W[b]) * 3) % 4 != 0 || (t.gw[b] % 2) != 0 || (img_off[b] % 4) != 0) wide = false;
   }
   const int units = t.unit_prefix[B];
-  if (wide) apc_pass1<true><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums);
-  else apc_pass1<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums);
+  if (wide) apc_pass1<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums);
+  else apc_pass1<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums);
   PACE_CHECK(check_launch());
-  if (wide) apc_pass2<true><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d_out, stats);
-  else apc_pass2<false><<<units, kApcThreads, 0, stream>>>(img, t, inv, sums, d_out, stats);
+  if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats);
+  else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats);
   PACE_CHECK(check_launch());
   TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
   apc_tail<<<B, 1024, tail_smem(t), stream>>>(t, d_out, tp, stats);
