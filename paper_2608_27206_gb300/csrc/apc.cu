@@ -655,8 +655,8 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
 // ------------------------------------------------------------------------------------------------
 // resample
 // ------------------------------------------------------------------------------------------------
-constexpr int kRsThreads = 128;  // threads of a resample CTA
-constexpr int kRsTH = 4;         // output rows of a generic tile (kRsTH x kRsTW = kRsThreads)
+constexpr int kRsThreads = 256;  // threads of a resample CTA
+constexpr int kRsTH = 8;         // output rows of a generic tile (kRsTH x kRsTW = kRsThreads)
 constexpr int kRsTW = 32;        // output columns of a generic tile
 constexpr int kRsChunk = 8;      // input rows filtered per step of the generic path
 
@@ -805,7 +805,7 @@ constexpr int kFPitch = 368;                 // bytes per staged row: 3 * kFCols
 constexpr int kFLine = kFTW * 3;             // floats per row of the horizontal result
 static_assert(kFPitch >= 3 * kFCols + 6 && kFPitch % 16 == 0, "staged row pitch");
 static_assert(kFRows >= kFTH * 2.75 + 14 && kFCols >= kFTW * 2.75 + 14 + kFMaxTaps, "staged window");
-static_assert(3 * kFTW <= kRsThreads && 64 + kFTH <= kRsThreads, "thread roles of the fast tile");
+static_assert(3 * kFTW <= kRsThreads / 2 && 64 + kFTH <= kRsThreads, "thread roles of the fast tile");
 constexpr size_t kFSmem = static_cast<size_t>(kFRows) * kFPitch + static_cast<size_t>(kFRows) * kFLine * 4 +
                           (kFTW + kFTH) * kFMaxTaps * 4 + (2 * kFTW + 2 * kFTH + kFRows + 4) * 4;
 constexpr int kRsCtasPerSm = 4;
@@ -849,46 +849,65 @@ __device__ __forceinline__ void resample_tile_fast(const uint8_t* __restrict__ i
   const int x0 = xlo[0], x1 = xlo[ncol - 1] + xn[ncol - 1];
   const int y0 = ylo[0], y1 = ylo[nrow - 1] + yn[nrow - 1];
   const int nin_c = x1 - x0, nin_r = y1 - y0;
-  // stage the input window (4-byte words covering each row segment)
+  // stage the input window (4-byte words covering each row segment), asynchronously: a warp per
+  // row, every copy in flight at once
   const int64_t pitch = static_cast<int64_t>(W) * 3;
+  const int64_t img_bytes = static_cast<int64_t>(H) * pitch;
   const int words = (nin_c * 3 + 3 + 3) >> 2;
-  for (int i = tid; i < nin_r * words; i += kRsThreads) {
-    const int r = i / words, w = i - r * words;
+  for (int r = tid >> 5; r < nin_r; r += kRsThreads / 32) {
     const int64_t start = (static_cast<int64_t>(y0 + r) * pitch + static_cast<int64_t>(x0) * 3);
     const int64_t a = start & ~int64_t{3};
-    if (w == 0) shift[r] = static_cast<int>(start - a);
-    const int64_t byte = a + 4 * w;
-    if (byte < static_cast<int64_t>(H) * pitch)
-      *reinterpret_cast<uint32_t*>(sin + r * kFPitch + 4 * w) = __ldg(reinterpret_cast<const uint32_t*>(img + byte));
+    if ((tid & 31) == 0) shift[r] = static_cast<int>(start - a);
+    for (int w = tid & 31; w < words; w += 32)
+      if (a + 4 * w < img_bytes) cp_async4(sin + r * kFPitch + 4 * w, img + a + 4 * w);
   }
+  cp_async_wait_all();
   __syncthreads();
-  if (tid < 3 * ncol) {
-    // horizontal pass: every staged row, this thread's (column, channel)
+  // the two halves of the CTA take the two halves of the rows; thread tt = (column, channel)
+  const int half = tid / (kRsThreads / 2), tt = tid - half * (kRsThreads / 2);
+  if (tt < 3 * ncol) {
+    // horizontal pass: this half's staged rows, this thread's (column, channel)
     // (taps past the window have weight 0 and read staged bytes that exist: the staged row
     // holds kFCols >= the window of the last column + MAXT pixels)
-    const int c = tid / 3, ch = tid - 3 * c;
+    const int c = tt / 3, ch = tt - 3 * c;
     const int n = xn[c];
     float w[MAXT];
 #pragma unroll
     for (int k = 0; k < MAXT; ++k) w[k] = k < n ? wx[c * kFMaxTaps + k] : 0.f;
     const int base = (xlo[c] - x0) * 3 + ch;
-    for (int r = 0; r < nin_r; ++r) {
+    const int r_end = half ? nin_r : (nin_r + 1) / 2;
+    int r = half ? (nin_r + 1) / 2 : 0;
+    for (; r + 1 < r_end; r += 2) {   // two rows at a time: twice the independent work in flight
+      const unsigned char* px0 = sin + r * kFPitch + shift[r] + base;
+      const unsigned char* px1 = sin + (r + 1) * kFPitch + shift[r + 1] + base;
+      float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll
+      for (int k = 0; k < MAXT; ++k) {
+        acc0 = fmaf(w[k], byte_to_float(px0[3 * k]), acc0);
+        acc1 = fmaf(w[k], byte_to_float(px1[3 * k]), acc1);
+      }
+      sh[r * kFLine + tt] = acc0;
+      sh[(r + 1) * kFLine + tt] = acc1;
+    }
+    if (r < r_end) {
       const unsigned char* px = sin + r * kFPitch + shift[r] + base;
       float acc = 0.f;
 #pragma unroll
       for (int k = 0; k < MAXT; ++k) acc = fmaf(w[k], byte_to_float(px[3 * k]), acc);
-      sh[r * kFLine + tid] = acc;
+      sh[r * kFLine + tt] = acc;
     }
   }
   __syncthreads();
-  if (tid < 3 * ncol) {
-    // vertical pass and the uint8 store (a row of the tile is 3 * ncol consecutive bytes)
-    uint8_t* o = out + (static_cast<int64_t>(oy0) * Wo + ox0) * 3 + tid;
-    for (int r = 0; r < nrow; ++r) {
+  if (tt < 3 * ncol) {
+    // vertical pass and the uint8 store (a row of the tile is 3 * ncol consecutive bytes); the
+    // halves take alternate output rows
+    uint8_t* o = out + (static_cast<int64_t>(oy0) * Wo + ox0) * 3 + tt;
+    for (int r = half; r < nrow; r += 2) {
       const float* w = wy + r * kFMaxTaps;
-      const float* col = sh + (ylo[r] - y0) * kFLine + tid;
+      const float* col = sh + (ylo[r] - y0) * kFLine + tt;
       const int n = yn[r];
       float acc = 0.f;
+#pragma unroll 4
       for (int k = 0; k < n; ++k) acc = fmaf(w[k], col[k * kFLine], acc);
       o[static_cast<int64_t>(r) * Wo * 3] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc))));
     }
