@@ -281,6 +281,97 @@ def algorithmic_counts(wl, keep, r_ratio):
     }
 
 
+def measure_next_rows(P, device, flush, peak_tf, hbm_gbs, reps=10):
+    """Times the calls of the paths beyond the step (preview-token density, full-sequence S_llm,
+    the prune step's gathers) on the 4K image's shapes, each replayed from a CUDA graph with L2
+    flushed before every replay; median over `reps`.  Inputs are seeded device tensors."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(1234)
+
+    def randn(*shape, scale=1.0):
+        return (torch.randn(*shape, generator=g, device=device) * scale).to(torch.bfloat16)
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        st = torch.cuda.Stream(device)
+        with torch.cuda.stream(st):
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=st):
+                fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            gr.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        return statistics.median(ts) * 1e-3   # seconds
+
+    out = {}
+    # f1: APC density on preview tokens: 42196 tokens x 1280 (ViT hidden width), bf16
+    n_tok, dim = 42196, 1280
+    T = randn(n_tok, dim)
+    cu = [0, n_tok]
+    d = torch.empty(n_tok, dtype=torch.float32, device=device)
+    st = torch.zeros((1, 10), dtype=torch.int32, device=device)
+    ws = torch.empty(max(P.pace_apc_density_tokens_workspace_size(cu, dim), 16), dtype=torch.uint8, device=device)
+    sec = timed(lambda: P.pace_apc_density_tokens(T, cu, [3836], [2156], d_out=d, stats=st, ws=ws))
+    nbytes = 2 * n_tok * dim * 2 + 4 * n_tok
+    out["f1_density_tokens"] = {"shape": f"T bf16 [{n_tok},{dim}]", "us": round(sec * 1e6, 2), "bound": "hbm",
+                                "bytes": nbytes, "achieved": round(nbytes / sec / 1e9, 1), "unit": "GB/s",
+                                "frac": round(nbytes / sec / 1e9 / hbm_gbs, 4)}
+    del T, d, ws
+    # f2: full-sequence S_llm (Vision+Text queries, causal): system 20 + 10549 visual + 256 text
+    v, nv, nt = 20, 10549, 256
+    S = v + nv + nt
+    Q = randn(S, 28, 128)
+    K = randn(S, 4, 128)
+    o = torch.empty(nv, dtype=torch.float32, device=device)
+    wsq = torch.empty(max(P.pace_llm_sequence_importance_workspace_size([0, S], [v], [nv], 28, 4), 16),
+                      dtype=torch.uint8, device=device)
+    sec = timed(lambda: P.pace_llm_sequence_importance(Q, K, [0, S], [v], [nv], "vision_text", out=o, ws=wsq))
+    # pass 1: query at position p (p >= v) sees p + 1 keys; pass 2: visual key at position q is
+    # seen by the S - q queries at or after it
+    pairs1 = sum(p + 1 for p in range(v, S))
+    pairs2 = sum(S - q for q in range(v, v + nv))
+    flops = 2 * 128 * 28 * (pairs1 + pairs2)
+    out["f2_sequence_importance"] = {"shape": f"Q bf16 [{S},28,128], K bf16 [{S},4,128], vision_text",
+                                     "us": round(sec * 1e6, 2), "bound": "tensor", "flops": flops,
+                                     "achieved": round(flops / sec / 1e12, 1), "unit": "TFLOP/s",
+                                     "frac": round(flops / sec / 1e12 / peak_tf, 4)}
+    del Q, K, o, wsq
+    # f3: prune step: row list + one gather of hidden states [S, 3584], the K and V rows of layers
+    # 0..2 ([S, 4, 128] each) and the M-RoPE ids [3, S] (int64), keep 10 % of the visual tokens
+    keep = P.pace_budget(nv, 0.10)
+    kept = torch.sort(torch.randperm(nv, generator=g, device=device)[:keep])[0].to(torch.int32)
+    n_out = S - nv + keep
+    idx = torch.empty(n_out, dtype=torch.int32, device=device)
+    hid = randn(S, 3584)
+    kv = [randn(S, 4, 128) for _ in range(6)]
+    pos = torch.arange(3 * S, device=device, dtype=torch.int64).view(3, S)
+    hid_o = torch.empty(n_out, 3584, dtype=torch.bfloat16, device=device)
+    kv_o = [torch.empty(n_out, 4, 128, dtype=torch.bfloat16, device=device) for _ in range(6)]
+    pos_o = torch.empty(3, n_out, dtype=torch.int64, device=device)
+    specs = [P.gather_spec(hid, hid_o, 0)] + [P.gather_spec(a, b, 0) for a, b in zip(kv, kv_o)] + \
+            [P.gather_spec(pos, pos_o, 1)]
+
+    def prune():
+        P.pace_prune_index([0, S], [v], [0, nv], [0, keep], kept, out=idx)
+        P.pace_gather_multi(specs, idx)
+    sec = timed(prune)
+    nbytes = 2 * n_out * (3584 * 2 + 6 * 4 * 128 * 2 + 3 * 8) + 4 * keep + 4 * n_out
+    out["f3_prune_gather"] = {"shape": f"{n_out} of {S} rows: hidden [S,3584] + 6 KV [S,4,128] bf16 + ids [3,S]",
+                              "us": round(sec * 1e6, 2), "bound": "hbm", "bytes": nbytes,
+                              "achieved": round(nbytes / sec / 1e9, 1), "unit": "GB/s",
+                              "frac": round(nbytes / sec / 1e9 / hbm_gbs, 4)}
+    return out
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -405,6 +496,7 @@ def run_gpu(args):
         llm_tf = cnt["llm_flops"] / (mean["llm"] * 1e-3) / 1e12
         other["llm"] = {"bound": "tensor", "us": round(mean["llm"] * 1e3, 2), "achieved": round(llm_tf, 1),
                         "peak": peak, "unit": "TFLOP/s", "frac": round(llm_tf / peak, 4), "flops": cnt["llm_flops"]}
+        nxt = measure_next_rows(P, device, flush, peak, hbm) if world == 1 else None
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
             tot, parts, sample = oracle_sample(wl, KEEP, vit_rows=args.ref_vit_rows)
@@ -431,6 +523,7 @@ def run_gpu(args):
                          "peak_source": f"{peak_src} bf16 dense burst (MEASURED_PEAKS.json)"
                          if peak_src == "measured" else "fallback 1.9 PFLOP/s bf16"},
             "rooflines_other": other,
+            "next_rows": nxt,
             "breakdown_us": {k: round(v * 1e3, 2) for k, v in mean.items()},
             "visual_tokens_scored_per_s": round(wl.n_vis[0] * world / (ms_per_step * 1e-3), 1),
             "cpu_baseline": cpu,
