@@ -40,6 +40,21 @@ Readings taken where the paper is silent or cannot be followed literally
       the visual span under the causal mask), after the visual span (Text) or
       at the last position (Last); each query's softmax runs over every
       position up to and including itself.
+  R14 pixel-statistic preview features (pixel_statistic_tokens; App. "Shallow
+      Feature Preview Ablation" names them without a definition): per 14x14
+      patch, with luma Y' = 299 R + 587 G + 114 B in integers (BT.601 weights
+      in thousandths; Y = Y' / 255000 in [0, 1]) and the patch's 12x12 interior
+      for the 3x3 operators:
+        rgb_stats      [mean_R, mean_G, mean_B, std_R, std_G, std_B, 1] of x / 255
+                       (population standard deviations);
+        color_entropy  [H_R, H_G, H_B, 4] / 4, H_c the Shannon entropy (bits) of
+                       the patch's 16-bin histogram of channel c (bin = value >> 4);
+        edge_density   [e, 1], e the fraction of interior pixels whose Sobel
+                       gradient magnitude of Y exceeds 0.25;
+        laplacian      [s, 1], s the population standard deviation of the
+                       4-neighbour Laplacian of Y over the interior.
+      The constant last coordinate plays the role it has in R1: a token is never
+      zero and the cosines of Eq. 1 see the size of the statistic.
 """
 from __future__ import annotations
 
@@ -132,6 +147,64 @@ def apc_density(img: np.ndarray, alpha: float = ALPHA, gamma: float = GAMMA,
                 tail_frac: float = TAIL_FRAC, r_min: float = 0.0, r_max: float = 1.0):
     """Full APC decision for one image: density statistics, r and the target size."""
     st = apc_density_tokens(patch_tokens(img), alpha, gamma, tail_frac)
+    st["r"] = retention_ratio(st["rho"], r_min, r_max)
+    st["H_out"], st["W_out"] = target_size(img.shape[0], img.shape[1], st["r"])
+    return st
+
+
+# Pixel-statistic preview features (App. "Shallow Feature Preview Ablation"), reading R14.
+PIXEL_FEATURES = ("rgb_stats", "color_entropy", "edge_density", "laplacian")
+FEATURE_DIMS = {"rgb_stats": 7, "color_entropy": 4, "edge_density": 2, "laplacian": 2}
+LUMA_WEIGHTS = (299, 587, 114)   # thousandths; Y' = 299 R + 587 G + 114 B
+LUMA_SCALE = 255000              # Y' of a white pixel
+EDGE_TAU = 0.25                  # Sobel magnitude threshold on Y in [0, 1]
+ENTROPY_BINS = 16
+
+
+def patches(img: np.ndarray) -> np.ndarray:
+    """The 14x14x3 patches of an image in raster order: uint8 [N, 14, 14, 3]."""
+    H, W, _ = img.shape
+    gh, gw = H // PATCH, W // PATCH
+    x = img[: gh * PATCH, : gw * PATCH]
+    return x.reshape(gh, PATCH, gw, PATCH, 3).transpose(0, 2, 1, 3, 4).reshape(gh * gw, PATCH, PATCH, 3)
+
+
+def pixel_statistic_tokens(img: np.ndarray, feature: str) -> np.ndarray:
+    """Reading R14: the feature token [N, FEATURE_DIMS[feature]] of every patch."""
+    P = patches(img).astype(np.int64)
+    N = P.shape[0]
+    one = np.ones((N, 1))
+    if feature == "rgb_stats":
+        x = P.reshape(N, PATCH * PATCH, 3) / 255.0
+        return np.concatenate([x.mean(axis=1), x.std(axis=1), one], axis=1)
+    if feature == "color_entropy":
+        H = np.zeros((N, 3))
+        for c in range(3):
+            bins = P[..., c].reshape(N, -1) >> 4
+            for i in range(N):
+                p = np.bincount(bins[i], minlength=ENTROPY_BINS) / float(PATCH * PATCH)
+                p = p[p > 0]
+                H[i, c] = float(-(p * np.log2(p)).sum())
+        return np.concatenate([H / 4.0, one], axis=1)
+    Y = P[..., 0] * LUMA_WEIGHTS[0] + P[..., 1] * LUMA_WEIGHTS[1] + P[..., 2] * LUMA_WEIGHTS[2]   # [N, 14, 14]
+    c = Y[:, 1:-1, 1:-1]
+    if feature == "edge_density":
+        gx = (Y[:, :-2, 2:] + 2 * Y[:, 1:-1, 2:] + Y[:, 2:, 2:]) - (Y[:, :-2, :-2] + 2 * Y[:, 1:-1, :-2] + Y[:, 2:, :-2])
+        gy = (Y[:, 2:, :-2] + 2 * Y[:, 2:, 1:-1] + Y[:, 2:, 2:]) - (Y[:, :-2, :-2] + 2 * Y[:, :-2, 1:-1] + Y[:, :-2, 2:])
+        thr = int(round(EDGE_TAU * LUMA_SCALE)) ** 2        # exact: magnitudes compared in integers
+        e = ((gx * gx + gy * gy) > thr).reshape(N, -1).mean(axis=1)
+        return np.stack([e, np.ones(N)], axis=1)
+    if feature == "laplacian":
+        lap = Y[:, 1:-1, :-2] + Y[:, 1:-1, 2:] + Y[:, :-2, 1:-1] + Y[:, 2:, 1:-1] - 4 * c
+        s = lap.reshape(N, -1).astype(np.float64).std(axis=1) / LUMA_SCALE
+        return np.stack([s, np.ones(N)], axis=1)
+    raise ValueError(feature)
+
+
+def apc_density_pixel(img: np.ndarray, feature: str, alpha: float = ALPHA, gamma: float = GAMMA,
+                      tail_frac: float = TAIL_FRAC, r_min: float = 0.0, r_max: float = 1.0):
+    """APC (Eq. 1-6, r, target size) with a pixel-statistic preview in place of T_v (R14)."""
+    st = apc_density_tokens(pixel_statistic_tokens(img, feature), alpha, gamma, tail_frac)
     st["r"] = retention_ratio(st["rho"], r_min, r_max)
     st["H_out"], st["W_out"] = target_size(img.shape[0], img.shape[1], st["r"])
     return st

@@ -398,3 +398,63 @@ def test_llm_sequence_importance_brute_force_and_mass():
     got = O.llm_sequence_importance(Q2 * 0 + 1.0, K2 * 0 + np.r_[np.ones(nv), np.zeros(S - nv)][:, None, None],
                                     [0, S], [0], [nv], 50.0, "text")
     assert got.sum() == pytest.approx((S - nv) * Hq, rel=1e-9)
+
+
+# ----------------------------------------------------------------------------------------------
+# Pixel-statistic preview features (App. "Shallow Feature Preview Ablation"; reading R14)
+# ----------------------------------------------------------------------------------------------
+def _one_patch(pix):
+    """A 14 x 14 image of one patch from a 14 x 14 grey-level array (R = G = B)."""
+    return np.repeat(np.asarray(pix, dtype=np.uint8)[:, :, None], 3, axis=2)
+
+
+def test_pixel_features_two_tone_closed_forms():
+    # left 7 columns black, right 7 white: every channel is 0 or 1 with probability 1/2, so
+    # mean = std = 1/2; two of 16 bins hold half the pixels each: 1 bit -> 1/4 after scaling.
+    # Sobel: only interior columns 6 and 7 straddle the boundary (2 x 12 of 144 pixels), with
+    # |G| = 4 (one full step weighted 1 + 2 + 1) > 0.25.  Laplacian: +1 on column 6 (one white
+    # neighbour), -1 on column 7 (one black neighbour), 0 elsewhere: std = sqrt(24 / 144).
+    pix = np.zeros((14, 14))
+    pix[:, 7:] = 255
+    img = _one_patch(pix)
+    np.testing.assert_allclose(O.pixel_statistic_tokens(img, "rgb_stats")[0], [0.5] * 6 + [1.0], atol=1e-15)
+    np.testing.assert_allclose(O.pixel_statistic_tokens(img, "color_entropy")[0], [0.25] * 3 + [1.0], atol=1e-15)
+    np.testing.assert_allclose(O.pixel_statistic_tokens(img, "edge_density")[0], [1 / 6, 1.0], atol=1e-15)
+    np.testing.assert_allclose(O.pixel_statistic_tokens(img, "laplacian")[0], [math.sqrt(1 / 6), 1.0], atol=1e-15)
+    # the same split across rows exercises the other gradient and neighbour directions
+    imgT = _one_patch(pix.T)
+    np.testing.assert_allclose(O.pixel_statistic_tokens(imgT, "edge_density")[0], [1 / 6, 1.0], atol=1e-15)
+    np.testing.assert_allclose(O.pixel_statistic_tokens(imgT, "laplacian")[0], [math.sqrt(1 / 6), 1.0], atol=1e-15)
+
+
+def test_pixel_features_checkerboard_and_ramp():
+    # 1-pixel checkerboard: the columns on either side of a pixel carry the same colours, so both
+    # Sobel components vanish (edge density 0), while every Laplacian is +-4 (all four neighbours
+    # opposite): std 4.  A ramp of one grey level per column has zero Laplacian and a Sobel
+    # magnitude of 4 * 2 / 255 < 0.25.
+    y, x = np.mgrid[0:14, 0:14]
+    img = _one_patch(((x + y) % 2) * 255)
+    assert O.pixel_statistic_tokens(img, "edge_density")[0, 0] == 0.0
+    np.testing.assert_allclose(O.pixel_statistic_tokens(img, "laplacian")[0], [4.0, 1.0], atol=1e-12)
+    np.testing.assert_allclose(O.pixel_statistic_tokens(img, "color_entropy")[0, :3], [0.25] * 3, atol=1e-15)
+    ramp = _one_patch(np.tile(np.arange(14) + 40, (14, 1)))
+    assert O.pixel_statistic_tokens(ramp, "laplacian")[0, 0] == 0.0
+    assert O.pixel_statistic_tokens(ramp, "edge_density")[0, 0] == 0.0
+
+
+def test_pixel_features_invariants_and_density():
+    rng = np.random.default_rng(21)
+    img = rng.integers(0, 256, size=(42, 56, 3), dtype=np.uint8)
+    for f in O.PIXEL_FEATURES:
+        T = O.pixel_statistic_tokens(img, f)
+        assert T.shape == (12, O.FEATURE_DIMS[f]) and np.all(T[:, -1] == 1.0)
+        # a constant image gives one token for every patch: phi = 1, d = 0
+        st = O.apc_density_pixel(np.full((28, 42, 3), 77, np.uint8), f)
+        assert abs(st["phi"] - 1.0) < 1e-12 and np.all(np.abs(st["d"]) < 1e-7)
+    # the first-order statistics do not depend on where a pixel sits in its patch
+    perm = rng.permutation(196)
+    P = O.patches(img)[0].reshape(196, 3)[perm].reshape(14, 14, 3)
+    for f in ("rgb_stats", "color_entropy"):
+        np.testing.assert_allclose(O.pixel_statistic_tokens(P, f)[0], O.pixel_statistic_tokens(img, f)[0], atol=1e-12)
+    ent = O.pixel_statistic_tokens(img, "color_entropy")[:, :3]
+    assert np.all(ent >= 0) and np.all(ent <= 1.0)
