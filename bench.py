@@ -325,7 +325,20 @@ def measure_next_rows(P, device, flush, peak_tf, hbm_gbs, reps=10):
     out["f1_density_tokens"] = {"shape": f"T bf16 [{n_tok},{dim}]", "us": round(sec * 1e6, 2), "bound": "hbm",
                                 "bytes": nbytes, "achieved": round(nbytes / sec / 1e9, 1), "unit": "GB/s",
                                 "frac": round(nbytes / sec / 1e9 / hbm_gbs, 4)}
-    del T, d, ws
+    del T, ws
+    # f1: APC density with the four pixel-statistic previews on the 4K image (HBM roofline: the
+    # image read once + 32 B of token written and read twice per patch + d)
+    img = torch.randint(0, 256, (2156 * 3836 * 3,), generator=g, device=device, dtype=torch.uint8)
+    wsp = torch.empty(max(P.pace_apc_density_pixel_workspace_size([2156], [3836]), 16), dtype=torch.uint8,
+                      device=device)
+    for feat in P.PIXEL_FEATURES:
+        sec = timed(lambda: P.pace_apc_density_pixel(img, [0], [2156], [3836], feat, d_out=d, stats=st, ws=wsp))
+        nbytes = img.numel() + n_tok * (3 * 32 + 4)
+        out[f"f1_density_pixel_{feat}"] = {"shape": "3836x2156 RGB uint8", "us": round(sec * 1e6, 2),
+                                           "bound": "hbm", "bytes": nbytes,
+                                           "achieved": round(nbytes / sec / 1e9, 1), "unit": "GB/s",
+                                           "frac": round(nbytes / sec / 1e9 / hbm_gbs, 4)}
+    del img, wsp, d
     # f2: full-sequence S_llm (Vision+Text queries, causal): system 20 + 10549 visual + 256 text
     v, nv, nt = 20, 10549, 256
     S = v + nv + nt

@@ -175,6 +175,50 @@ PACE_API pace_status_t pace_apc_density_tokens(const void* T, const int32_t* cu_
                                                float* d_out, pace_apc_stats* stats, void* ws, size_t ws_bytes,
                                                pace_stream_t stream);
 
+/* Pixel-statistic previews: the four training-free statistics that the preview ablation
+ * (App. "Shallow Feature Preview Ablation") puts in place of the ViT feature.  The paper names
+ * them without a definition; these are the readings used here, per 14 x 14 patch, with integer
+ * luma Y' = 299 R + 587 G + 114 B (Y = Y' / 255000) and the patch's 12 x 12 interior for the
+ * 3 x 3 operators:
+ *   RGB_STATS      [mean_R, mean_G, mean_B, std_R, std_G, std_B, 1] of x / 255 (population std)
+ *   COLOR_ENTROPY  [H_R, H_G, H_B, 4] / 4, H_c the entropy in bits of the 16-bin histogram
+ *                  (value >> 4) of channel c
+ *   EDGE_DENSITY   [e, 1], e the fraction of interior pixels whose Sobel magnitude of Y > 0.25
+ *                  (decided exactly, in integers)
+ *   LAPLACIAN      [s, 1], s the population std of the 4-neighbour Laplacian of Y
+ * A token is stored as 8 floats, zero-padded. */
+typedef enum pace_apc_feature {
+  PACE_APC_FEATURE_RGB_STATS = 0,
+  PACE_APC_FEATURE_COLOR_ENTROPY = 1,
+  PACE_APC_FEATURE_EDGE_DENSITY = 2,
+  PACE_APC_FEATURE_LAPLACIAN = 3
+} pace_apc_feature;
+
+/*
+ * The feature tokens of every patch (raster order per image, images packed).
+ *
+ *  img, img_off, H, W, B  as for pace_apc_density
+ *  feature   pace_apc_feature
+ *  tokens    device  float [sum N_b][8], 16-byte aligned
+ *  Invalid arguments: PACE_ERR_INVALID_ARG before any launch.
+ */
+PACE_API pace_status_t pace_apc_pixel_features(const uint8_t* img, const int64_t* img_off, const int32_t* H,
+                                       const int32_t* W, int B, int feature, float* tokens,
+                                       pace_stream_t stream);
+
+/* Scratch bytes for pace_apc_density_pixel (host H, W [B]). */
+PACE_API size_t pace_apc_density_pixel_workspace_size(int B, const int32_t* H, const int32_t* W);
+
+/*
+ * APC (Sec. 3.2, Eq. 1-6, r and the target size) with a pixel-statistic preview in place of
+ * T_v: the feature tokens above, l2-normalised, through the same statistics and tail as
+ * pace_apc_density.  Arguments as for pace_apc_density plus `feature`; ws holds the tokens.
+ */
+PACE_API pace_status_t pace_apc_density_pixel(const uint8_t* img, const int64_t* img_off, const int32_t* H,
+                                      const int32_t* W, int B, int feature, const pace_apc_params* params,
+                                      float* d_out, pace_apc_stats* stats, void* ws, size_t ws_bytes,
+                                      pace_stream_t stream);
+
 /*
  * APC resize (Sec. 3.2 "Adaptive Condensation"; App. B.3: width and height scaled by
  * sqrt(r), bicubic).  Separable cubic convolution (a = -0.5) with centre-aligned

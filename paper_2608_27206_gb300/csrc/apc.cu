@@ -653,6 +653,242 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
 }
 
 // ------------------------------------------------------------------------------------------------
+// pixel-statistic previews (App. "Shallow Feature Preview Ablation"): one small token per patch,
+// then Eq. 1-6 on those tokens
+// ------------------------------------------------------------------------------------------------
+// Token of patch i: kPixDim floats, zero-padded.  Feature codes as pace_apc_feature.
+constexpr int kPixDim = 8;
+constexpr int kFeatRgb = 0, kFeatEntropy = 1, kFeatEdge = 2, kFeatLaplacian = 3;
+constexpr int kLumaR = 299, kLumaG = 587, kLumaB = 114;   // Y' = 299 R + 587 G + 114 B (BT.601, thousandths)
+constexpr int kLumaScale = 255000;                         // Y' of white
+constexpr long long kEdgeThr2 = 63750LL * 63750LL;         // (0.25 * 255000)^2: Sobel magnitude test in integers
+
+__device__ __forceinline__ int warp_sum_i(int v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ long long warp_sum_ll(long long v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// One warp computes the feature token of the patch at `px` (staged strip, row pitch
+// kStripRowBytes): out[0 .. kPixDim).  `luma` (196 ints) and `hist` (48 ints) are the warp's
+// scratch in shared memory.
+__device__ __forceinline__ void patch_feature(const uint8_t* px, int feature, int* luma, int* hist, float* out) {
+  const int lane = threadIdx.x & 31;
+  float tok[kPixDim] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if (feature == kFeatRgb) {
+    uint32_t s[3] = {0u, 0u, 0u}, q[3] = {0u, 0u, 0u};
+    for (int i = lane; i < kPatch * kPatch; i += 32) {
+      const uint8_t* p = px + (i / kPatch) * kStripRowBytes + (i % kPatch) * 3;
+#pragma unroll
+      for (int c = 0; c < 3; ++c) {
+        const uint32_t v = p[c];
+        s[c] += v;
+        q[c] += v * v;
+      }
+    }
+#pragma unroll
+    for (int c = 0; c < 3; ++c) {
+      const uint32_t S = static_cast<uint32_t>(warp_sum_i(static_cast<int>(s[c])));
+      const uint32_t Q = static_cast<uint32_t>(warp_sum_i(static_cast<int>(q[c])));
+      constexpr float kInv = 1.0f / (196.0f * 255.0f);
+      tok[c] = static_cast<float>(S) * kInv;
+      tok[3 + c] = sqrtf(static_cast<float>(196u * Q - S * S)) * kInv;   // 196 Q - S^2 >= 0, < 2^32
+    }
+    tok[6] = 1.f;
+  } else if (feature == kFeatEntropy) {
+    for (int i = lane; i < 48; i += 32) hist[i] = 0;
+    __syncwarp();
+    for (int i = lane; i < kPatch * kPatch; i += 32) {
+      const uint8_t* p = px + (i / kPatch) * kStripRowBytes + (i % kPatch) * 3;
+#pragma unroll
+      for (int c = 0; c < 3; ++c) atomicAdd(&hist[c * 16 + (p[c] >> 4)], 1);
+    }
+    __syncwarp();
+#pragma unroll
+    for (int c = 0; c < 3; ++c) {
+      float h = 0.f;
+      if (lane < 16) {
+        const int n = hist[c * 16 + lane];
+        if (n > 0) {
+          const float pr = static_cast<float>(n) * (1.0f / 196.0f);
+          h = -pr * log2f(pr);
+        }
+      }
+      h = warp_sum_f(h);
+      tok[c] = h * 0.25f;
+    }
+    tok[3] = 1.f;
+    __syncwarp();   // hist is rewritten by the warp's next patch
+  } else {
+    for (int i = lane; i < kPatch * kPatch; i += 32) {
+      const uint8_t* p = px + (i / kPatch) * kStripRowBytes + (i % kPatch) * 3;
+      luma[i] = kLumaR * p[0] + kLumaG * p[1] + kLumaB * p[2];
+    }
+    __syncwarp();
+    int cnt = 0, sl = 0;
+    long long sl2 = 0;
+    for (int i = lane; i < 144; i += 32) {   // the 12 x 12 interior
+      const int y = 1 + i / 12, x = 1 + i % 12;
+      const int* r0 = luma + (y - 1) * kPatch + x;
+      const int* r1 = r0 + kPatch;
+      const int* r2 = r1 + kPatch;
+      if (feature == kFeatEdge) {
+        const long long gx = (r0[1] + 2 * r1[1] + r2[1]) - (r0[-1] + 2 * r1[-1] + r2[-1]);
+        const long long gy = (r2[-1] + 2 * r2[0] + r2[1]) - (r0[-1] + 2 * r0[0] + r0[1]);
+        cnt += (gx * gx + gy * gy > kEdgeThr2) ? 1 : 0;
+      } else {
+        const int l = r1[-1] + r1[1] + r0[0] + r2[0] - 4 * r1[0];
+        sl += l;
+        sl2 += static_cast<long long>(l) * l;
+      }
+    }
+    if (feature == kFeatEdge) {
+      tok[0] = static_cast<float>(warp_sum_i(cnt)) * (1.0f / 144.0f);
+    } else {
+      const long long S = static_cast<long long>(warp_sum_i(sl)), Q = warp_sum_ll(sl2);
+      const long long num = 144 * Q - S * S;   // 144^2 var in Y'^2 units, exact
+      tok[0] = sqrtf(static_cast<float>(num)) * (1.0f / (144.0f * static_cast<float>(kLumaScale)));
+    }
+    tok[1] = 1.f;
+    __syncwarp();   // luma is rewritten by the warp's next patch
+  }
+  if (lane < kPixDim) {
+    float v = tok[0];
+#pragma unroll
+    for (int k = 1; k < kPixDim; ++k)
+      if (lane == k) v = tok[k];
+    out[lane] = v;
+  }
+}
+
+// Feature tokens of every patch: a resident grid over the strips (as the density passes),
+// a warp per patch.
+template <bool WIDE>
+__global__ void __launch_bounds__(kApcThreads) apc_pix_features(const uint8_t* __restrict__ img,
+                                                                const __grid_constant__ ApcTable t, int units,
+                                                                int feature, float* __restrict__ tokens) {
+  __shared__ __align__(16) uint8_t s2[2][kPatch * kStripRowBytes];
+  __shared__ int luma[kApcThreads / 32][kPatch * kPatch];
+  __shared__ int hist[kApcThreads / 32][48];
+  int unit = blockIdx.x;
+  if (unit >= units) return;
+  const int warp = threadIdx.x >> 5;
+  issue_strip<WIDE>(img, t, unit, s2[0]);
+  for (int i = 0; unit < units; ++i, unit += gridDim.x) {
+    const int next = unit + static_cast<int>(gridDim.x);
+    if (next < units) {
+      issue_strip<WIDE>(img, t, next, s2[(i + 1) & 1]);
+      cp_async_wait_group<1>();
+    } else {
+      cp_async_wait_group<0>();
+    }
+    __syncthreads();
+    const Strip q = strip_of(t, unit);
+    const uint8_t* s = s2[i & 1];
+    for (int p = warp; p < q.np; p += kApcThreads / 32)
+      patch_feature(s + p * 42, feature, luma[warp], hist[warp],
+                    tokens + (static_cast<int64_t>(t.patch0[q.b]) + q.py * t.gw[q.b] + q.px0 + p) * kPixDim);
+    __syncthreads();   // this buffer is refilled two strips on
+  }
+}
+
+// Density of kPixDim-float tokens, pass 1: t_hat in place and the chunk's column sums (2^-32
+// fixed point, deterministic).  A CTA takes kApcThreads tokens of one image, a thread per token.
+struct PixTable {
+  int tok0[kApcMaxB];
+  int n[kApcMaxB];
+  int ktail[kApcMaxB];
+  int unit_prefix[kApcMaxB + 1];
+  int nb;
+  int b_base;
+};
+
+__device__ __forceinline__ int find_pix_image(const PixTable& t, int unit) {
+  int b = 0;
+  while (b + 1 < t.nb && t.unit_prefix[b + 1] <= unit) ++b;
+  return b;
+}
+
+__global__ void __launch_bounds__(kApcThreads) apc_pix_pass1(const __grid_constant__ PixTable t,
+                                                             float* __restrict__ tokens,
+                                                             unsigned long long* __restrict__ sums) {
+  __shared__ float part[kApcThreads / 32][kPixDim];
+  const int b = find_pix_image(t, blockIdx.x);
+  const int i = (blockIdx.x - t.unit_prefix[b]) * kApcThreads + threadIdx.x;
+  const bool live = i < t.n[b];
+  float v[kPixDim] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  float4* row = reinterpret_cast<float4*>(tokens + (static_cast<int64_t>(t.tok0[b]) + (live ? i : 0)) * kPixDim);
+  if (live) {
+    const float4 a = row[0], c = row[1];
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = c.x; v[5] = c.y; v[6] = c.z; v[7] = c.w;
+    float n2 = 0.f;
+#pragma unroll
+    for (int k = 0; k < kPixDim; ++k) n2 = fmaf(v[k], v[k], n2);
+    const float iv = n2 > 0.f ? 1.0f / sqrtf(n2) : 0.f;
+#pragma unroll
+    for (int k = 0; k < kPixDim; ++k) v[k] *= iv;
+    row[0] = make_float4(v[0], v[1], v[2], v[3]);
+    row[1] = make_float4(v[4], v[5], v[6], v[7]);
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+  for (int k = 0; k < kPixDim; ++k) {
+    const float w = warp_sum_f(v[k]);
+    if (lane == 0) part[warp][k] = w;
+  }
+  __syncthreads();
+  if (threadIdx.x < kPixDim) {
+    float a = 0.f;
+#pragma unroll
+    for (int w = 0; w < kApcThreads / 32; ++w) a += part[w][threadIdx.x];
+    atomicAdd(sums + static_cast<int64_t>(t.b_base + b) * kPixDim + threadIdx.x, fix32_signed(a));
+  }
+}
+
+// Pass 2: c = sums / N, phi = |c|^2, c_hat = c / |c|, d_i = |t_hat_i - c_hat| (thread per token).
+__global__ void __launch_bounds__(kApcThreads) apc_pix_pass2(const __grid_constant__ PixTable t,
+                                                             const float* __restrict__ tokens,
+                                                             const unsigned long long* __restrict__ sums,
+                                                             float* __restrict__ d_out,
+                                                             pace_apc_stats* __restrict__ stats) {
+  const int b = find_pix_image(t, blockIdx.x);
+  const int u = blockIdx.x - t.unit_prefix[b];
+  const int i = u * kApcThreads + threadIdx.x;
+  const int N = t.n[b];
+  const float inv_n = 1.0f / static_cast<float>(N);
+  float c[kPixDim];
+  float phi = 0.f;
+#pragma unroll
+  for (int k = 0; k < kPixDim; ++k) {
+    c[k] = unfix32<true>(sums[static_cast<int64_t>(t.b_base + b) * kPixDim + k], inv_n);
+    phi = fmaf(c[k], c[k], phi);
+  }
+  const float inv_c = phi > 0.f ? 1.0f / sqrtf(phi) : 0.f;
+  if (u == 0 && threadIdx.x == 0) {
+    stats[t.b_base + b].phi = phi;
+    stats[t.b_base + b].rho_g = 1.0f - phi;
+    stats[t.b_base + b].n_patches = N;
+    stats[t.b_base + b].k_tail = t.ktail[b];
+  }
+  if (i >= N) return;
+  const float4* row = reinterpret_cast<const float4*>(tokens + (static_cast<int64_t>(t.tok0[b]) + i) * kPixDim);
+  const float4 a = row[0], e = row[1];
+  const float v[kPixDim] = {a.x, a.y, a.z, a.w, e.x, e.y, e.z, e.w};
+  float acc = 0.f;
+#pragma unroll
+  for (int k = 0; k < kPixDim; ++k) {
+    const float x = v[k] - c[k] * inv_c;
+    acc = fmaf(x, x, acc);
+  }
+  d_out[t.tok0[b] + i] = sqrtf(acc);
+}
+
+// ------------------------------------------------------------------------------------------------
 // resample
 // ------------------------------------------------------------------------------------------------
 constexpr int kRsThreads = 256;  // threads of a resample CTA
@@ -1339,6 +1575,134 @@ extern "C" pace_status_t pace_apc_density_tokens(const void* T, const int32_t* c
     apc_tok_pass1<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums);
     PACE_CHECK(check_launch());
     apc_tok_pass2<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums, d_out, stats);
+    PACE_CHECK(check_launch());
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
+    apc_tail<<<nb, 1024, tail_smem(at), stream>>>(at, d_out, tp, stats);
+    PACE_CHECK(check_launch());
+  }
+  return PACE_OK;
+}
+
+// ------------------------------------------------------------------------------------------------
+// pixel-statistic previews
+// ------------------------------------------------------------------------------------------------
+namespace pace {
+namespace {
+
+// Strip table of images c0 .. c0 + nb - 1 (as the density passes build it); false if an image
+// is not laid out for 4-byte copies (then the narrow loader is used).
+bool fill_strip_table(ApcTable& t, int c0, int nb, const int64_t* img_off, const int32_t* H, const int32_t* W,
+                      float tail_frac, int& patch0) {
+  bool wide = true;
+  t = ApcTable{};
+  t.nb = nb;
+  t.b_base = c0;
+  t.unit_prefix[0] = 0;
+  for (int i = 0; i < nb; ++i) {
+    const int b = c0 + i;
+    t.off[i] = img_off[b];
+    t.H[i] = H[b];
+    t.W[i] = W[b];
+    t.gw[i] = W[b] / kPatch;
+    t.chunks[i] = (t.gw[i] + kStrip - 1) / kStrip;
+    t.patch0[i] = patch0;
+    const int N = (H[b] / kPatch) * t.gw[i];
+    t.n[i] = N;
+    double kt = std::floor(static_cast<double>(tail_frac) * N + 0.5);
+    if (kt < 1) kt = 1;
+    if (kt > N) kt = N;
+    t.ktail[i] = static_cast<int>(kt);
+    patch0 += N;
+    t.unit_prefix[i + 1] = t.unit_prefix[i] + (H[b] / kPatch) * t.chunks[i];
+    if ((static_cast<int64_t>(W[b]) * 3) % 4 != 0 || (t.gw[i] % 2) != 0 || (img_off[b] % 4) != 0) wide = false;
+  }
+  return wide;
+}
+
+pace_status_t launch_pix_features(const uint8_t* img, const ApcTable& t, bool wide, int feature, float* tokens,
+                                  cudaStream_t stream) {
+  const int units = t.unit_prefix[t.nb];
+  if (wide) apc_pix_features<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, feature, tokens);
+  else apc_pix_features<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, feature, tokens);
+  return check_launch();
+}
+
+int64_t total_patches(int B, const int32_t* H, const int32_t* W) {
+  int64_t n = 0;
+  for (int b = 0; b < B; ++b) n += static_cast<int64_t>(H[b] / kPatch) * (W[b] / kPatch);
+  return n;
+}
+
+}  // namespace
+}  // namespace pace
+
+extern "C" pace_status_t pace_apc_pixel_features(const uint8_t* img, const int64_t* img_off, const int32_t* H,
+                                                 const int32_t* W, int B, int feature, float* tokens,
+                                                 pace_stream_t stream) {
+  PACE_CHECK(check_images(img, img_off, H, W, B));
+  if (B == 0) return PACE_OK;
+  if (feature < kFeatRgb || feature > kFeatLaplacian || tokens == nullptr || reinterpret_cast<uintptr_t>(tokens) % 16)
+    return PACE_ERR_INVALID_ARG;
+  PACE_CHECK(check_device());
+  int patch0 = 0;
+  for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
+    ApcTable t;
+    const bool wide = fill_strip_table(t, c0, std::min(kApcMaxB, B - c0), img_off, H, W, 0.1f, patch0);
+    PACE_CHECK(launch_pix_features(img, t, wide, feature, tokens, stream));
+  }
+  return PACE_OK;
+}
+
+extern "C" size_t pace_apc_density_pixel_workspace_size(int B, const int32_t* H, const int32_t* W) {
+  if (B <= 0 || H == nullptr || W == nullptr) return 0;
+  for (int b = 0; b < B; ++b)
+    if (H[b] < kPatch || W[b] < kPatch) return 0;
+  return align_up(static_cast<size_t>(total_patches(B, H, W)) * kPixDim * sizeof(float), 256) +
+         align_up(static_cast<size_t>(B) * kPixDim * sizeof(unsigned long long), 256);
+}
+
+extern "C" pace_status_t pace_apc_density_pixel(const uint8_t* img, const int64_t* img_off, const int32_t* H,
+                                                const int32_t* W, int B, int feature, const pace_apc_params* params,
+                                                float* d_out, pace_apc_stats* stats, void* ws, size_t ws_bytes,
+                                                pace_stream_t stream) {
+  PACE_CHECK(check_images(img, img_off, H, W, B));
+  if (B == 0) return PACE_OK;
+  if (feature < kFeatRgb || feature > kFeatLaplacian || d_out == nullptr || stats == nullptr)
+    return PACE_ERR_INVALID_ARG;
+  pace_apc_params p;
+  if (params) p = *params; else pace_apc_params_default(&p);
+  if (!(p.tail_frac > 0.f && p.tail_frac <= 1.f) || !(p.gamma > 0.f) || !(p.alpha >= 0.f && p.alpha <= 1.f) ||
+      !(p.r_min <= p.r_max) || p.align < 1)
+    return PACE_ERR_INVALID_ARG;
+  const size_t tok_bytes = align_up(static_cast<size_t>(total_patches(B, H, W)) * kPixDim * sizeof(float), 256);
+  if (ws == nullptr || ws_bytes < pace_apc_density_pixel_workspace_size(B, H, W) ||
+      reinterpret_cast<uintptr_t>(ws) % 16)
+    return PACE_ERR_WORKSPACE;
+  PACE_CHECK(check_device());
+  PACE_CHECK(tail_smem_attr());
+  auto* tokens = static_cast<float*>(ws);
+  auto* sums = reinterpret_cast<unsigned long long*>(static_cast<uint8_t*>(ws) + tok_bytes);
+  PACE_CUDA(cudaMemsetAsync(sums, 0, static_cast<size_t>(B) * kPixDim * sizeof(unsigned long long), stream));
+  int patch0 = 0;
+  for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
+    const int nb = std::min(kApcMaxB, B - c0);
+    ApcTable at;
+    const bool wide = fill_strip_table(at, c0, nb, img_off, H, W, p.tail_frac, patch0);
+    PACE_CHECK(launch_pix_features(img, at, wide, feature, tokens, stream));
+    PixTable pt{};
+    pt.nb = nb;
+    pt.b_base = c0;
+    pt.unit_prefix[0] = 0;
+    for (int i = 0; i < nb; ++i) {
+      pt.tok0[i] = at.patch0[i];
+      pt.n[i] = at.n[i];
+      pt.ktail[i] = at.ktail[i];
+      pt.unit_prefix[i + 1] = pt.unit_prefix[i] + (at.n[i] + kApcThreads - 1) / kApcThreads;
+    }
+    const int units = pt.unit_prefix[nb];
+    apc_pix_pass1<<<units, kApcThreads, 0, stream>>>(pt, tokens, sums);
+    PACE_CHECK(check_launch());
+    apc_pix_pass2<<<units, kApcThreads, 0, stream>>>(pt, tokens, sums, d_out, stats);
     PACE_CHECK(check_launch());
     TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
     apc_tail<<<nb, 1024, tail_smem(at), stream>>>(at, d_out, tp, stats);

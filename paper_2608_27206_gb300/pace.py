@@ -41,6 +41,9 @@ class DdaeParams(ctypes.Structure):
 
 # fusion modes of DdaeParams (pace_ddae_fusion)
 DDAE_ADAPTIVE, DDAE_ONLY_LLM, DDAE_ONLY_VIT, DDAE_FIXED = 0, 1, 2, 3
+FEATURE_RGB_STATS, FEATURE_COLOR_ENTROPY, FEATURE_EDGE_DENSITY, FEATURE_LAPLACIAN = 0, 1, 2, 3
+PIXEL_FEATURES = {"rgb_stats": 0, "color_entropy": 1, "edge_density": 2, "laplacian": 3}
+PIXEL_FEATURE_DIM = 8   # floats per feature token (zero-padded)
 QUERY_VISION_TEXT, QUERY_TEXT, QUERY_LAST = 0, 1, 2
 QUERY_SETS = {"vision_text": QUERY_VISION_TEXT, "text": QUERY_TEXT, "last": QUERY_LAST}
 
@@ -75,6 +78,10 @@ _SIGS = {
                                                ctypes.POINTER(ApcParams), _P, _P, _P, ctypes.c_size_t, _P]),
     "pace_apc_density": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, ctypes.c_int, ctypes.POINTER(ApcParams), _P, _P,
                                         _P, ctypes.c_size_t, _P]),
+    "pace_apc_pixel_features": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, ctypes.c_int, ctypes.c_int, _P, _P]),
+    "pace_apc_density_pixel_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, _I32P]),
+    "pace_apc_density_pixel": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, ctypes.c_int, ctypes.c_int,
+                                              ctypes.POINTER(ApcParams), _P, _P, _P, ctypes.c_size_t, _P]),
     "pace_apc_density_static": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, ctypes.c_int, ctypes.POINTER(ApcParams),
                                                _P, _P, _P]),
     "pace_apc_resample": (ctypes.c_int, [_P, _I64P, _I32P, _I32P, _P, _P, _I64P, ctypes.c_int, _P]),
@@ -238,6 +245,50 @@ def pace_apc_density(img: torch.Tensor, img_off, H, W, params: Optional[ApcParam
                                 ctypes.byref(params) if params is not None else None, _dev(d_out), _dev(stats),
                                 _dev(ws), ws.numel() * ws.element_size(), _stream(stream))
     _check("pace_apc_density", st)
+    return d_out[:n], stats[:B]
+
+
+def _feature(feature) -> int:
+    return PIXEL_FEATURES[feature] if isinstance(feature, str) else int(feature)
+
+
+def pace_apc_pixel_features(img: torch.Tensor, img_off, H, W, feature, out: Optional[torch.Tensor] = None,
+                            stream=None) -> torch.Tensor:
+    """Pixel-statistic feature tokens float32 [sum N, 8] of B packed uint8 images; feature is
+    "rgb_stats", "color_entropy", "edge_density", "laplacian" or a FEATURE_* code."""
+    off, h, w = _i64(img_off), _i32(H), _i32(W)
+    B = len(h)
+    n = int(((h // 14).astype(np.int64) * (w // 14)).sum())
+    if out is None:
+        out = torch.empty((max(n, 1), PIXEL_FEATURE_DIM), dtype=torch.float32, device=img.device)
+    st = lib().pace_apc_pixel_features(_dev(img), _pi64(off), _pi32(h), _pi32(w), B, _feature(feature), _dev(out),
+                                       _stream(stream))
+    _check("pace_apc_pixel_features", st)
+    return out[:n]
+
+
+def pace_apc_density_pixel_workspace_size(H, W) -> int:
+    h, w = _i32(H), _i32(W)
+    return int(lib().pace_apc_density_pixel_workspace_size(len(h), _pi32(h), _pi32(w)))
+
+
+def pace_apc_density_pixel(img: torch.Tensor, img_off, H, W, feature, params: Optional[ApcParams] = None,
+                           d_out: Optional[torch.Tensor] = None, stats: Optional[torch.Tensor] = None,
+                           ws: Optional[torch.Tensor] = None, stream=None):
+    """APC density with a pixel-statistic preview.  Returns (d [sum N], stats [B, 10])."""
+    off, h, w = _i64(img_off), _i32(H), _i32(W)
+    B = len(h)
+    n = int(((h // 14).astype(np.int64) * (w // 14)).sum())
+    dev = img.device
+    if d_out is None:
+        d_out = torch.empty(max(n, 1), dtype=torch.float32, device=dev)
+    if stats is None:
+        stats = torch.zeros((max(B, 1), 10), dtype=torch.int32, device=dev)
+    ws = _workspace(pace_apc_density_pixel_workspace_size(h, w), ws, dev)
+    st = lib().pace_apc_density_pixel(_dev(img), _pi64(off), _pi32(h), _pi32(w), B, _feature(feature),
+                                      ctypes.byref(params) if params is not None else None, _dev(d_out), _dev(stats),
+                                      _dev(ws), ws.numel() * ws.element_size(), _stream(stream))
+    _check("pace_apc_density_pixel", st)
     return d_out[:n], stats[:B]
 
 

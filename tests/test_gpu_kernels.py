@@ -168,6 +168,44 @@ def test_density_tokens_params_and_rejects(pace):
         pace.pace_apc_density_tokens(Tt, [0, 10, 10], [28, 28], [28, 28])   # an image without tokens
 
 
+@pytest.mark.parametrize("feature", ["rgb_stats", "color_entropy", "edge_density", "laplacian"])
+def test_pixel_features_and_density(pace, feature):
+    """Pixel-statistic previews: the feature tokens, then Eq. 1-6 on them, against the oracle."""
+    rng = np.random.default_rng(17)
+    imgs = [synth.make_image(rng, h, w, 3, 2, f) for h, w, f in [(448, 448, 0.3), (70, 462, 0.6), (1008, 28, 0.1)]]
+    imgs.append(np.full((56, 84, 3), 200, np.uint8))                         # a constant image
+    buf, off = synth.pack_images(imgs)
+    H = [im.shape[0] for im in imgs]
+    W = [im.shape[1] for im in imgs]
+    img_t = torch.from_numpy(buf).cuda()
+    tok = pace.pace_apc_pixel_features(img_t, off, H, W, feature).cpu().numpy()
+    d, st = pace.pace_apc_density_pixel(img_t, off, H, W, feature)
+    d, st = d.cpu().numpy(), pace.stats_dict(st)
+    p0 = 0
+    dim = O.FEATURE_DIMS[feature]
+    for im, s in zip(imgs, st):
+        ref_tok = O.pixel_statistic_tokens(im, feature)
+        n = ref_tok.shape[0]
+        # integer-derived statistics: fp32 rounding only; the padding stays zero
+        np.testing.assert_allclose(tok[p0:p0 + n, :dim], ref_tok, rtol=2e-6, atol=2e-6, err_msg=feature)
+        assert not tok[p0:p0 + n, dim:].any()
+        ref = O.apc_density_pixel(im, feature)
+        assert s["n_patches"] == n and s["k_tail"] == ref["k_tail"]
+        assert_scores_close(d[p0:p0 + n], ref["d"], atol_frac=2e-3, atol=1e-5, what=f"d_i ({feature})")
+        for k in ("phi", "d_top", "rho_d", "r"):
+            assert abs(s[k] - ref[k]) <= 2e-3 * max(abs(ref[k]), 1e-3), (feature, k, s[k], ref[k])
+        p0 += n
+    _no_device_error(pace)
+
+
+def test_pixel_features_rejects(pace):
+    img = torch.zeros(28 * 28 * 3, dtype=torch.uint8, device="cuda")
+    with pytest.raises(pace.PaceError):
+        pace.pace_apc_pixel_features(img, [0], [28], [28], 4)          # unknown feature
+    with pytest.raises(pace.PaceError):
+        pace.pace_apc_density_pixel(img, [0], [28], [30], "laplacian")   # not a multiple of 14
+
+
 def test_density_constant_images(pace):
     imgs = [np.full((112, 168, 3), v, dtype=np.uint8) for v in (0, 77, 255)]
     d, st = _density(pace, imgs)
