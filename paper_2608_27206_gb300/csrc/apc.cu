@@ -369,12 +369,17 @@ constexpr int kTokMaxD = 4096;   // longest token accepted (c_hat is staged in s
 struct TokTable {
   int64_t tok0[kApcMaxB];        // first token of image b
   int n[kApcMaxB];               // tokens of image b
-  int unit_prefix[kApcMaxB + 1]; // chunks of kTokChunk tokens
+  int unit_prefix[kApcMaxB + 1]; // chunks of kTokChunk tokens (pass 2)
+  int unit_prefix1[kApcMaxB + 1]; // chunks of rows1 tokens (pass 1)
   int ktail[kApcMaxB];
   int nb;
   int b_base;
   int D;
+  int rows1;                     // tokens per pass-1 chunk (a chunk fits a 40 KB stage)
 };
+
+constexpr int kTok1StageBytes = 40960;   // one pass-1 stage: rows1 token rows
+constexpr int kTok1MaxSlots = kTokMaxD / 2 / kApcThreads;   // column pairs per thread (8)
 
 __device__ __forceinline__ int find_tok_image(const TokTable& t, int unit) {
   int b = 0;
@@ -385,47 +390,104 @@ __device__ __forceinline__ int find_tok_image(const TokTable& t, int unit) {
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
-// Pass 1: 1/|T_i| per token (warp per token) and the chunk's column sums of t_hat = T_i / |T_i|,
-// added to the image's D-vector as signed 2^-32 fixed point (exact, order-independent).
+// Pass 1: 1/|T_i| per token (warp per token) and the column sums of t_hat = T_i / |T_i|, as
+// signed 2^-32 fixed point (exact, order-independent).  A grid of resident CTAs walks chunks of
+// rows1 tokens; each chunk is staged in shared memory with cp.async while the previous one is
+// worked on, so T is read once.  Per-chunk sums are rounded and added in registers; one atomic
+// per column when the CTA moves to another image or ends.
+__device__ __forceinline__ void tok_issue_chunk(const uint32_t* __restrict__ T, const TokTable& t, int unit,
+                                                uint32_t* dst) {
+  int b = 0;
+  while (b + 1 < t.nb && t.unit_prefix1[b + 1] <= unit) ++b;
+  const int r0 = (unit - t.unit_prefix1[b]) * t.rows1;
+  const int nt = min(t.rows1, t.n[b] - r0);
+  const int words = t.D >> 1;
+  const uint32_t* src = T + (t.tok0[b] + r0) * words;
+  for (int i = threadIdx.x; i < nt * words; i += kApcThreads) cp_async4(dst + i, src + i);
+  cp_async_commit();
+}
+
 __global__ void __launch_bounds__(kApcThreads) apc_tok_pass1(const uint32_t* __restrict__ T,
-                                                             const __grid_constant__ TokTable t,
+                                                             const __grid_constant__ TokTable t, int units,
                                                              float* __restrict__ inv_norm,
                                                              unsigned long long* __restrict__ sums) {
-  __shared__ float inv[kTokChunk];
-  const int unit = blockIdx.x;
-  const int b = find_tok_image(t, unit);
-  const int c0 = (unit - t.unit_prefix[b]) * kTokChunk;
-  const int nt = min(kTokChunk, t.n[b] - c0);
+  extern __shared__ __align__(16) uint32_t tok_smem[];   // two stages of rows1 x words
+  __shared__ float inv[2][32];
+  int unit = blockIdx.x;
+  if (unit >= units) return;
   const int words = t.D >> 1;   // bf16 pairs per token
-  const uint32_t* base = T + (t.tok0[b] + c0) * words;
+  const int stage = t.rows1 * words;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int p = warp; p < nt; p += kApcThreads / 32) {
-    const uint32_t* row = base + static_cast<int64_t>(p) * words;
-    float ss = 0.f;
-    for (int w = lane; w < words; w += 32) {
-      const uint32_t v = row[w];
-      const float lo = bf16_lo(v), hi = bf16_hi(v);
-      ss = fmaf(lo, lo, fmaf(hi, hi, ss));
+  unsigned long long acc[kTok1MaxSlots][2];
+#pragma unroll
+  for (int q = 0; q < kTok1MaxSlots; ++q) acc[q][0] = acc[q][1] = 0ull;
+  int cur_b = -1;
+  auto flush = [&]() {
+    if (cur_b < 0) return;
+    unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + cur_b) * t.D;
+#pragma unroll
+    for (int q = 0; q < kTok1MaxSlots; ++q) {
+      const int w = threadIdx.x + q * kApcThreads;
+      if (w < words) {
+        atomicAdd(sb + 2 * w, acc[q][0]);
+        atomicAdd(sb + 2 * w + 1, acc[q][1]);
+      }
+      acc[q][0] = acc[q][1] = 0ull;
     }
-    ss = warp_sum_f(ss);
-    if (lane == 0) {
-      const float iv = ss > 0.f ? 1.0f / sqrtf(ss) : 0.f;
-      inv[p] = iv;
-      inv_norm[t.tok0[b] + c0 + p] = iv;
+  };
+  tok_issue_chunk(T, t, unit, tok_smem);
+  for (int i = 0; unit < units; ++i, unit += gridDim.x) {
+    const int next = unit + static_cast<int>(gridDim.x);
+    if (next < units) {
+      tok_issue_chunk(T, t, next, tok_smem + ((i + 1) & 1) * stage);
+      cp_async_wait_group<1>();
+    } else {
+      cp_async_wait_group<0>();
     }
+    __syncthreads();
+    int b = 0;
+    while (b + 1 < t.nb && t.unit_prefix1[b + 1] <= unit) ++b;
+    const int r0 = (unit - t.unit_prefix1[b]) * t.rows1;
+    const int nt = min(t.rows1, t.n[b] - r0);
+    if (b != cur_b) {
+      flush();
+      cur_b = b;
+    }
+    const uint32_t* rows = tok_smem + (i & 1) * stage;
+    float* iv_s = inv[i & 1];
+    for (int p = warp; p < nt; p += kApcThreads / 32) {
+      const uint32_t* row = rows + p * words;
+      float ss = 0.f;
+      for (int w = lane; w < words; w += 32) {
+        const uint32_t v = row[w];
+        const float lo = bf16_lo(v), hi = bf16_hi(v);
+        ss = fmaf(lo, lo, fmaf(hi, hi, ss));
+      }
+      ss = warp_sum_f(ss);
+      if (lane == 0) {
+        const float iv = ss > 0.f ? 1.0f / sqrtf(ss) : 0.f;
+        iv_s[p] = iv;
+        inv_norm[t.tok0[b] + r0 + p] = iv;
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < kTok1MaxSlots; ++q) {
+      const int w = threadIdx.x + q * kApcThreads;
+      if (w < words) {
+        float2 a = make_float2(0.f, 0.f);
+        for (int p = 0; p < nt; ++p) {
+          const uint32_t v = rows[p * words + w];
+          const float iv = iv_s[p];
+          a = ptx::ffma2(make_float2(iv, iv), make_float2(bf16_lo(v), bf16_hi(v)), a);
+        }
+        acc[q][0] += fix32_signed(a.x);
+        acc[q][1] += fix32_signed(a.y);
+      }
+    }
+    __syncthreads();   // this stage is refilled two chunks on
   }
-  __syncthreads();
-  unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + b) * t.D;
-  for (int w = threadIdx.x; w < words; w += kApcThreads) {
-    float a0 = 0.f, a1 = 0.f;
-    for (int p = 0; p < nt; ++p) {   // the chunk's rows were just read: L1 hits
-      const uint32_t v = base[static_cast<int64_t>(p) * words + w];
-      a0 = fmaf(inv[p], bf16_lo(v), a0);
-      a1 = fmaf(inv[p], bf16_hi(v), a1);
-    }
-    atomicAdd(sb + 2 * w, fix32_signed(a0));
-    atomicAdd(sb + 2 * w + 1, fix32_signed(a1));
-  }
+  flush();
 }
 
 // Pass 2: c = sums / N, phi = |c|^2, c_hat = c / |c|, then d_i = |t_hat_i - c_hat| directly
@@ -1504,6 +1566,34 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
 // ------------------------------------------------------------------------------------------------
 namespace pace {
 namespace {
+// Opts pass 1 of the token density into two 40 KB stages (once per device).
+pace_status_t tok_pass1_attr() {
+  static std::atomic<uint64_t> done{0};
+  int dev = 0;
+  PACE_CUDA(cudaGetDevice(&dev));
+  const uint64_t bit = uint64_t{1} << (dev & 63);
+  if (done.load(std::memory_order_acquire) & bit) return PACE_OK;
+  PACE_CUDA(cudaFuncSetAttribute(apc_tok_pass1, cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kTok1StageBytes));
+  done.fetch_or(bit, std::memory_order_acq_rel);
+  return PACE_OK;
+}
+
+// Grid of pass 1: the CTAs resident at once (capped by the chunks).
+unsigned tok_pass1_grid(int units) {
+  static std::atomic<int> cap[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) dev = 0;
+  int c = cap[dev & 63].load(std::memory_order_relaxed);
+  if (c == 0) {
+    int nsm = 0, per = 0;
+    cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, apc_tok_pass1, kApcThreads, 2 * kTok1StageBytes);
+    c = std::max(1, nsm * std::max(per, 1));
+    cap[dev & 63].store(c, std::memory_order_relaxed);
+  }
+  return static_cast<unsigned>(std::max(1, std::min(units, c)));
+}
+
 struct TokLayout {
   size_t sums_off, inv_off, total;
 };
@@ -1556,7 +1646,9 @@ extern "C" pace_status_t pace_apc_density_tokens(const void* T, const int32_t* c
     tt.nb = at.nb = nb;
     tt.b_base = at.b_base = c0;
     tt.D = D;
+    tt.rows1 = std::max(1, std::min(32, kTok1StageBytes / (D * 2)));
     tt.unit_prefix[0] = 0;
+    tt.unit_prefix1[0] = 0;
     for (int i = 0; i < nb; ++i) {
       const int b = c0 + i;
       const int N = cu_tokens[b + 1] - cu_tokens[b];
@@ -1567,12 +1659,16 @@ extern "C" pace_status_t pace_apc_density_tokens(const void* T, const int32_t* c
       if (kt > N) kt = N;
       tt.ktail[i] = at.ktail[i] = static_cast<int>(kt);
       tt.unit_prefix[i + 1] = tt.unit_prefix[i] + (N + kTokChunk - 1) / kTokChunk;
+      tt.unit_prefix1[i + 1] = tt.unit_prefix1[i] + (N + tt.rows1 - 1) / tt.rows1;
       at.H[i] = H[b];
       at.W[i] = W[b];
       at.patch0[i] = cu_tokens[b];
     }
     const int units = tt.unit_prefix[nb];
-    apc_tok_pass1<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums);
+    const int units1 = tt.unit_prefix1[nb];
+    const size_t smem1 = 2 * static_cast<size_t>(tt.rows1) * D * 2;
+    PACE_CHECK(tok_pass1_attr());
+    apc_tok_pass1<<<tok_pass1_grid(units1), kApcThreads, smem1, stream>>>(T32, tt, units1, inv, sums);
     PACE_CHECK(check_launch());
     apc_tok_pass2<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums, d_out, stats);
     PACE_CHECK(check_launch());
