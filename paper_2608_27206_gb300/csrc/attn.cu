@@ -63,7 +63,6 @@ constexpr int kAttnMaxB = 64;
 constexpr uint32_t kTmemCols = 512;
 constexpr float kShiftMargin = 90.f;      // pass 1: fixed shift = first chunk maximum + this (base 2)
 constexpr int kNoMask = 1 << 29;          // diag of a non-causal image: every key is seen
-constexpr int kTargetItems = 152;         // work items (two CTAs each): two waves over the SMs
 
 // An operand tile of ROWS rows and head dimension D is stored as NB blocks of 64 columns
 // (ROWS x 128 bytes, 128-byte swizzle) followed by R slices of 16 columns (ROWS x 32 bytes,
@@ -812,7 +811,13 @@ struct AttnLayout {
   size_t L_off, part_off, ml_off, total;
 };
 
-// Key splits of pass 1: enough work items to cover the GPU about twice.
+// Key splits of pass 1.  A CTA costs about kSplitOverheadTiles streamed tiles of start-up and
+// drain on top of its key tiles, and CTAs run in rounds of kPlanSms (one per SM), so the split
+// count that minimises rounds x (tiles per CTA + overhead) is taken (the smallest on ties).  The
+// GB300's SM count is a planning constant here, so that the workspace size queries need no device.
+constexpr int kPlanSms = 152;
+constexpr double kSplitOverheadTiles = 4.4;
+
 int choose_splits(const std::vector<Seg>& segs, int H) {
   int64_t items = 0;
   int max_kt = 1;
@@ -820,10 +825,18 @@ int choose_splits(const std::vector<Seg>& segs, int H) {
     items += static_cast<int64_t>(H) * ((sg.nq + kPair - 1) / kPair);
     max_kt = std::max(max_kt, (sg.nk + kStream - 1) / kStream);
   }
-  if (items >= kTargetItems || items == 0) return 1;
-  int s = static_cast<int>((kTargetItems + items - 1) / items);
-  s = std::min(s, std::min(max_kt, 32));
-  return std::max(s, 1);
+  if (items == 0) return 1;
+  int best = 1;
+  double best_cost = 0.0;
+  for (int s = 1; s <= std::min(max_kt, 32); ++s) {
+    const int64_t rounds = (2 * items * s + kPlanSms - 1) / kPlanSms;
+    const double cost = static_cast<double>(rounds) * ((max_kt + s - 1) / s + kSplitOverheadTiles);
+    if (s == 1 || cost < best_cost) {
+      best = s;
+      best_cost = cost;
+    }
+  }
+  return best;
 }
 
 AttnLayout attn_layout(const std::vector<Seg>& segs, int H, int groups) {
