@@ -8,6 +8,7 @@
 // ballots, the lower index winning among equal scores.
 //
 // pace_gather: one warp per kept row, 16-byte vector loads and stores.
+#include <algorithm>
 #include <atomic>
 #include <cfloat>
 #include <cmath>
@@ -214,35 +215,39 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
   }
 }
 
-// One warp per row; 16-byte vectors.
+// One warp per 2 KB piece of a row (128 16-byte vectors, 4 per lane, all in flight), so that a
+// few thousand short rows still spread over every SM.
+constexpr int kGatherU = 4;
+constexpr int kGatherPiece = 32 * kGatherU;   // vectors per warp-piece
+
 __global__ void __launch_bounds__(256) gather_rows_v16(const uint4* __restrict__ src, int64_t n_src,
                                                        int64_t row_vec, const int32_t* __restrict__ idx,
                                                        int64_t n_idx, uint4* __restrict__ dst, int* status) {
   const int lane = threadIdx.x & 31;
   const int64_t warp0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
-  constexpr int U = 16;
-  for (int64_t r = warp0; r < n_idx; r += nwarps) {
+  const int64_t pieces = (row_vec + kGatherPiece - 1) / kGatherPiece;
+  for (int64_t w = warp0; w < n_idx * pieces; w += nwarps) {
+    const int64_t r = w / pieces;
+    const int64_t c0 = (w - r * pieces) * kGatherPiece;
     const int64_t s = idx[r];
     uint4* dp = dst + r * row_vec;
     if (s < 0 || s >= n_src) {
-      for (int64_t c = lane; c < row_vec; c += 32) dp[c] = make_uint4(0u, 0u, 0u, 0u);
-      if (lane == 0) record_error(status, PACE_ERR_INVALID_ARG, K_GATHER);
+      for (int64_t c = c0 + lane; c < min(row_vec, c0 + kGatherPiece); c += 32) dp[c] = make_uint4(0u, 0u, 0u, 0u);
+      if (lane == 0 && c0 == 0) record_error(status, PACE_ERR_INVALID_ARG, K_GATHER);
       continue;
     }
     const uint4* sp = src + s * row_vec;
-    for (int64_t c0 = 0; c0 < row_vec; c0 += 32 * U) {
-      uint4 v[U];
+    uint4 v[kGatherU];
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int64_t c = c0 + u * 32 + lane;
-        if (c < row_vec) v[u] = __ldcs(sp + c);
-      }
+    for (int u = 0; u < kGatherU; ++u) {
+      const int64_t c = c0 + u * 32 + lane;
+      if (c < row_vec) v[u] = __ldcs(sp + c);
+    }
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int64_t c = c0 + u * 32 + lane;
-        if (c < row_vec) __stcs(dp + c, v[u]);
-      }
+    for (int u = 0; u < kGatherU; ++u) {
+      const int64_t c = c0 + u * 32 + lane;
+      if (c < row_vec) __stcs(dp + c, v[u]);
     }
   }
 }
@@ -431,6 +436,8 @@ extern "C" pace_status_t pace_gather(const void* src, int64_t n_src_rows, int64_
   const bool vec = (row_bytes % 16 == 0) && (reinterpret_cast<uintptr_t>(src) % 16 == 0) &&
                    (reinterpret_cast<uintptr_t>(dst) % 16 == 0);
   if (vec) {
+    const int64_t pieces = (row_bytes / 16 + kGatherPiece - 1) / kGatherPiece;
+    blocks = std::min<int64_t>((n_idx * pieces + warps_per_block - 1) / warps_per_block, static_cast<int64_t>(sms) * 8);
     gather_rows_v16<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
         static_cast<const uint4*>(src), n_src_rows, row_bytes / 16, idx, n_idx, static_cast<uint4*>(dst), status);
   } else {
