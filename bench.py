@@ -509,7 +509,7 @@ def run_gpu(args):
         llm_tf = cnt["llm_flops"] / (mean["llm"] * 1e-3) / 1e12
         other["llm"] = {"bound": "tensor", "us": round(mean["llm"] * 1e3, 2), "achieved": round(llm_tf, 1),
                         "peak": peak, "unit": "TFLOP/s", "frac": round(llm_tf / peak, 4), "flops": cnt["llm_flops"]}
-        nxt = measure_next_rows(P, device, flush, peak, hbm) if world == 1 else None
+        nxt = measure_next_rows(P, device, flush, peak, hbm) if world == 1 and not args.no_next_rows else None
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
             tot, parts, sample = oracle_sample(wl, KEEP, vit_rows=args.ref_vit_rows)
@@ -586,6 +586,7 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--ref-vit-rows", type=int, default=2048)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-next-rows", action="store_true", help="skip the timing of the NEXT-row calls")
     ap.add_argument("--profile", choices=("density", "resample", "vit", "llm", "select", "gather"),
                     help="run only this call --reps times (for profiler captures)")
     ap.add_argument("--reps", type=int, default=1)
