@@ -268,6 +268,24 @@ PACE_API pace_status_t pace_vit_attn_importance(const void* Q, const void* K, co
                                        int n_heads, int head_dim, float scale, int merge, float* s_vis_raw,
                                        void* ws, size_t ws_bytes, pace_stream_t stream);
 
+/*
+ * pace_vit_attn_importance with the row log-sum-exp pass split by query rows, so that it can
+ * start while Q is still being copied in: the pass-1 work whose query rows all lie below
+ * chunk_end_rows[c] (and whose last row is not below chunk_end_rows[c - 1]) is launched after
+ * the stream waits for the CUDA event chunk_ready[c].  Results are bit-identical to
+ * pace_vit_attn_importance.  K must be complete when chunk_ready[0] fires.
+ *
+ *  n_chunks        1 .. 64
+ *  chunk_end_rows  host  int64 [n_chunks], nondecreasing global Q rows, the last = cu_seqlens[B]
+ *  chunk_ready     host  cudaEvent_t [n_chunks] (passed as void*), recorded by the caller
+ *  other arguments as for pace_vit_attn_importance
+ */
+PACE_API pace_status_t pace_vit_attn_importance_chunked(const void* Q, const void* K, const int32_t* cu_seqlens,
+                                               int B, int n_heads, int head_dim, float scale, int merge,
+                                               float* s_vis_raw, void* ws, size_t ws_bytes, int n_chunks,
+                                               const int64_t* chunk_end_rows, void* const* chunk_ready,
+                                               pace_stream_t stream);
+
 /* Scratch bytes for pace_llm_text_visual_importance (host cu_q, cu_k [B+1]). */
 PACE_API size_t pace_llm_text_visual_importance_workspace_size(int B, const int32_t* cu_q, const int32_t* cu_k,
                                                       int n_q_heads, int n_kv_heads);

@@ -126,6 +126,7 @@ struct AttnTable {
   int diag[kAttnMaxB];                // causal mask: local key k is seen by local query i iff k <= i + diag
   int out0[kAttnMaxB];                // first part-map row of image b (pass 2)
   int lpad[kAttnMaxB];                // first padded L row of image b (multiple of 256)
+  int pair_lo[kAttnMaxB], pair_n[kAttnMaxB];   // pass 1: the query pairs this launch takes
   int item_prefix[kAttnMaxB + 1];
   int nb;
   int H;        // query heads
@@ -382,10 +383,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
   int r = item - t.item_prefix[b];
   const int split = r % t.splits;
   r /= t.splits;
-  const int npair = (t.nq[b] + kPair - 1) / kPair;
+  const int npair = t.pair_n[b];
   const int diag = t.diag[b];
   // causal images: the last query rows see the most keys, so they are scheduled first
-  const int pair = CAUSAL ? npair - 1 - r % npair : r % npair;
+  const int pair = t.pair_lo[b] + (CAUSAL ? npair - 1 - r % npair : r % npair);
   const int h = r / npair;
   const int g = h / t.G;
   const int qrow0 = pair * kPair + kTile * static_cast<int>(rank);     // this CTA's first local query row
@@ -505,7 +506,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         if (round == 0) lse_fixed(sv, valid - 64, c, m_run, l_run);
         else if (valid > 64) lse_update64(sv, valid - 64, c, m_run, l_run);
       }
-      if (!(l_run < INFINITY)) ctl->redo = 1;   // inf or NaN: this row needs the exact round
+      // inf or NaN in a row of the image: it needs the exact round (rows past the image are
+      // ignored, so whatever their Q rows hold cannot change the valid rows' results)
+      if (!(l_run < INFINITY) && qrow0 + rr < t.nq[b]) ctl->redo = 1;
       // merge the four warpgroups' (m, l) of each row
       if (e > 0) {
         ctl->xchg[e - 1][0][rr] = m_run;
@@ -921,10 +924,18 @@ pace_status_t launch_pairs(void (*kernel)(Params...), int items, size_t smem, cu
   return check_launch();
 }
 
+// Pass 1 in pieces: piece c waits for event ready[c] and takes the query pairs whose last row
+// (a global row of Q) is below end_row[c] (and not below end_row[c - 1]).
+struct QueryChunks {
+  int n = 0;
+  const int64_t* end_row = nullptr;
+  cudaEvent_t const* ready = nullptr;
+};
+
 template <int D, bool CAUSAL>
 pace_status_t run_importance(const void* Q, const void* K, int64_t qrows, int64_t krows,
                              const std::vector<Seg>& segs, int Hq, int Hkv, float scale, int merge, float* out,
-                             void* ws, cudaStream_t stream) {
+                             void* ws, cudaStream_t stream, const QueryChunks& chunks = QueryChunks{}) {
   const int B = static_cast<int>(segs.size());
   const int G = Hq / Hkv;
   const AttnLayout Lay = attn_layout(segs, Hq, Hkv);
@@ -973,7 +984,30 @@ pace_status_t run_importance(const void* Q, const void* K, int64_t qrows, int64_
       t.item_prefix[i + 1] = items1;
       ctiles += (sg.nq + kPair - 1) / kPair * 2;
     }
-    PACE_CHECK(launch_pairs(attn_row_lse<D, CAUSAL>, items1, s1, stream, mq, mq32, mk, mk32, t, c, Lw, ml, status));
+    const int pieces = chunks.n > 0 ? chunks.n : 1;
+    for (int pc = 0; pc < pieces; ++pc) {
+      int items_pc = 0;
+      t.item_prefix[0] = 0;
+      for (int i = 0; i < nb; ++i) {
+        const Seg& sg = segs[c0 + i];
+        const int npair = (sg.nq + kPair - 1) / kPair;
+        int lo = 0, hi = npair;
+        if (chunks.n > 0) {   // pairs whose last row falls in [end_row[pc - 1], end_row[pc])
+          auto last_row = [&](int pr) { return static_cast<int64_t>(sg.q0) + std::min((pr + 1) * kPair, sg.nq) - 1; };
+          const int64_t from = pc > 0 ? chunks.end_row[pc - 1] : INT64_MIN, to = chunks.end_row[pc];
+          while (lo < npair && last_row(lo) < from) ++lo;
+          hi = lo;
+          while (hi < npair && last_row(hi) < to) ++hi;
+        }
+        t.pair_lo[i] = lo;
+        t.pair_n[i] = hi - lo;
+        items_pc += Hq * (hi - lo) * Lay.splits;
+        t.item_prefix[i + 1] = items_pc;
+      }
+      if (chunks.n > 0) PACE_CUDA(cudaStreamWaitEvent(stream, chunks.ready[pc], 0));
+      PACE_CHECK(launch_pairs(attn_row_lse<D, CAUSAL>, items_pc, s1, stream, mq, mq32, mk, mk32, t, c, Lw, ml, status));
+    }
+    (void)items1;
     if (Lay.splits > 1 && ctiles > 0) {
       attn_lse_combine<<<dim3(ctiles, Hq), kTile, 0, stream>>>(t, c, ml, Lw);
       PACE_CHECK(check_launch());
@@ -1012,20 +1046,20 @@ pace_status_t check_heads(int Hq, int Hkv, int D, float scale, const void* Q, co
 template <bool CAUSAL>
 pace_status_t dispatch(const void* Q, const void* K, int64_t qrows, int64_t krows, const std::vector<Seg>& segs,
                        int Hq, int Hkv, int D, float scale, int merge, float* out, void* ws, size_t ws_bytes,
-                       cudaStream_t stream) {
+                       cudaStream_t stream, const QueryChunks& chunks = QueryChunks{}) {
   const AttnLayout Lay = attn_layout(segs, Hq, Hkv);
   if (ws == nullptr || ws_bytes < Lay.total || reinterpret_cast<uintptr_t>(ws) % 16) return PACE_ERR_WORKSPACE;
   PACE_CHECK(check_device());
   switch (D) {
-    case 64: return run_importance<64, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream);
-    case 80: return run_importance<80, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream);
-    default: return run_importance<128, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream);
+    case 64: return run_importance<64, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream, chunks);
+    case 80: return run_importance<80, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream, chunks);
+    default: return run_importance<128, CAUSAL>(Q, K, qrows, krows, segs, Hq, Hkv, scale, merge, out, ws, stream, chunks);
   }
 }
 
 pace_status_t importance(const void* Q, const void* K, const int32_t* cu_q, const int32_t* cu_k, int B, int Hq,
                          int Hkv, int D, float scale, int merge, float* out, void* ws, size_t ws_bytes,
-                         cudaStream_t stream) {
+                         cudaStream_t stream, const QueryChunks& chunks = QueryChunks{}) {
   if (B < 0) return PACE_ERR_INVALID_ARG;
   if (B == 0) return PACE_OK;
   if (out == nullptr) return PACE_ERR_INVALID_ARG;
@@ -1034,7 +1068,7 @@ pace_status_t importance(const void* Q, const void* K, const int32_t* cu_q, cons
   if (cu_k != cu_q) PACE_CHECK(check_segments(B, cu_k, merge));
   if (static_cast<int64_t>(cu_q[B]) + static_cast<int64_t>(kTile) * B > (int64_t{1} << 30)) return PACE_ERR_INVALID_ARG;
   return dispatch<false>(Q, K, cu_q[B], cu_k[B], cross_segs(B, cu_q, cu_k), Hq, Hkv, D, scale, merge, out, ws, ws_bytes,
-                  stream);
+                  stream, chunks);
 }
 
 // Checks the sequence layout of the full-sequence S_llm.
@@ -1106,4 +1140,27 @@ extern "C" pace_status_t pace_llm_sequence_importance(const void* Q, const void*
   PACE_CHECK(check_sequences(B, cu_seq, vis_start, n_vis, query_set));
   return dispatch<true>(Q, K, cu_seq[B], cu_seq[B], sequence_segs(B, cu_seq, vis_start, n_vis, query_set), n_q_heads,
                   n_kv_heads, head_dim, scale, 1, s_llm_raw, ws, ws_bytes, stream);
+}
+
+extern "C" pace_status_t pace_vit_attn_importance_chunked(const void* Q, const void* K, const int32_t* cu_seqlens,
+                                                          int B, int n_heads, int head_dim, float scale, int merge,
+                                                          float* s_vis_raw, void* ws, size_t ws_bytes, int n_chunks,
+                                                          const int64_t* chunk_end_rows, void* const* chunk_ready,
+                                                          pace_stream_t stream) {
+  if (merge != 1 && merge != 2 && merge != 4) return PACE_ERR_INVALID_ARG;
+  if (B < 0) return PACE_ERR_INVALID_ARG;
+  if (B == 0) return PACE_OK;
+  if (cu_seqlens == nullptr || n_chunks < 1 || n_chunks > 64 || chunk_end_rows == nullptr || chunk_ready == nullptr)
+    return PACE_ERR_INVALID_ARG;
+  for (int c = 0; c < n_chunks; ++c) {
+    if (chunk_ready[c] == nullptr || chunk_end_rows[c] < 0) return PACE_ERR_INVALID_ARG;
+    if (c > 0 && chunk_end_rows[c] < chunk_end_rows[c - 1]) return PACE_ERR_INVALID_ARG;
+  }
+  if (chunk_end_rows[n_chunks - 1] != cu_seqlens[B]) return PACE_ERR_INVALID_ARG;
+  QueryChunks ch;
+  ch.n = n_chunks;
+  ch.end_row = chunk_end_rows;
+  ch.ready = reinterpret_cast<cudaEvent_t const*>(chunk_ready);
+  return importance(Q, K, cu_seqlens, cu_seqlens, B, n_heads, n_heads, head_dim, scale, merge, s_vis_raw, ws,
+                    ws_bytes, stream, ch);
 }

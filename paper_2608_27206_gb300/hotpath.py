@@ -98,30 +98,47 @@ class HotPath:
             f()
 
     # -- one step from host memory ---------------------------------------------------------------
-    # Input tensors in the order the calls need them; each group is copied on a side stream and
-    # the compute stream waits only for the group its next call reads.
-    COPY_GROUPS = (("img",), ("vit_q", "vit_k"), ("llm_q", "llm_k"), ("embed",))
-    CALL_NEEDS = {"density": 0, "vit": 1, "llm": 2, "gather": 3}
+    # Input tensors in the order the calls need them.  They are copied on a side stream and the
+    # compute stream waits only for what its next call reads; the ViT query rows come in
+    # VIT_CHUNKS pieces after the keys, and the row log-sum-exp pass takes each piece as it lands.
+    COPY_GROUPS = (("img",), ("vit_k",), ("vit_q",), ("llm_q", "llm_k"), ("embed",))
+    CALL_NEEDS = {"density": "img", "llm": "llm_k", "gather": "embed"}
+    VIT_CHUNKS = 4
 
     def step_from_host(self, pinned: dict, out_host: dict, copy_stream: Optional[torch.cuda.Stream] = None):
         """Copies this step's inputs from pinned host tensors (keys as in `self.host`), runs the six
         calls, and copies the results named in `out_host` back to (pinned) host tensors.
 
-        The host-to-device copies run on `copy_stream` in call order, so the ViT Q/K copy overlaps
-        density and resampling; each call waits only for the inputs it reads.  The next step's copies
+        The host-to-device copies run on `copy_stream` in call order, so the ViT K/Q copy overlaps
+        density and resampling, and the ViT row pass starts on the first query rows while the rest
+        are still in flight; each call waits only for the inputs it reads.  The next step's copies
         wait for this step's calls to finish (the device input buffers are reused)."""
         main = torch.cuda.current_stream(self.dev)
         cs = copy_stream if copy_stream is not None else torch.cuda.Stream(self.dev)
         cs.wait_stream(main)        # the previous step's calls have read their inputs
-        ready = []
+        ready, q_ready = {}, []
+        ends = P.vit_chunk_rows(self.cu_patches, self.VIT_CHUNKS)
         with torch.cuda.stream(cs):
             for group in self.COPY_GROUPS:
+                if group == ("vit_q",):
+                    r0 = 0
+                    for r1 in ends:
+                        self.d["vit_q"][r0:r1].copy_(pinned["vit_q"][r0:r1], non_blocking=True)
+                        ev = torch.cuda.Event()
+                        ev.record(cs)
+                        q_ready.append(ev)
+                        r0 = int(r1)
+                    continue
                 for k in group:
                     self.d[k].copy_(pinned[k], non_blocking=True)
                 ev = torch.cuda.Event()
                 ev.record(cs)
-                ready.append(ev)
+                ready[group[-1]] = ev
         for name, f in self.parts:
+            if name == "vit":
+                P.pace_vit_attn_importance_chunked(self.d["vit_q"], self.d["vit_k"], self.cu_patches, ends, q_ready,
+                                                   1.0 / math.sqrt(synth.VIT_DIM), 4, out=self.s_vis, ws=self.ws_vit)
+                continue
             if name in self.CALL_NEEDS:
                 main.wait_event(ready[self.CALL_NEEDS[name]])
             f()

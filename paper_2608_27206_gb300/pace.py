@@ -89,6 +89,9 @@ _SIGS = {
     "pace_vit_attn_importance_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, ctypes.c_int]),
     "pace_vit_attn_importance": (ctypes.c_int, [_P, _P, _I32P, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                                 ctypes.c_float, ctypes.c_int, _P, _P, ctypes.c_size_t, _P]),
+    "pace_vit_attn_importance_chunked": (ctypes.c_int, [_P, _P, _I32P, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                                        ctypes.c_float, ctypes.c_int, _P, _P, ctypes.c_size_t,
+                                                        ctypes.c_int, _I64P, ctypes.POINTER(ctypes.c_void_p), _P]),
     "pace_llm_text_visual_importance_workspace_size": (ctypes.c_size_t, [ctypes.c_int, _I32P, _I32P, ctypes.c_int,
                                                                          ctypes.c_int]),
     "pace_llm_text_visual_importance": (ctypes.c_int, [_P, _P, _I32P, _I32P, ctypes.c_int, ctypes.c_int,
@@ -435,6 +438,47 @@ def pace_vit_attn_importance(Q: torch.Tensor, K: torch.Tensor, cu_seqlens, scale
     st = lib().pace_vit_attn_importance(_dev(Q), _dev(K), _pi32(cu), B, Hh, D, float(scale), int(merge), _dev(out),
                                         _dev(ws), ws.numel() * ws.element_size(), _stream(stream))
     _check("pace_vit_attn_importance", st)
+    return out[: int(cu[-1]) // merge]
+
+
+def vit_chunk_rows(cu_seqlens, n_chunks: int, pair: int = 256) -> np.ndarray:
+    """End rows of `n_chunks` near-equal pieces of Q, each end moved down to the end of a
+    `pair`-row block of its image (or the image's end), so no block waits for a later piece."""
+    cu = _i32(cu_seqlens).astype(np.int64)
+    total = int(cu[-1])
+    ends = []
+    for c in range(1, n_chunks):
+        r = total * c // n_chunks
+        b = int(np.searchsorted(cu, r, side="right")) - 1
+        b = min(max(b, 0), len(cu) - 2)
+        e = int(cu[b]) + (r - int(cu[b])) // pair * pair
+        ends.append(max(e, ends[-1] if ends else 0))
+    ends.append(total)
+    return np.asarray(ends, dtype=np.int64)
+
+
+def pace_vit_attn_importance_chunked(Q: torch.Tensor, K: torch.Tensor, cu_seqlens, chunk_end_rows,
+                                     chunk_ready: Sequence[torch.cuda.Event], scale: Optional[float] = None,
+                                     merge: int = 4, out: Optional[torch.Tensor] = None,
+                                     ws: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """pace_vit_attn_importance whose row log-sum-exp pass runs in pieces of query rows, piece c
+    after the (already recorded) event chunk_ready[c]; bit-identical results."""
+    cu = _i32(cu_seqlens)
+    B = len(cu) - 1
+    total, Hh, D = Q.shape
+    if scale is None:
+        scale = float(D) ** -0.5
+    if out is None:
+        out = torch.empty(max(int(cu[-1]) // merge, 1), dtype=torch.float32, device=Q.device)
+    ends = _i64(chunk_end_rows)
+    if len(chunk_ready) != len(ends):
+        raise ValueError("one event per chunk")
+    evs = (ctypes.c_void_p * max(len(ends), 1))(*[int(e.cuda_event) for e in chunk_ready])
+    ws = _workspace(pace_vit_attn_importance_workspace_size(cu, Hh), ws, Q.device)
+    st = lib().pace_vit_attn_importance_chunked(_dev(Q), _dev(K), _pi32(cu), B, Hh, D, float(scale), int(merge),
+                                                _dev(out), _dev(ws), ws.numel() * ws.element_size(), len(ends),
+                                                _pi64(ends), evs, _stream(stream))
+    _check("pace_vit_attn_importance_chunked", st)
     return out[: int(cu[-1]) // merge]
 
 

@@ -103,3 +103,16 @@ def test_budget_vanilla_matches_oracle(libpace):
         f = float(rng.choice([0.05, 0.1, 0.25, rng.uniform(0, 1.2)]))
         assert libpace.pace_budget_vanilla(nv, nc, f) == O.budget_vanilla(nv, nc, f)
     assert libpace.pace_budget_vanilla(10549, 2660, 0.10) == 1055 and libpace.pace_budget_vanilla(10549, 900, 0.10) == 900
+
+
+def test_vit_chunk_rows_ends_on_pair_blocks(libpace):
+    """Chunk ends for the split row pass: nondecreasing, the last at the total, every end an
+    image boundary or a whole number of 256-row blocks into its image."""
+    cu = np.array([0, 516, 520, 648, 1948, 2336, 4388], np.int32)
+    for n in (1, 2, 3, 5, 8, 40):
+        e = libpace.vit_chunk_rows(cu, n)
+        assert len(e) == n and e[-1] == cu[-1] and np.all(np.diff(e) >= 0) and e[0] >= 0
+        for x in e:
+            b = int(np.searchsorted(cu, x, side="right")) - 1
+            assert x in cu or (x - cu[b]) % 256 == 0
+    assert list(libpace.vit_chunk_rows([0, 42196], 4)) == [10496, 20992, 31488, 42196]

@@ -372,6 +372,60 @@ def test_vit_importance_high_run_below_margin(pace):
     _no_device_error(pace)
 
 
+@pytest.mark.parametrize("ends", ["auto1", "auto3", "auto7", "ragged"])
+def test_vit_importance_chunked_matches_unchunked(pace, ends):
+    """The row pass split by query rows, each piece after an event that marks its Q rows copied
+    in on a side stream, gives the same bits as the one-launch call.  Q starts as NaN, so a piece
+    that read rows not yet copied would show up unless those rows are only past its images."""
+    lens = [516, 4, 128, 1300, 388, 2052]
+    H, D, merge = 16, 80, 4
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    total = int(cu[-1])
+    Qb = synth.random_small_qk(21, total, H, D)
+    Kb = synth.random_small_qk(1021, total, H, D)
+    spike = np.zeros((total,), np.float32)
+    spike[[40, 700, 2000]] = 9.0              # three query rows with 10x norm
+    Qb = synth.f32_to_bf16_bits(f64(Qb).astype(np.float32) * (1 + spike[:, None, None]))
+    Q, K = bf16_tensor(Qb), bf16_tensor(Kb)
+    scale = 1.0 / math.sqrt(D)
+    want = pace.pace_vit_attn_importance(Q, K, cu, scale, merge)
+    if ends == "ragged":
+        e = np.array([37, 37, 900, 2500, total], np.int64)    # unaligned, with an empty piece
+    else:
+        e = pace.vit_chunk_rows(cu, int(ends[4:]))
+    assert e[-1] == total and np.all(np.diff(e) >= 0)
+    host = Q.cpu().pin_memory()
+    dq = torch.full_like(Q, float("nan"))
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    evs, r0 = [], 0
+    with torch.cuda.stream(side):
+        for r1 in e:
+            dq[r0:r1].copy_(host[r0:r1], non_blocking=True)
+            ev = torch.cuda.Event()
+            ev.record(side)
+            evs.append(ev)
+            r0 = int(r1)
+    got = pace.pace_vit_attn_importance_chunked(dq, K, cu, e, evs, scale, merge)
+    torch.cuda.synchronize()
+    assert torch.equal(got, want)
+    ref = O.vit_attn_importance(f64(Qb), f64(Kb), cu, scale, merge)
+    assert_scores_close(got.cpu().numpy(), ref, what="chunked S_vis_raw")
+    _no_device_error(pace)
+
+
+def test_vit_importance_chunked_rejects_bad_chunks(pace):
+    Q = torch.zeros((8, 1, 64), dtype=torch.bfloat16, device="cuda")
+    ev = torch.cuda.Event()
+    ev.record()
+    with pytest.raises(pace.PaceError):
+        pace.pace_vit_attn_importance_chunked(Q, Q, [0, 8], [4], [ev], merge=4)       # last end != total
+    with pytest.raises(pace.PaceError):
+        pace.pace_vit_attn_importance_chunked(Q, Q, [0, 8], [6, 4, 8], [ev, ev, ev], merge=4)   # decreasing
+    with pytest.raises(ValueError):
+        pace.pace_vit_attn_importance_chunked(Q, Q, [0, 8], [4, 8], [ev], merge=4)    # one event per chunk
+
+
 def test_llm_importance_wide_score_range(pace):
     """A spike about 245 (base 2) above the other scores through the GQA path with key splits
     (few query tiles, many key tiles): the fixed-shift sum overflows in every split that holds
