@@ -14,7 +14,9 @@ Prints one JSON line.  `value` is microseconds per image with inputs resident in
 timed with CUDA events around each step (each libpace call replayed from a CUDA graph),
 L2 flushed by a 256 MiB write before every step.  `e2e` is the same metric through the
 Python binding with the inputs copied from pinned host memory and the results copied
-back inside the timed region.  Under torchrun every rank processes its own image
+back inside the timed region (two device input slots, so one image's copies run under the
+previous image's calls; `e2e.latency_us_one_image` is one step with nothing else in
+flight).  Under torchrun every rank processes its own image
 (weak scaling, no collective on the data path); the max over ranks is reported.
 `--impl reference` times the fp64 CPU oracle on a bounded sample of the same workload.
 """
@@ -467,10 +469,11 @@ def run_gpu(args):
     h2d = sum(v.numel() * v.element_size() for v in pinned.values())
     d2h = sum(v.numel() * v.element_size() for v in out_host.values())
 
-    copy_stream = torch.cuda.Stream(device)
+    copy_stream, readback_stream = torch.cuda.Stream(device), torch.cuda.Stream(device)
 
     def e2e_step():
-        pipe.step_from_host(pinned, out_host, copy_stream)
+        # returns the event after which the step's results are in the pinned host tensors
+        return pipe.step_from_host(pinned, out_host, copy_stream, readback_stream)
 
     for _ in range(max(1, args.warmup)):
         e2e_step()
@@ -480,14 +483,27 @@ def run_gpu(args):
         dist.barrier()
     torch.cuda.synchronize()
     e_start.record()
+    copy_stream.wait_event(e_start)       # no copy of the timed steps starts before the clock
     for _ in range(args.steps):
-        e2e_step()
+        last = e2e_step()
+    torch.cuda.current_stream(device).wait_event(last)     # every step's results are on the host
     e_end.record()
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e_start.elapsed_time(e_end), world, device)
     if world > 1:
         dist.barrier()
     e2e_value = per_image_us(e2e_ms, args.steps, world)
+    # single-image latency: one step from host memory with nothing else in flight
+    lat = []
+    for _ in range(3):
+        torch.cuda.synchronize()
+        l0, l1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        l0.record()
+        torch.cuda.current_stream(device).wait_event(e2e_step())
+        l1.record()
+        torch.cuda.synchronize()
+        lat.append(l0.elapsed_time(l1))
+    latency_us = max_over_ranks(statistics.median(lat), world, device) * 1e3
 
     if rank == 0:
         peaks, peak_src = load_peaks()
@@ -540,7 +556,10 @@ def run_gpu(args):
             "breakdown_us": {k: round(v * 1e3, 2) for k, v in mean.items()},
             "visual_tokens_scored_per_s": round(wl.n_vis[0] * world / (ms_per_step * 1e-3), 1),
             "cpu_baseline": cpu,
-            "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "e2e": {"value": round(e2e_value, 3), "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "pipelining": "two device input slots: image n+1's host-to-device copies run during image "
+                                  "n's calls; every step's copies and result read-back are inside the timed region",
+                    "latency_us_one_image": round(latency_us, 1)},
             "gpu_launches": launches_per_step * args.steps,
             "clocks": clocks,
             "apc": {"rho": round(stats["rho"], 5), "r": round(stats["r"], 5),

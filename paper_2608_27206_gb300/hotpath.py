@@ -70,80 +70,124 @@ class HotPath:
         self.parts = [("density", self.density), ("resample", self.resample), ("vit", self.vit),
                       ("llm", self.llm), ("select", self.select), ("gather", self.gather)]
 
-    # -- the six calls ---------------------------------------------------------------------------
-    def density(self):
-        P.pace_apc_density(self.d["img"], self.img_off, self.H, self.W, d_out=self.dist, stats=self.stats,
+    # -- the six calls (inputs from `d`, default: the resident copies) ---------------------------
+    def density(self, d=None):
+        d = d or self.d
+        P.pace_apc_density(d["img"], self.img_off, self.H, self.W, d_out=self.dist, stats=self.stats,
                            ws=self.ws_density)
 
-    def resample(self):
-        P.pace_apc_resample(self.d["img"], self.img_off, self.H, self.W, self.stats, self.resized, self.dst_off)
+    def resample(self, d=None):
+        d = d or self.d
+        P.pace_apc_resample(d["img"], self.img_off, self.H, self.W, self.stats, self.resized, self.dst_off)
 
-    def vit(self):
-        P.pace_vit_attn_importance(self.d["vit_q"], self.d["vit_k"], self.cu_patches,
+    def vit(self, d=None):
+        d = d or self.d
+        P.pace_vit_attn_importance(d["vit_q"], d["vit_k"], self.cu_patches,
                                    1.0 / math.sqrt(synth.VIT_DIM), 4, out=self.s_vis, ws=self.ws_vit)
 
-    def llm(self):
-        P.pace_llm_text_visual_importance(self.d["llm_q"], self.d["llm_k"], self.cu_q, self.cu_vis,
+    def llm(self, d=None):
+        d = d or self.d
+        P.pace_llm_text_visual_importance(d["llm_q"], d["llm_k"], self.cu_q, self.cu_vis,
                                           1.0 / math.sqrt(synth.LLM_DIM), out=self.s_llm, ws=self.ws_llm)
 
-    def select(self):
+    def select(self, d=None):
         P.pace_ddae_select(self.s_llm, self.s_vis, self.cu_vis, self.cu_keep, s_final=self.s_final,
                            weights=self.weights, kept=self.kept)
 
-    def gather(self):
-        P.pace_gather(self.d["embed"], self.kept[: int(self.cu_keep[-1])], dst=self.rows)
+    def gather(self, d=None):
+        d = d or self.d
+        P.pace_gather(d["embed"], self.kept[: int(self.cu_keep[-1])], dst=self.rows)
 
     def step(self):
         for _, f in self.parts:
             f()
 
     # -- one step from host memory ---------------------------------------------------------------
-    # Input tensors in the order the calls need them.  They are copied on a side stream and the
-    # compute stream waits only for what its next call reads; the ViT query rows come in
-    # VIT_CHUNKS pieces after the keys, and the row log-sum-exp pass takes each piece as it lands.
+    # Input tensors in the order the calls need them.  They are copied on a side stream into one of
+    # two device input slots, and the compute stream waits only for what its next call reads.
     COPY_GROUPS = (("img",), ("vit_k",), ("vit_q",), ("llm_q", "llm_k"), ("embed",))
     CALL_NEEDS = {"density": "img", "llm": "llm_k", "gather": "embed"}
+    # which call overwrites each result that can be read back
+    WRITERS = {"stats": "density", "dist": "density", "resized": "resample", "s_vis": "vit", "s_llm": "llm",
+               "s_final": "select", "weights": "select", "kept": "select", "rows": "gather"}
     VIT_CHUNKS = 4
 
-    def step_from_host(self, pinned: dict, out_host: dict, copy_stream: Optional[torch.cuda.Stream] = None):
+    def step_from_host(self, pinned: dict, out_host: dict, copy_stream: Optional[torch.cuda.Stream] = None,
+                       readback_stream: Optional[torch.cuda.Stream] = None) -> torch.cuda.Event:
         """Copies this step's inputs from pinned host tensors (keys as in `self.host`), runs the six
-        calls, and copies the results named in `out_host` back to (pinned) host tensors.
+        calls, and copies the results named in `out_host` back to (pinned) host tensors.  Returns
+        the event after which those host tensors hold this step's results.
 
-        The host-to-device copies run on `copy_stream` in call order, so the ViT K/Q copy overlaps
-        density and resampling, and the ViT row pass starts on the first query rows while the rest
-        are still in flight; each call waits only for the inputs it reads.  The next step's copies
-        wait for this step's calls to finish (the device input buffers are reused)."""
+        Steps alternate between two device input slots: a step's copies wait only for the calls of
+        the step before the previous one (the last reader of their slot), so while image n is being
+        processed the inputs of image n + 1 are already crossing the host link, and the results of
+        image n go back on `readback_stream` while image n + 1 is processed (a call that overwrites
+        a result waits for its read-back).  Within a step the ViT K/Q copy overlaps density and
+        resampling.  When nothing else is in flight (the previous step has finished), the ViT
+        query rows are copied in VIT_CHUNKS pieces and the row log-sum-exp pass takes each piece
+        as it lands; behind a running step the copy is done long before the ViT call, and one
+        launch avoids the pieces' partial last waves."""
         main = torch.cuda.current_stream(self.dev)
         cs = copy_stream if copy_stream is not None else torch.cuda.Stream(self.dev)
-        cs.wait_stream(main)        # the previous step's calls have read their inputs
+        if not hasattr(self, "_slots"):
+            self._slots = [self.d, {k: torch.empty_like(v) for k, v in self.d.items()}]
+            self._slot_free = [None, None]
+            self._slot_next = 0
+            self._readback = {}
+        rs = readback_stream if readback_stream is not None else torch.cuda.Stream(self.dev)
+        si = self._slot_next
+        self._slot_next ^= 1
+        d = self._slots[si]
+        prev = self._slot_free[si ^ 1]
+        chunked = prev is None or prev.query()
+        if self._slot_free[si] is not None:
+            cs.wait_event(self._slot_free[si])      # the calls that last read this slot are done
+        else:
+            cs.wait_stream(main)
         ready, q_ready = {}, []
-        ends = P.vit_chunk_rows(self.cu_patches, self.VIT_CHUNKS)
+        ends = P.vit_chunk_rows(self.cu_patches, self.VIT_CHUNKS if chunked else 1)
         with torch.cuda.stream(cs):
             for group in self.COPY_GROUPS:
                 if group == ("vit_q",):
                     r0 = 0
                     for r1 in ends:
-                        self.d["vit_q"][r0:r1].copy_(pinned["vit_q"][r0:r1], non_blocking=True)
+                        d["vit_q"][r0:r1].copy_(pinned["vit_q"][r0:r1], non_blocking=True)
                         ev = torch.cuda.Event()
                         ev.record(cs)
                         q_ready.append(ev)
                         r0 = int(r1)
                     continue
                 for k in group:
-                    self.d[k].copy_(pinned[k], non_blocking=True)
+                    d[k].copy_(pinned[k], non_blocking=True)
                 ev = torch.cuda.Event()
                 ev.record(cs)
                 ready[group[-1]] = ev
         for name, f in self.parts:
+            if name in self._readback:
+                main.wait_event(self._readback.pop(name))   # the previous results of this call are read
             if name == "vit":
-                P.pace_vit_attn_importance_chunked(self.d["vit_q"], self.d["vit_k"], self.cu_patches, ends, q_ready,
-                                                   1.0 / math.sqrt(synth.VIT_DIM), 4, out=self.s_vis, ws=self.ws_vit)
-                continue
-            if name in self.CALL_NEEDS:
+                if chunked:
+                    P.pace_vit_attn_importance_chunked(d["vit_q"], d["vit_k"], self.cu_patches, ends, q_ready,
+                                                       1.0 / math.sqrt(synth.VIT_DIM), 4, out=self.s_vis,
+                                                       ws=self.ws_vit)
+                    continue
+                main.wait_event(q_ready[-1])
+            elif name in self.CALL_NEEDS:
                 main.wait_event(ready[self.CALL_NEEDS[name]])
-            f()
-        for k, v in out_host.items():      # attribute name -> host tensor of the same shape
-            v.copy_(getattr(self, k), non_blocking=True)
+            f(d)
+        free = torch.cuda.Event()
+        free.record(main)
+        self._slot_free[si] = free
+        rs.wait_event(free)
+        order = [k for name, _ in self.parts for k in out_host if self.WRITERS.get(k, "density") == name]
+        done = free
+        with torch.cuda.stream(rs):
+            for k in order:     # in the order the next step overwrites them
+                out_host[k].copy_(getattr(self, k), non_blocking=True)
+                done = torch.cuda.Event()
+                done.record(rs)
+                self._readback[self.WRITERS.get(k, "density")] = done
+        return done
 
     # -- results on the host ---------------------------------------------------------------------
     def resized_images(self):

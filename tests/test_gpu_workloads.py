@@ -136,3 +136,31 @@ def test_img4k_budget_5_percent(pace):
     ref = O.ddae_fuse(s_llm.astype(np.float32).astype(np.float64), s_vis.astype(np.float32).astype(np.float64))
     assert_scores_close(sf.cpu().numpy(), ref["S_final"], atol_frac=2e-3)
     assert_kept_matches(kept.cpu().numpy(), ref["S_final"], K)
+
+
+@pytest.mark.parametrize("name", ["img1344", "ragged16"])
+def test_step_from_host_matches_resident_step(pace, name):
+    """Three steps from pinned host memory (alternating device input slots, the ViT row pass in
+    query-row pieces behind the copies) give the same bits as one step on resident inputs."""
+    from paper_2608_27206_gb300.hotpath import HotPath
+    wl = synth.make_workload(name, seed=1)
+    hp = HotPath(wl, "cuda")
+    hp.step()
+    torch.cuda.synchronize()
+    names = ("stats", "dist", "s_vis", "s_llm", "s_final", "weights", "kept", "rows")
+    want = {k: getattr(hp, k).clone() for k in names}
+    pinned = {k: v.pin_memory() for k, v in hp.host.items()}
+    out = {k: torch.empty(tuple(getattr(hp, k).shape), dtype=getattr(hp, k).dtype).pin_memory()
+           for k in ("kept", "rows", "s_final", "stats")}
+    for v in hp.d.values():            # the resident copies must not be what the steps read
+        v.zero_()
+    cs = torch.cuda.Stream()
+    for _ in range(3):
+        hp.step_from_host(pinned, out, cs)
+    torch.cuda.synchronize()
+    code, where = pace.pace_device_status(clear=True)
+    assert code == 0, (code, where)
+    for k, v in out.items():
+        assert torch.equal(v, want[k].cpu()), k
+    for k in names:
+        assert torch.equal(getattr(hp, k), want[k]), k
