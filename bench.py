@@ -288,6 +288,7 @@ def measure_next_rows(P, device, flush, peak_tf, hbm_gbs, reps=10):
     the prune step's gathers) on the 4K image's shapes, each replayed from a CUDA graph with L2
     flushed before every replay; median over `reps`.  Inputs are seeded device tensors."""
     import torch
+    from paper_2608_27206_gb300 import synth
     g = torch.Generator(device=device)
     g.manual_seed(1234)
 
@@ -384,6 +385,27 @@ def measure_next_rows(P, device, flush, peak_tf, hbm_gbs, reps=10):
                               "us": round(sec * 1e6, 2), "bound": "hbm", "bytes": nbytes,
                               "achieved": round(nbytes / sec / 1e9, 1), "unit": "GB/s",
                               "frac": round(nbytes / sec / 1e9 / hbm_gbs, 4)}
+    del hid, kv, hid_o, kv_o, pos, pos_o
+    # a5/a6 on batches (one 4K map is latency-bound at 131 KB): the 16-image ragged batch's map
+    # sizes and keep fractions, and 64 copies of the 4K image's map; positive random scores
+    for name, nvs, fracs in (("a5a6_select_ragged16", [s.H // synth.MERGE_PX * (s.W // synth.MERGE_PX)
+                                                      for s in synth.workload_specs("ragged16")],
+                              [s.keep for s in synth.workload_specs("ragged16")]),
+                             ("a5a6_select_img4k_x64", [nv] * 64, [0.10] * 64)):
+        cu_v = np.concatenate([[0], np.cumsum(nvs)]).astype(np.int32)
+        ks = [P.pace_budget(n, f) for n, f in zip(nvs, fracs)]
+        cu_k = np.concatenate([[0], np.cumsum(ks)]).astype(np.int32)
+        tot = int(cu_v[-1])
+        s_llm = torch.rand(tot, generator=g, device=device) * 8
+        s_vis = torch.rand(tot, generator=g, device=device).pow(3) * 16
+        sf = torch.empty(tot, dtype=torch.float32, device=device)
+        wts = torch.empty((len(nvs), 2), dtype=torch.float32, device=device)
+        kp = torch.empty(int(cu_k[-1]), dtype=torch.int32, device=device)
+        sec = timed(lambda: P.pace_ddae_select(s_llm, s_vis, cu_v, cu_k, s_final=sf, weights=wts, kept=kp))
+        nbytes = 3 * 4 * tot + 4 * int(cu_k[-1]) + 8 * len(nvs)
+        out[name] = {"shape": f"{len(nvs)} maps, {tot} scores, keep {int(cu_k[-1])}", "us": round(sec * 1e6, 2),
+                     "bound": "hbm", "bytes": nbytes, "achieved": round(nbytes / sec / 1e9, 1), "unit": "GB/s",
+                     "frac": round(nbytes / sec / 1e9 / hbm_gbs, 4)}
     return out
 
 
