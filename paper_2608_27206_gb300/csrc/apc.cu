@@ -98,18 +98,19 @@ __device__ __forceinline__ void load_strip(const uint8_t* __restrict__ img, int 
   const int seg = np * kPatch * 3;  // bytes per row (even; a multiple of 4 when WIDE)
   const int64_t pitch = static_cast<int64_t>(W) * 3;
   const uint8_t* base = img + static_cast<int64_t>(py) * kPatch * pitch + static_cast<int64_t>(px0) * kPatch * 3;
-  if (WIDE) {
-    const int words = seg >> 2;
-    for (int i = threadIdx.x; i < kPatch * words; i += kApcThreads) {
-      const int y = i / words, w = i - y * words;
-      cp_async4(s + y * kStripRowBytes + 4 * w, reinterpret_cast<const uint32_t*>(base + y * pitch) + w);
-    }
-  } else {
-    const int halves = seg >> 1;
-    for (int i = threadIdx.x; i < kPatch * halves; i += kApcThreads) {
-      const int y = i / halves, w = i - y * halves;
-      const uint16_t v = __ldg(reinterpret_cast<const uint16_t*>(base + y * pitch) + w);
-      *reinterpret_cast<uint16_t*>(s + y * kStripRowBytes + 2 * w) = v;
+  // a warp per image row (rows warp, warp + 8), lanes along the row: no per-element division
+  const int lane = threadIdx.x & 31;
+  for (int y = threadIdx.x >> 5; y < kPatch; y += kApcThreads / 32) {
+    const uint8_t* src = base + y * pitch;
+    uint8_t* dst = s + y * kStripRowBytes;
+    if (WIDE) {
+      const int words = seg >> 2;
+      for (int w = lane; w < words; w += 32)
+        cp_async4(dst + 4 * w, reinterpret_cast<const uint32_t*>(src) + w);
+    } else {
+      const int halves = seg >> 1;
+      for (int w = lane; w < halves; w += 32)
+        *reinterpret_cast<uint16_t*>(dst + 2 * w) = __ldg(reinterpret_cast<const uint16_t*>(src) + w);
     }
   }
 }
@@ -187,7 +188,7 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restri
                                                          unsigned long long* __restrict__ sums) {
   __shared__ __align__(16) uint8_t s2[2][kPatch * kStripRowBytes];
   __shared__ uint32_t ssq[8][kStrip];
-  __shared__ float inv[kStrip];
+  __shared__ __align__(16) float inv[kStrip];
   int unit = blockIdx.x;
   if (unit >= units) return;
   // weighted column sums: thread slot j (j = tid, tid + 256) owns columns 2j, 2j+1 (a pair never
@@ -249,15 +250,32 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restri
       inv_norm[t.patch0[q.b] + q.py * t.gw[q.b] + q.px0 + p] = iv;
     }
     __syncthreads();
+    float ivr[kStrip];   // full strips: the 32 inverse norms in registers, the patch loop unrolled
+    if (q.np == kStrip) {
+#pragma unroll
+      for (int p = 0; p < kStrip; p += 4) {
+        const float4 v4 = *reinterpret_cast<const float4*>(inv + p);
+        ivr[p] = v4.x;
+        ivr[p + 1] = v4.y;
+        ivr[p + 2] = v4.z;
+        ivr[p + 3] = v4.w;
+      }
+    }
 #pragma unroll
     for (int qs = 0; qs < 2; ++qs) {
       const int j = threadIdx.x + qs * kApcThreads;
       if (j < kPatchBytes / 2) {
         const uint16_t* col = reinterpret_cast<const uint16_t*>(s + pair_offset(j));
         float2 a = make_float2(0.f, 0.f);
-        for (int p = 0; p < q.np; ++p) {
-          const float iv = inv[p];
-          a = ptx::ffma2(make_float2(iv, iv), bytes2_to_float2(col[p * 21]), a);
+        if (q.np == kStrip) {
+#pragma unroll
+          for (int p = 0; p < kStrip; ++p)
+            a = ptx::ffma2(make_float2(ivr[p], ivr[p]), bytes2_to_float2(col[p * 21]), a);
+        } else {
+          for (int p = 0; p < q.np; ++p) {
+            const float iv = inv[p];
+            a = ptx::ffma2(make_float2(iv, iv), bytes2_to_float2(col[p * 21]), a);
+          }
         }
         acc[qs][0] += fix32(a.x * (1.0f / 255.0f));
         acc[qs][1] += fix32(a.y * (1.0f / 255.0f));
@@ -290,12 +308,15 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
 #pragma unroll
   for (int it = 0; it < kPairIters; ++it) off[it] = pair_offset(min(lane + 32 * it, kPatchBytes / 2 - 1));
   int cur_b = -1;
+  bool reload = false;
+  float2 chr[kPairIters];   // c_hat of this lane's coordinate pairs, in registers
   issue_strip<WIDE>(img, t, unit, s2[0]);
   for (int i = 0; unit < units; ++i, unit += gridDim.x) {
     const int next = unit + static_cast<int>(gridDim.x);
     const Strip q = strip_of(t, unit);
     if (q.b != cur_b) {   // c = sums / N, |c|^2 (fixed summation order), c_hat = c / |c|
       cur_b = q.b;
+      reload = true;
       const int N = (t.H[q.b] / kPatch) * t.gw[q.b];
       const float inv_n = 1.0f / static_cast<float>(N);
       const unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + q.b) * kTokDim;
@@ -332,6 +353,11 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
     // d_i = |t_i - c_hat| computed directly: warp per patch, lanes over column pairs
     const float* pinv = inv_norm + t.patch0[q.b] + q.py * t.gw[q.b] + q.px0;
     const float2* chat2 = reinterpret_cast<const float2*>(chat);
+    if (reload) {
+#pragma unroll
+      for (int it = 0; it < kPairIters; ++it) chr[it] = chat2[min(lane + 32 * it, kPatchBytes / 2 - 1)];
+      reload = false;
+    }
     for (int p = warp; p < q.np; p += kApcThreads / 32) {
       const float sc = pinv[p] * (1.0f / 255.0f);
       const float2 sc2 = make_float2(sc, sc);
@@ -341,8 +367,7 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
         const int j = lane + 32 * it;
         if (it < kPairIters - 1 || j < kPatchBytes / 2) {
           const uint32_t v = *reinterpret_cast<const uint16_t*>(s + off[it] + p * 42);
-          const float2 ch = chat2[j];
-          const float2 e = ptx::ffma2(bytes2_to_float2(v), sc2, make_float2(-ch.x, -ch.y));
+          const float2 e = ptx::ffma2(bytes2_to_float2(v), sc2, make_float2(-chr[it].x, -chr[it].y));
           acc2 = ptx::ffma2(e, e, acc2);
         }
       }
