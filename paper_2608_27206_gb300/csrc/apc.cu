@@ -579,18 +579,22 @@ struct TailParams {
 
 constexpr int kTailSmemMax = 48 * 1024;   // d values staged in shared memory (floats)
 constexpr int kTailBins = 4096;            // level-1 buckets of the tail select
+constexpr int kTailBins2 = 1024;           // level-2 offset bins over a compacted bucket
 
 // Bucket of a distance d >= 0: floor(2048 d), capped at the top bucket (monotone in d).
 __device__ __forceinline__ int tail_bucket(float v) { return min(static_cast<int>(v * 2048.0f), kTailBins - 1); }
 
-// Called by all 1024 threads: the bin holding the r-th largest entry, counting from bin 4095 down
-// (1 <= r <= total): sel[0] = that bin, sel[1] = entries in the bins above it.  wsum: 32 words.
+// Called by all 1024 threads: the bin holding the r-th largest entry, counting from bin NBINS - 1
+// down (1 <= r <= total): sel[0] = that bin, sel[1] = entries in the bins above it.  wsum: 32 words.
+template <int NBINS>
 __device__ __forceinline__ void select_from_top(const unsigned* bins, unsigned r, unsigned* sel, unsigned* wsum) {
+  constexpr int PER = NBINS / 1024;   // bins per thread
+  static_assert(PER >= 1 && PER * 1024 == NBINS, "bins");
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int top = kTailBins - 1 - 4 * static_cast<int>(threadIdx.x);   // this thread: bins top .. top - 3
-  unsigned c4[4], s4 = 0u;
+  const int top = NBINS - 1 - PER * static_cast<int>(threadIdx.x);   // this thread: bins top .. top - PER + 1
+  unsigned c4[PER], s4 = 0u;
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
+  for (int q = 0; q < PER; ++q) {
     c4[q] = bins[top - q];
     s4 += c4[q];
   }
@@ -618,7 +622,7 @@ __device__ __forceinline__ void select_from_top(const unsigned* bins, unsigned r
     unsigned above = excl;
     int q = 0;
 #pragma unroll
-    for (int qq = 0; qq < 3; ++qq)
+    for (int qq = 0; qq < PER - 1; ++qq)
       if (q == qq && above + c4[qq] < r) {
         above += c4[qq];
         q = qq + 1;
@@ -633,9 +637,12 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
                                                  TailParams prm, pace_apc_stats* __restrict__ stats) {
   extern __shared__ float sd[];
   __shared__ unsigned bins[kTailBins];
+  __shared__ unsigned hist2[kTailBins2];
   __shared__ unsigned sel[2];
   __shared__ float red[32];
   __shared__ unsigned cred[32];
+  __shared__ unsigned long long fred[32];
+  __shared__ unsigned ncomp;
   const int b = blockIdx.x;
   const int N = t.n[b];
   const float* db = d + t.patch0[b];
@@ -655,67 +662,131 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
 #pragma unroll 4
   for (int i = threadIdx.x; i < N; i += blockDim.x) atomicAdd(&bins[tail_bucket(db[i])], 1u);
   __syncthreads();
-  select_from_top(bins, k, sel, cred);
+  select_from_top<kTailBins>(bins, k, sel, cred);
   const int tb = static_cast<int>(sel[0]);
-  // Level 2: the bucket's members by key offset from its first key, 4096 offsets (2^shift keys
-  // each) at a time, until one key is left: the k-th largest distance.
+  const unsigned cb = bins[tb];   // entries in the k-th largest's bucket
   unsigned lo = __float_as_uint(static_cast<float>(tb) * (1.0f / 2048.0f));
   unsigned span = (tb == kTailBins - 1 ? 0x7F800001u : __float_as_uint(static_cast<float>(tb + 1) * (1.0f / 2048.0f))) - lo;
   unsigned remaining = k - sel[1];
-  while (true) {
-    const int bits = 32 - __clz(span - 1u);        // keys lo .. lo + span - 1 need `bits` bits
-    const int shift = bits > 12 ? bits - 12 : 0;
-    __syncthreads();                               // everyone has read sel and the bins
-    for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
+  float s = 0.f;                    // this thread's share of the entries above the k-th largest
+  unsigned long long s_fix = 0ull;  // ... the bucket members among them, 2^-32 fixed point
+  unsigned cnt = 0u;
+  unsigned prefix;
+  if (cb <= kTailBins) {
+    // Level 2 on a short list.  One pass compacts the bucket's members into `bins` (free after
+    // the level-1 select) and sums the entries of the buckets above it; the members are then
+    // narrowed by key offset from the bucket's first key, 1024 offsets (2^shift keys each) at a
+    // time, until one key is left: the k-th largest distance.  The list order depends on warp
+    // timing, so the members' sum is taken in fixed point (exact, order-independent).
+    __syncthreads();   // everyone has read sel and bins[tb]
+    if (threadIdx.x == 0) ncomp = 0u;
     __syncthreads();
-    for (int base = 0; base < N; base += blockDim.x) {   // uniform trip count: __match_any_sync below
+    for (int base = 0; base < N; base += blockDim.x) {   // uniform trip count: __ballot_sync below
       const int i = base + static_cast<int>(threadIdx.x);
-      const unsigned off = i < N ? __float_as_uint(db[i]) - lo : span;   // wraps for keys below lo
-      const bool in = off < span;
-      const unsigned digit = in ? off >> shift : kTailBins;
+      const float v = i < N ? db[i] : 0.f;
+      const int bk = i < N ? tail_bucket(v) : -1;
+      if (bk > tb) {
+        s += v;
+        ++cnt;
+      }
+      const bool in = bk == tb;
       const unsigned members = __ballot_sync(0xffffffffu, in);
-      if (__popc(members) > 4) {
-        // many members in this warp: lanes with the same digit add once (identical distances
-        // would otherwise serialise on one counter)
-        const unsigned peers = __match_any_sync(0xffffffffu, digit);
-        if (in && lane_id == __ffs(peers) - 1) atomicAdd(&bins[digit], static_cast<unsigned>(__popc(peers)));
-      } else if (in) {
-        atomicAdd(&bins[digit], 1u);
+      if (members != 0u) {
+        const int leader = __ffs(members) - 1;
+        unsigned slot = 0u;
+        if (lane_id == leader) slot = atomicAdd(&ncomp, static_cast<unsigned>(__popc(members)));
+        slot = __shfl_sync(0xffffffffu, slot, leader);
+        if (in) bins[slot + __popc(members & ((1u << lane_id) - 1u))] = __float_as_uint(v);
       }
     }
     __syncthreads();
-    select_from_top(bins, remaining, sel, cred);
-    lo += sel[0] << shift;
-    remaining -= sel[1];
-    if (shift == 0) break;
-    span = min(span - (sel[0] << shift), 1u << shift);
-  }
-  const unsigned prefix = lo;
-  const float T = __uint_as_float(prefix);   // k-th largest d
-  float s = 0.f;
-  unsigned cnt = 0u;
-  for (int i = threadIdx.x; i < N; i += blockDim.x) {
-    const float v = db[i];
-    if (__float_as_uint(v) > prefix) {
-      s += v;
-      ++cnt;
+    while (true) {
+      const int bits = 32 - __clz(span - 1u);
+      const int shift = bits > 10 ? bits - 10 : 0;
+      for (int i = threadIdx.x; i < kTailBins2; i += blockDim.x) hist2[i] = 0u;
+      __syncthreads();
+      for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
+        const unsigned off = bins[i] - lo;   // wraps for keys below lo
+        if (off < span) atomicAdd(&hist2[off >> shift], 1u);
+      }
+      __syncthreads();
+      select_from_top<kTailBins2>(hist2, remaining, sel, cred);
+      lo += sel[0] << shift;
+      remaining -= sel[1];
+      if (shift == 0) break;
+      span = min(span - (sel[0] << shift), 1u << shift);
+    }
+    prefix = lo;
+    for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
+      const unsigned key = bins[i];
+      if (key > prefix) {
+        s_fix += fix32(__uint_as_float(key));
+        ++cnt;
+      }
+    }
+  } else {
+    // Level 2 over the whole array (a crowded bucket): the bucket's members by key offset from
+    // its first key, 4096 offsets (2^shift keys each) at a time, until one key is left.
+    while (true) {
+      const int bits = 32 - __clz(span - 1u);        // keys lo .. lo + span - 1 need `bits` bits
+      const int shift = bits > 12 ? bits - 12 : 0;
+      __syncthreads();                               // everyone has read sel and the bins
+      for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
+      __syncthreads();
+      for (int base = 0; base < N; base += blockDim.x) {   // uniform trip count: __match_any_sync below
+        const int i = base + static_cast<int>(threadIdx.x);
+        const unsigned off = i < N ? __float_as_uint(db[i]) - lo : span;   // wraps for keys below lo
+        const bool in = off < span;
+        const unsigned digit = in ? off >> shift : kTailBins;
+        const unsigned members = __ballot_sync(0xffffffffu, in);
+        if (__popc(members) > 4) {
+          // many members in this warp: lanes with the same digit add once (identical distances
+          // would otherwise serialise on one counter)
+          const unsigned peers = __match_any_sync(0xffffffffu, digit);
+          if (in && lane_id == __ffs(peers) - 1) atomicAdd(&bins[digit], static_cast<unsigned>(__popc(peers)));
+        } else if (in) {
+          atomicAdd(&bins[digit], 1u);
+        }
+      }
+      __syncthreads();
+      select_from_top<kTailBins>(bins, remaining, sel, cred);
+      lo += sel[0] << shift;
+      remaining -= sel[1];
+      if (shift == 0) break;
+      span = min(span - (sel[0] << shift), 1u << shift);
+    }
+    prefix = lo;
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+      const float v = db[i];
+      if (__float_as_uint(v) > prefix) {
+        s += v;
+        ++cnt;
+      }
     }
   }
+  const float T = __uint_as_float(prefix);   // k-th largest d
   s = warp_sum_f(s);
-  for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+  for (int o = 16; o > 0; o >>= 1) {
+    cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+    s_fix += __shfl_xor_sync(0xffffffffu, s_fix, o);
+  }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (lane == 0) {
     red[warp] = s;
     cred[warp] = cnt;
+    fred[warp] = s_fix;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
     float tot = 0.f;
     unsigned c = 0u;
+    unsigned long long f = 0ull;
     for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) {
       tot += red[w];
       c += cred[w];
+      f += fred[w];
     }
+    tot += unfix32<false>(f, 1.0f);
     tot += static_cast<float>(k - c) * T;  // the remaining entries all equal T
     const float d_top = tot / static_cast<float>(k);
     const float rho_g = stats[t.b_base + b].rho_g;
