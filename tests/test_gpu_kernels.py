@@ -215,6 +215,24 @@ def test_density_constant_images(pace):
         assert (s["h_out"], s["w_out"]) == (28, 28)
 
 
+@pytest.mark.parametrize("side,noisy", [(1008, 0.05), (896, 0.03), (896, 0.5)])
+def test_density_crowded_tail(pace, side, noisy):
+    """Images whose tail bucket is crowded with identical distances: a constant background with
+    a fraction of noise patches.  1008^2 at 5 % puts ~4900 equal distances in the k-th largest's
+    bucket (more than the 4096-entry list: whole-array selection rounds); 896^2 at 3 % puts ~3970
+    there (the compacted list, full of equal keys); 896^2 at 50 % has the k-th largest among the
+    noise patches."""
+    rng = np.random.default_rng(side + int(noisy * 100))
+    img = np.full((side, side, 3), 120, dtype=np.uint8)
+    g = side // 14
+    for q in rng.choice(g * g, size=int(noisy * g * g), replace=False):
+        y, x = divmod(int(q), g)
+        img[14 * y:14 * y + 14, 14 * x:14 * x + 14] = rng.integers(0, 256, (14, 14, 3), dtype=np.uint8)
+    d, st = _density(pace, [img])
+    _check_density(d, st, [img])
+    _no_device_error(pace)
+
+
 def test_density_rejects_bad_sizes(pace):
     img = np.zeros((30, 28, 3), dtype=np.uint8)
     with pytest.raises(pace.PaceError) as e:
