@@ -294,6 +294,22 @@ __device__ __forceinline__ void lse_fixed64(const uint32_t (&v)[64], int valid, 
   l_run += a.x + a.y;
 }
 
+// Fixed-shift update of a full chunk once the shift is set (no masking, no maximum).
+__device__ __forceinline__ void lse_fixed_full(const uint32_t (&v)[64], float c, float m_run, float& l_run) {
+  const float2 cc = make_float2(c, c);
+  const float2 nm = make_float2(-m_run, -m_run);
+  float2 a0 = make_float2(0.f, 0.f), a1 = a0;
+#pragma unroll
+  for (int e = 0; e < 64; e += 4) {
+    const float2 x0 = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), cc, nm);
+    const float2 x1 = ffma2(make_float2(__uint_as_float(v[e + 2]), __uint_as_float(v[e + 3])), cc, nm);
+    a0 = fadd2(a0, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
+    a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
+  }
+  const float2 a = fadd2(a0, a1);
+  l_run += a.x + a.y;
+}
+
 // Dispatch of the fixed-shift update: the first chunk with keys sets the shift.  The two
 // cases are separate instantiations so that the maximum is not issued (predicated off) for
 // every chunk.
@@ -497,6 +513,16 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         const int valid = CAUSAL ? min(t.nk[b] - cs, diag + qrow0 + rr - cs + 1) : t.nk[b] - cs;
         uint32_t sv[64];
         load_cols64(tbuf, sv);
+        const bool lean = __all_sync(0xffffffffu, round == 0 && valid >= 128 && m_run > -INFINITY);
+        if (lean) {   // the common tile: both chunks full, shift already fixed
+          lse_fixed_full(sv, c, m_run, l_run);
+          load_cols64(tbuf + 64, sv);
+          tc_fence_before_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(b_sfree(p));
+          lse_fixed_full(sv, c, m_run, l_run);
+          continue;
+        }
         if (round == 0) lse_fixed(sv, valid, c, m_run, l_run);
         else lse_update64(sv, valid, c, m_run, l_run);
         load_cols64(tbuf + 64, sv);
