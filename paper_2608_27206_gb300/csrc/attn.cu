@@ -294,11 +294,12 @@ __device__ __forceinline__ void lse_fixed64(const uint32_t (&v)[64], int valid, 
   l_run += a.x + a.y;
 }
 
-// Fixed-shift update of a full chunk once the shift is set (no masking, no maximum).
-__device__ __forceinline__ void lse_fixed_full(const uint32_t (&v)[64], float c, float m_run, float& l_run) {
+// Fixed-shift update of a full chunk once the shift is set (no masking, no maximum); the sum
+// stays in two packed partial sums that the caller folds into l once, after its last chunk.
+__device__ __forceinline__ void lse_fixed_full(const uint32_t (&v)[64], float c, float m_run, float2& a0,
+                                               float2& a1) {
   const float2 cc = make_float2(c, c);
   const float2 nm = make_float2(-m_run, -m_run);
-  float2 a0 = make_float2(0.f, 0.f), a1 = a0;
 #pragma unroll
   for (int e = 0; e < 64; e += 4) {
     const float2 x0 = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), cc, nm);
@@ -306,8 +307,6 @@ __device__ __forceinline__ void lse_fixed_full(const uint32_t (&v)[64], float c,
     a0 = fadd2(a0, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
     a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
   }
-  const float2 a = fadd2(a0, a1);
-  l_run += a.x + a.y;
 }
 
 // Dispatch of the fixed-shift update: the first chunk with keys sets the shift.  The two
@@ -319,27 +318,26 @@ __device__ __forceinline__ void lse_fixed(const uint32_t (&v)[64], int valid, fl
   else lse_fixed64<false>(v, valid, c, m_run, l_run);
 }
 
-// acc += sum_e 2^(c a_e) over 64 columns, a_e = s_e - L / c straight from the MMA.
-__device__ __forceinline__ float2 colsum64(const uint32_t (&v)[64], float c, float2 acc) {
+// (a0, a1) += sum_e 2^(c a_e) over 64 columns, a_e = s_e - L / c straight from the MMA, as two
+// packed partial sums carried across chunks.
+__device__ __forceinline__ void colsum64(const uint32_t (&v)[64], float c, float2& a0, float2& a1) {
   const float2 cc = make_float2(c, c);
   const float2 zero = make_float2(0.f, 0.f);
-  float2 a1 = zero;
 #pragma unroll
   for (int e = 0; e < 64; e += 4) {
     const float2 x0 = ffma2(make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), cc, zero);
     const float2 x1 = ffma2(make_float2(__uint_as_float(v[e + 2]), __uint_as_float(v[e + 3])), cc, zero);
-    acc = fadd2(acc, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
+    a0 = fadd2(a0, make_float2(ex2_approx(x0.x), ex2_approx(x0.y)));
     a1 = fadd2(a1, make_float2(ex2_approx(x1.x), ex2_approx(x1.y)));
   }
-  return fadd2(acc, a1);
 }
 
 // colsum64 over the columns e >= lo only (the causal mask of pass 2).
-__device__ __forceinline__ float2 colsum64_from(const uint32_t (&v)[64], int lo, float c, float2 acc) {
+__device__ __forceinline__ void colsum64_from(const uint32_t (&v)[64], int lo, float c, float2& a0, float2& a1) {
   uint32_t w[64];
 #pragma unroll
   for (int e = 0; e < 64; ++e) w[e] = e < lo ? 0xFF800000u : v[e];   // -inf: 2^(c * -inf) = 0
-  return colsum64(w, c, acc);
+  colsum64(w, c, a0, a1);
 }
 
 // Brings the CTA to a quiet point: waits for its MMAs (phase `done_phase` of b_done) and lets
@@ -498,6 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
     } else {
       // epilogue warpgroup e = 2p + hh: accumulator p (stream tiles it % 2 == p), columns hh * 128 ..
       float m_run = -INFINITY, l_run = 0.f;
+      float2 la0 = make_float2(0.f, 0.f), la1 = la0;   // the full chunks' sums (round 0 only)
       const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
       for (int j = (p - it0) & 1; j < nj; j += 2) {
         const int it = it0 + j;
@@ -515,12 +514,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         load_cols64(tbuf, sv);
         const bool lean = __all_sync(0xffffffffu, round == 0 && valid >= 128 && m_run > -INFINITY);
         if (lean) {   // the common tile: both chunks full, shift already fixed
-          lse_fixed_full(sv, c, m_run, l_run);
+          lse_fixed_full(sv, c, m_run, la0, la1);
           load_cols64(tbuf + 64, sv);
           tc_fence_before_sync();
           __syncwarp();
           if (lane == 0) mbar_arrive(b_sfree(p));
-          lse_fixed_full(sv, c, m_run, l_run);
+          lse_fixed_full(sv, c, m_run, la0, la1);
           continue;
         }
         if (round == 0) lse_fixed(sv, valid, c, m_run, l_run);
@@ -531,6 +530,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         if (lane == 0) mbar_arrive(b_sfree(p));
         if (round == 0) lse_fixed(sv, valid - 64, c, m_run, l_run);
         else if (valid > 64) lse_update64(sv, valid - 64, c, m_run, l_run);
+      }
+      {
+        const float2 a = fadd2(la0, la1);
+        l_run += a.x + a.y;
       }
       // inf or NaN in a row of the image: it needs the exact round (rows past the image are
       // ignored, so whatever their Q rows hold cannot change the valid rows' results)
@@ -736,7 +739,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
     const int p = e >> 1, hh = e & 1;
     const int quad = warp & 3;
     const int rr = quad * 32 + lane;
-    float2 acc = make_float2(0.f, 0.f);
+    float2 acc = make_float2(0.f, 0.f), acc1 = acc;
     const uint32_t tbuf = tmem + (static_cast<uint32_t>(quad * 32) << 16) + p * 256 + hh * 128;
     const int key = krow0 + rr;
     for (int j = p; j < nj; j += 2) {
@@ -756,13 +759,16 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
       }
       uint32_t sv[64];
       load_cols64(tbuf, sv);
-      acc = masked ? colsum64_from(sv, lo, c, acc) : colsum64(sv, c, acc);
+      if (masked) colsum64_from(sv, lo, c, acc, acc1);
+      else colsum64(sv, c, acc, acc1);
       load_cols64(tbuf + 64, sv);
       tc_fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(b_sfree(p));
-      acc = masked ? colsum64_from(sv, lo - 64, c, acc) : colsum64(sv, c, acc);
+      if (masked) colsum64_from(sv, lo - 64, c, acc, acc1);
+      else colsum64(sv, c, acc, acc1);
     }
+    acc = fadd2(acc, acc1);
     const float a = acc.x + acc.y;
     if (e > 0) ctl->xchg[e - 1][0][rr] = a;
     named_barrier_sync(1, 32 * kEpiWarps);
