@@ -502,7 +502,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         const int it = it0 + j;
         const int v = it >> 1;
         const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs));
-        if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
+        // warp-uniform exit: the tcgen05.ld below is warp-wide.  The epilogue does not poll the
+        // abort flag per tile: an abort elsewhere reaches it through its own bounded wait.
+        if (!ok) {
           set_abort(ctl, status, K_ATTN_ROW_LSE);
           break;
         }
@@ -512,7 +514,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         const int valid = CAUSAL ? min(t.nk[b] - cs, diag + qrow0 + rr - cs + 1) : t.nk[b] - cs;
         uint32_t sv[64];
         load_cols64(tbuf, sv);
-        const bool lean = __all_sync(0xffffffffu, round == 0 && valid >= 128 && m_run > -INFINITY);
+        const bool lean = CAUSAL ? __all_sync(0xffffffffu, round == 0 && valid >= 128 && m_run > -INFINITY)
+                                 : (round == 0 && valid >= 128 && m_run > -INFINITY);
         if (lean) {   // the common tile: both chunks full, shift already fixed
           lse_fixed_full(sv, c, m_run, la0, la1);
           load_cols64(tbuf + 64, sv);
@@ -745,7 +748,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
     for (int j = p; j < nj; j += 2) {
       const int v = j >> 1;
       const bool ok = __all_sync(0xffffffffu, mbar_wait(b_sfull(p), v & 1, kWaitLimitNs));
-      if (!ok || aborted(ctl)) {   // warp-uniform exit: the tcgen05.ld below is warp-wide
+      if (!ok) {   // warp-uniform exit (see pass 1): the tcgen05.ld below is warp-wide
         set_abort(ctl, status, K_ATTN_COLSUM);
         break;
       }
