@@ -384,49 +384,5 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
   return m;
 }
 
-// Pair add rounded toward -infinity, and pair subtraction.
-__device__ __forceinline__ float2 fadd2_rm(float2 a, float2 b) {
-  float2 d;
-  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-      "mov.b64 ra, {%2, %3};\n\t"
-      "mov.b64 rb, {%4, %5};\n\t"
-      "add.rm.ftz.f32x2 rd, ra, rb;\n\t"
-      "mov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d.x), "=f"(d.y)
-      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-  return d;
-}
-__device__ __forceinline__ float2 fsub2(float2 a, float2 b) {
-  float2 d;
-  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-      "mov.b64 ra, {%2, %3};\n\t"
-      "mov.b64 rb, {%4, %5};\n\t"
-      "sub.rn.ftz.f32x2 rd, ra, rb;\n\t"
-      "mov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d.x), "=f"(d.y)
-      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-  return d;
-}
-
-// 2^x for two lanes on the FMA pipe, for x < 127 (inputs below -126 are raised to -126, whose
-// result 2^-126 is negligible next to any term the callers sum with it).  Cody-Waite style
-// split x = j + f with j = floor(x) read from the low mantissa bits of x + 1.5 * 2^23 rounded
-// toward -infinity and f in [0, 1); 2^f by a cubic whose coefficients minimise the maximum
-// relative error on [0, 1) (fitted for this code by a Remez exchange: max relative error
-// 7.5e-5 in float32 Horner form); 2^j by adding j to the exponent field.  The cubic is
-// 0.99993 at f = 0, just below 1, so j >= -126 keeps the exponent field non-negative.
-__device__ __forceinline__ float2 exp2_fma2(float2 x) {
-  x.x = fmaxf(x.x, -126.f);
-  x.y = fmaxf(x.y, -126.f);
-  const float2 magic = make_float2(12582912.f, 12582912.f);
-  const float2 t = fadd2_rm(x, magic);
-  const float2 f = fsub2(x, fsub2(t, magic));
-  float2 q = ffma2(f, make_float2(0.0780245215f, 0.0780245215f), make_float2(0.226067156f, 0.226067156f));
-  q = ffma2(q, f, make_float2(0.695833564f, 0.695833564f));
-  q = ffma2(q, f, make_float2(0.999925196f, 0.999925196f));
-  return make_float2(__uint_as_float(__float_as_uint(q.x) + (__float_as_uint(t.x) << 23)),
-                     __uint_as_float(__float_as_uint(q.y) + (__float_as_uint(t.y) << 23)));
-}
-
 }  // namespace ptx
 }  // namespace pace
