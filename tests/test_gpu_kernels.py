@@ -687,3 +687,59 @@ def test_prune_index_and_gather_multi(pace):
     code, where = pace.pace_device_status(clear=True)
     assert code == 1 and where == 13
     assert torch.equal(o2[0], hid[0]) and bool((o2[1] == 0).all())
+
+
+# ----------------------------------------------------------------------------------------------
+# batches larger than one kernel-parameter table (the host loops over groups of images)
+# ----------------------------------------------------------------------------------------------
+def test_many_images_attention(pace):
+    """70 images: the attention calls take 64 images per launch table, so this runs two groups
+    (ViT one-launch and in query-row pieces, LLM text -> visual)."""
+    rng = np.random.default_rng(70)
+    lens = [4 * int(x) for x in rng.integers(1, 40, 70)]
+    out, ref, cu = _vit_case(pace, lens, H=4, merge=4, seed=70)
+    assert_scores_close(out, ref, what="S_vis_raw, 70 images")
+    Qb = synth.random_small_qk(70, int(cu[-1]), 4, 80)
+    Kb = synth.random_small_qk(1070, int(cu[-1]), 4, 80)
+    Q, K = bf16_tensor(Qb), bf16_tensor(Kb)
+    scale = 1.0 / math.sqrt(80)
+    want = pace.pace_vit_attn_importance(Q, K, cu, scale, 4)
+    e = pace.vit_chunk_rows(cu, 5)
+    evs = []
+    for _ in e:
+        ev = torch.cuda.Event()
+        ev.record()
+        evs.append(ev)
+    got = pace.pace_vit_attn_importance_chunked(Q, K, cu, e, evs, scale, 4)
+    torch.cuda.synchronize()
+    assert torch.equal(got, want)
+    tq = [int(x) for x in rng.integers(1, 20, 70)]
+    nv = [int(x) for x in rng.integers(1, 90, 70)]
+    out, ref, _, _ = _llm_case(pace, tq, nv, Hq=8, Hkv=2, seed=71)
+    assert_scores_close(out, ref, what="S_llm_raw, 70 images")
+    _no_device_error(pace)
+
+
+def test_many_images_density_and_select(pace):
+    """70 images through the density (64 per table), resample from the device statistics, and
+    70 maps through fusion + top-K."""
+    rng = np.random.default_rng(71)
+    imgs = [synth.make_image(rng, 28 * int(h), 28 * int(w), 2, 2, float(f))
+            for h, w, f in zip(rng.integers(1, 6, 70), rng.integers(1, 6, 70), rng.uniform(0.1, 0.9, 70))]
+    d, st = _density(pace, imgs)
+    _check_density(d, st, imgs)
+    lens = [int(x) for x in rng.integers(1, 400, 70)]
+    fracs = [float(x) for x in rng.choice([0.05, 0.1, 0.25, 1.0], 70)]
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    sl = rng.gamma(0.5, 2.0, size=cu[-1]).astype(np.float32)
+    sv = rng.lognormal(0, 1, size=cu[-1]).astype(np.float32)
+    keep = [O.budget(n, f) for n, f in zip(lens, fracs)]
+    s_final, w, kept = _select(pace, sl, sv, cu, keep)
+    k0 = 0
+    for b, n in enumerate(lens):
+        v0, v1 = cu[b], cu[b + 1]
+        f = O.ddae_fuse(sl[v0:v1].astype(np.float64), sv[v0:v1].astype(np.float64))
+        assert_scores_close(s_final[v0:v1], f["S_final"], atol_frac=2e-3, what="S_final, 70 maps")
+        assert_kept_matches(kept[k0:k0 + keep[b]], f["S_final"], keep[b], offset=v0)
+        k0 += keep[b]
+    _no_device_error(pace)
