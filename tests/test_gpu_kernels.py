@@ -743,3 +743,36 @@ def test_many_images_density_and_select(pace):
         assert_kept_matches(kept[k0:k0 + keep[b]], f["S_final"], keep[b], offset=v0)
         k0 += keep[b]
     _no_device_error(pace)
+
+
+def test_many_images_resample_tokens_sequences(pace):
+    """70 images through the resample (target sizes read on the device), the preview-token
+    density and the full-sequence S_llm: each takes 64 images per parameter table."""
+    rng = np.random.default_rng(72)
+    imgs = [synth.make_image(rng, 28 * int(h), 28 * int(w), 2, 2, float(f))
+            for h, w, f in zip(rng.integers(1, 5, 70), rng.integers(1, 5, 70), rng.uniform(0.1, 0.9, 70))]
+    buf, off = synth.pack_images(imgs)
+    H = [im.shape[0] for im in imgs]
+    W = [im.shape[1] for im in imgs]
+    src = torch.from_numpy(buf).cuda()
+    _, st = pace.pace_apc_density(src, off, H, W)
+    sd = pace.stats_dict(st)
+    dst_off = np.concatenate([[0], np.cumsum([h * w * 3 for h, w in zip(H, W)])])[:-1].astype(np.int64)
+    dst = torch.zeros(int(sum(h * w * 3 for h, w in zip(H, W))), dtype=torch.uint8, device="cuda")
+    pace.pace_apc_resample(src, off, H, W, st, dst, dst_off)
+    flat = dst.cpu().numpy()
+    for b, (img, s) in enumerate(zip(imgs, sd)):
+        ho, wo = s["h_out"], s["w_out"]
+        mine = flat[dst_off[b]:dst_off[b] + ho * wo * 3].reshape(ho, wo, 3).astype(np.int32)
+        assert np.abs(mine - O.apc_resample(img, ho, wo).astype(np.int32)).max() <= 1, b
+    lens = [int(x) for x in rng.integers(1, 60, 70)]
+    T, cu, Ht, Wt, d, stt = _tokens_case(pace, lens, 64, seed=72, sizes=[(28 * 4, 28 * 4)] * 70)
+    for b in range(70):
+        ref = O.apc_density_preview(T[cu[b]:cu[b + 1]], Ht[b], Wt[b])
+        assert_scores_close(d[cu[b]:cu[b + 1]], ref["d"], atol_frac=2e-3, atol=1e-5, what="token d_i, 70 images")
+    S = [int(x) for x in rng.integers(12, 80, 70)]
+    vis = [int(rng.integers(0, s // 3)) for s in S]
+    nvis = [int(rng.integers(1, s - v)) for s, v in zip(S, vis)]
+    out, ref = _seq_case(pace, S, vis, nvis, "vision_text", Hq=8, Hkv=2, seed=72)
+    assert_scores_close(out, ref, what="full-sequence S_llm_raw, 70 sequences")
+    _no_device_error(pace)
