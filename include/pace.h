@@ -277,8 +277,12 @@ PACE_API pace_status_t pace_vit_attn_importance(const void* Q, const void* K, co
  *
  *  n_chunks        1 .. 64
  *  chunk_end_rows  host  int64 [n_chunks], nondecreasing global Q rows, the last = cu_seqlens[B]
- *  chunk_ready     host  cudaEvent_t [n_chunks] (passed as void*), recorded by the caller
+ *  chunk_ready     host  cudaEvent_t [n_chunks] (passed as void*), recorded by the caller; the
+ *                  call only enqueues waits on them, so the caller may release them afterwards
  *  other arguments as for pace_vit_attn_importance
+ *  Invalid chunks (n_chunks out of range, a null event, decreasing ends, a last end other than
+ *  cu_seqlens[B]): PACE_ERR_INVALID_ARG; anything pace_vit_attn_importance rejects: its status.
+ *  Either way before any launch or wait is enqueued.
  */
 PACE_API pace_status_t pace_vit_attn_importance_chunked(const void* Q, const void* K, const int32_t* cu_seqlens,
                                                int B, int n_heads, int head_dim, float scale, int merge,
