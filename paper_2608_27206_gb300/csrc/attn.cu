@@ -514,8 +514,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
         const int valid = CAUSAL ? min(t.nk[b] - cs, diag + qrow0 + rr - cs + 1) : t.nk[b] - cs;
         uint32_t sv[64];
         load_cols64(tbuf, sv);
+        // Warp-uniform by construction (both branches hold warp-wide TMEM loads): with a causal
+        // mask the lanes vote; without one, valid is the same for every lane and the shift is set
+        // once this pair's first tile is done (tested on j, not on m_run, which a NaN in a row's
+        // scores would make differ between lanes).
         const bool lean = CAUSAL ? __all_sync(0xffffffffu, round == 0 && valid >= 128 && m_run > -INFINITY)
-                                 : (round == 0 && valid >= 128 && m_run > -INFINITY);
+                                 : (round == 0 && valid >= 128 && j != ((p - it0) & 1));
         if (lean) {   // the common tile: both chunks full, shift already fixed
           lse_fixed_full(sv, c, m_run, la0, la1);
           load_cols64(tbuf + 64, sv);
