@@ -57,7 +57,13 @@ PACE_API const char* pace_status_string(pace_status_t status);
 PACE_API int pace_last_cuda_error(void);
 
 /* Checks that `device` is an sm_103 GPU and prepares per-device state (device
- * status word).  Optional: every entry point does the same check lazily. */
+ * status word).  Optional: every entry point does the same check lazily.
+ * Each call starts the device's set-up afresh: the status word is cleared and its
+ * address, the addresses of the library's device arrays and the kernels' shared-memory
+ * opt-ins are looked up again on the next call that needs them.  After cudaDeviceReset
+ * (or anything else that destroys the device's primary context) call pace_init again
+ * before any other call on that device; the cached values of the old context are stale.
+ * Call it while no other libpace call is in flight on that device. */
 PACE_API pace_status_t pace_init(int device);
 
 /* Reads the device status word of the current device (synchronises the device).
@@ -141,7 +147,9 @@ PACE_API pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img_o
  *    (14x14) in total per call; larger calls return PACE_ERR_INVALID_ARG and launch nothing.
  *  - d_out is required (the per-patch distances are an output, not scratch).
  *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress)
- *    with that device current; make that first call before any stream capture.
+ *    with that device current; make that first call before any stream capture.  The
+ *    address is kept until pace_init(device) is called again, which a device reset
+ *    requires (the old address belongs to the destroyed context).
  *  - Every call shares the one array and it keeps the last call's contents (the call clears
  *    the part that must start at zero).  Calls whose work overlaps on the GPU — on different
  *    streams, or from different threads — race on it; serialise them.

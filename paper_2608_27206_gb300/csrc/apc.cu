@@ -1395,14 +1395,13 @@ size_t tail_smem(const ApcTable& t) {
 }
 
 pace_status_t tail_smem_attr() {
-  static std::atomic<uint64_t> done{0};
+  static DeviceOnce once;
   int dev = 0;
   PACE_CUDA(cudaGetDevice(&dev));
-  const uint64_t bit = uint64_t{1} << (dev & 63);
-  if (!(done.load(std::memory_order_acquire) & bit)) {
+  if (!once.done(dev)) {
     PACE_CUDA(cudaFuncSetAttribute(apc_tail, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    static_cast<int>(kTailSmemMax * sizeof(float))));
-    done.fetch_or(bit, std::memory_order_acq_rel);
+    once.mark(dev);
   }
   return PACE_OK;
 }
@@ -1509,18 +1508,17 @@ static pace_status_t resample_impl(const uint8_t* src, const int64_t* src_off, c
   int sms = 1;
   {
     // opt in to the fast path's shared memory and read the SM count, once per device
-    static std::atomic<uint64_t> done{0};
+    static DeviceOnce once;
     static std::atomic<int> sm_count[64];
     int dev = 0;
     PACE_CUDA(cudaGetDevice(&dev));
-    const uint64_t bit = uint64_t{1} << (dev & 63);
-    if (!(done.load(std::memory_order_acquire) & bit)) {
+    if (!once.done(dev)) {
       int n = 0;
       PACE_CUDA(cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev));
       sm_count[dev & 63].store(n, std::memory_order_relaxed);
       PACE_CUDA(cudaFuncSetAttribute(apc_resample, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(kFSmem)));
-      done.fetch_or(bit, std::memory_order_acq_rel);
+      once.mark(dev);
     }
     sms = std::max(sm_count[dev & 63].load(std::memory_order_relaxed), 1);
   }
@@ -1578,20 +1576,23 @@ constexpr size_t kStaticBytes = kStaticInvOff + static_cast<size_t>(PACE_APC_STA
 static __device__ __align__(256) unsigned char g_apc_static_scratch[kStaticBytes];
 
 std::mutex g_static_mutex;
-void* g_static_ptr[64] = {};
+void* g_static_ptr[kMaxDevices] = {};
+DeviceOnce g_static_once;
 
 // Device address of the array for the current device.  The name g_apc_static_scratch in host
-// code is only a host-side handle, so the address is looked up once per device.
+// code is only a host-side handle, so the address is looked up once per device and set-up
+// generation (pace_init starts a new one, e.g. after cudaDeviceReset).
 pace_status_t static_scratch(unsigned char** out) {
   int dev = -1;
   PACE_CUDA(cudaGetDevice(&dev));
-  if (dev < 0 || dev >= 64) return PACE_ERR_INVALID_ARG;
+  if (dev < 0 || dev >= kMaxDevices) return PACE_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> lk(g_static_mutex);
-  if (g_static_ptr[dev] == nullptr) {
+  if (!g_static_once.done(dev)) {
     void* p = nullptr;
     PACE_CUDA(cudaGetSymbolAddress(&p, g_apc_static_scratch));
     if (p == nullptr) return set_cuda_error(cudaErrorInvalidSymbol);
     g_static_ptr[dev] = p;
+    g_static_once.mark(dev);
   }
   *out = static_cast<unsigned char*>(g_static_ptr[dev]);
   return PACE_OK;
@@ -1664,13 +1665,12 @@ namespace pace {
 namespace {
 // Opts pass 1 of the token density into two 40 KB stages (once per device).
 pace_status_t tok_pass1_attr() {
-  static std::atomic<uint64_t> done{0};
+  static DeviceOnce once;
   int dev = 0;
   PACE_CUDA(cudaGetDevice(&dev));
-  const uint64_t bit = uint64_t{1} << (dev & 63);
-  if (done.load(std::memory_order_acquire) & bit) return PACE_OK;
+  if (once.done(dev)) return PACE_OK;
   PACE_CUDA(cudaFuncSetAttribute(apc_tok_pass1, cudaFuncAttributeMaxDynamicSharedMemorySize, 2 * kTok1StageBytes));
-  done.fetch_or(bit, std::memory_order_acq_rel);
+  once.mark(dev);
   return PACE_OK;
 }
 

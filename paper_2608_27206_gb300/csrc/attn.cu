@@ -942,16 +942,15 @@ pace_status_t set_smem_attrs(size_t* s1, size_t* s2) {
   *s1 = 1024 + C::A::BYTES + C::STAGES * C::B::BYTES + sizeof(SmemCtl);
   *s2 = 1024 + C::A::BYTES + kTile * kShiftCols * 2 + C::STAGES * (C::B::BYTES + kStream * kShiftCols * 2) +
         sizeof(SmemCtl);
-  static std::atomic<uint64_t> done{0};
+  static DeviceOnce once;
   int dev = 0;
   PACE_CUDA(cudaGetDevice(&dev));
-  const uint64_t bit = uint64_t{1} << (dev & 63);
-  if (done.load(std::memory_order_acquire) & bit) return PACE_OK;
+  if (once.done(dev)) return PACE_OK;
   PACE_CUDA(cudaFuncSetAttribute(attn_row_lse<D, CAUSAL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(*s1)));
   PACE_CUDA(cudaFuncSetAttribute(attn_colsum<D, CAUSAL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(*s2)));
-  done.fetch_or(bit, std::memory_order_acq_rel);
+  once.mark(dev);
   return PACE_OK;
 }
 

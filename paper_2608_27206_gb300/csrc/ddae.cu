@@ -392,14 +392,13 @@ extern "C" pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s
   const size_t smem = static_cast<size_t>(2 * max_nv) * sizeof(float);
   {
     // opt in to the largest size once per device
-    static std::atomic<uint64_t> done{0};
+    static DeviceOnce once;
     int dev = 0;
     PACE_CUDA(cudaGetDevice(&dev));
-    const uint64_t bit = uint64_t{1} << (dev & 63);
-    if (!(done.load(std::memory_order_acquire) & bit)) {
+    if (!once.done(dev)) {
       PACE_CUDA(cudaFuncSetAttribute(ddae_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      static_cast<int>(2 * PACE_DDAE_MAX_TOKENS * sizeof(float))));
-      done.fetch_or(bit, std::memory_order_acq_rel);
+      once.mark(dev);
     }
   }
   for (int c0 = 0; c0 < B; c0 += kSelMaxB) {

@@ -10,17 +10,21 @@
 namespace pace {
 
 namespace {
-constexpr int kMaxDevices = 64;
 thread_local int t_last_cuda_error = 0;
 std::atomic<uint64_t> g_launches{0};
 std::mutex g_mutex;
 // Per-device state: 0 = not checked yet, 1 = sm_103 and initialised, 2 = unsupported.
 std::atomic<int> g_state[kMaxDevices];
 int* g_status[kMaxDevices] = {};
+std::atomic<uint32_t> g_generation[kMaxDevices];
 
 // Status word of every device that loads the library: [code, kernel id].
 __device__ int g_status_word[2];
 }  // namespace
+
+uint32_t device_generation(int dev) {
+  return (dev >= 0 && dev < kMaxDevices) ? g_generation[dev].load(std::memory_order_acquire) : 0u;
+}
 
 pace_status_t set_cuda_error(cudaError_t e) {
   t_last_cuda_error = static_cast<int>(e);
@@ -111,6 +115,11 @@ uint64_t pace_kernel_launch_count(void) { return pace::g_launches.load(std::memo
 
 pace_status_t pace_init(int device) {
   std::lock_guard<std::mutex> lk(pace::g_mutex);
+  if (device < 0 || device >= pace::kMaxDevices) return PACE_ERR_INVALID_ARG;
+  // Start a new set-up generation: the status word's address and every per-device cache of the
+  // library are looked up again (they are stale after a cudaDeviceReset).
+  pace::g_generation[device].fetch_add(1u, std::memory_order_acq_rel);
+  pace::g_state[device].store(0, std::memory_order_release);
   return pace::init_device_locked(device);
 }
 

@@ -2,6 +2,7 @@
 // per-device status word, and the sm_103 check.
 #pragma once
 #include <cuda_runtime.h>
+#include <atomic>
 #include <cstdint>
 #include <cstddef>
 
@@ -40,6 +41,28 @@ pace_status_t set_cuda_error(cudaError_t e);
 pace_status_t check_device();              // current device is sm_103 and initialised
 int* device_status_word();                 // status word of the current device
 pace_status_t check_launch();              // cudaGetLastError -> status
+
+// Generation of the library's per-device set-up.  pace_init(dev) advances it, so every cache
+// built on DeviceOnce below (function attributes, symbol addresses) is filled again on the next
+// call: after cudaDeviceReset the cached values belong to a destroyed context.
+constexpr int kMaxDevices = 64;
+uint32_t device_generation(int dev);
+
+// Per-device one-time set-up tied to the generation: done(dev) is true once mark(dev) ran in
+// the device's current generation.  Objects of this type live in static storage (zeroed).
+class DeviceOnce {
+ public:
+  bool done(int dev) const {
+    return dev >= 0 && dev < kMaxDevices &&
+           flag_[dev].load(std::memory_order_acquire) == device_generation(dev) + 1u;
+  }
+  void mark(int dev) {
+    if (dev >= 0 && dev < kMaxDevices) flag_[dev].store(device_generation(dev) + 1u, std::memory_order_release);
+  }
+
+ private:
+  std::atomic<uint32_t> flag_[kMaxDevices];
+};
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 

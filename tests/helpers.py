@@ -29,6 +29,14 @@ def assert_scores_close(got, ref, rtol=RTOL, atol_frac=1e-6, atol=0.0, what=""):
                            f"max rel err {np.max(err / np.maximum(np.abs(ref), 1e-300)):.3e}")
 
 
+def assert_distances_close(got, ref, what=""):
+    """APC distances d_i (Eq. 4): |got - ref| <= 2e-3 |ref| + 1e-5 element by element.
+
+    The 1e-5 absolute term is there for distances whose exact value is 0 (identical tokens);
+    every other d_i is held to the relative bound alone."""
+    assert_scores_close(got, ref, rtol=RTOL, atol_frac=0.0, atol=1e-5, what=what)
+
+
 def assert_kept_matches(kept_gpu, s_final_ref, K, offset=0, rtol=RTOL):
     """Kept set equals the oracle's except for tokens within rtol of the K-th score."""
     kept = np.asarray(kept_gpu, dtype=np.int64) - offset

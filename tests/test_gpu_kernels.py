@@ -11,7 +11,7 @@ import torch
 
 from oracle import pace_oracle as O
 from paper_2608_27206_gb300 import synth
-from tests.helpers import assert_kept_matches, assert_scores_close, bf16_tensor, f64
+from tests.helpers import assert_distances_close, assert_kept_matches, assert_scores_close, bf16_tensor, f64
 
 pytestmark = pytest.mark.gpu
 
@@ -76,7 +76,7 @@ def _check_density(d, st, images, alpha=0.6, gamma=1.5, tail=0.1, r_min=0.0, r_m
         assert s["n_patches"] == n and s["k_tail"] == ref["k_tail"]
         # d_i are distances between unit vectors (O(1)); 1e-5 absolute covers fp32 rounding
         # where the exact distance is 0 (identical tokens)
-        assert_scores_close(d[p0:p0 + n], ref["d"], atol_frac=2e-3, atol=1e-5, what="d_i")
+        assert_distances_close(d[p0:p0 + n], ref["d"], what="d_i")
         for k in ("phi", "d_top", "rho_d", "r"):
             assert abs(s[k] - ref[k]) <= 2e-3 * max(abs(ref[k]), 1e-3), (k, s[k], ref[k])
         assert abs(s["rho_g"] - ref["rho_g"]) <= 2e-3 * max(abs(ref["rho_g"]), 1e-3) + 2e-6
@@ -144,7 +144,7 @@ def test_density_tokens(pace, lens, D):
         ref = O.apc_density_preview(T[cu[b]:cu[b + 1]], H[b], W[b])
         s = st[b]
         assert s["n_patches"] == lens[b] and s["k_tail"] == ref["k_tail"]
-        assert_scores_close(d[cu[b]:cu[b + 1]], ref["d"], atol_frac=2e-3, atol=1e-5, what="token d_i")
+        assert_distances_close(d[cu[b]:cu[b + 1]], ref["d"], what="token d_i")
         for k in ("phi", "d_top", "rho_d", "r"):
             assert abs(s[k] - ref[k]) <= 2e-3 * max(abs(ref[k]), 1e-3), (k, s[k], ref[k])
         assert abs(s["rho"] - ref["rho"]) <= 2e-3 * max(abs(ref["rho"]), 1e-3) + 2e-6
@@ -191,7 +191,7 @@ def test_pixel_features_and_density(pace, feature):
         assert not tok[p0:p0 + n, dim:].any()
         ref = O.apc_density_pixel(im, feature)
         assert s["n_patches"] == n and s["k_tail"] == ref["k_tail"]
-        assert_scores_close(d[p0:p0 + n], ref["d"], atol_frac=2e-3, atol=1e-5, what=f"d_i ({feature})")
+        assert_distances_close(d[p0:p0 + n], ref["d"], what=f"d_i ({feature})")
         for k in ("phi", "d_top", "rho_d", "r"):
             assert abs(s[k] - ref[k]) <= 2e-3 * max(abs(ref[k]), 1e-3), (feature, k, s[k], ref[k])
         p0 += n
@@ -769,7 +769,7 @@ def test_many_images_resample_tokens_sequences(pace):
     T, cu, Ht, Wt, d, stt = _tokens_case(pace, lens, 64, seed=72, sizes=[(28 * 4, 28 * 4)] * 70)
     for b in range(70):
         ref = O.apc_density_preview(T[cu[b]:cu[b + 1]], Ht[b], Wt[b])
-        assert_scores_close(d[cu[b]:cu[b + 1]], ref["d"], atol_frac=2e-3, atol=1e-5, what="token d_i, 70 images")
+        assert_distances_close(d[cu[b]:cu[b + 1]], ref["d"], what="token d_i, 70 images")
     S = [int(x) for x in rng.integers(12, 80, 70)]
     vis = [int(rng.integers(0, s // 3)) for s in S]
     nvis = [int(rng.integers(1, s - v)) for s, v in zip(S, vis)]

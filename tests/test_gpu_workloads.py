@@ -14,7 +14,8 @@ import torch
 
 from oracle import pace_oracle as O
 from paper_2608_27206_gb300 import synth
-from tests.helpers import assert_kept_matches, assert_scores_close, f64, oracle_vit, spawn_pool
+from tests.helpers import (assert_distances_close, assert_kept_matches, assert_scores_close, f64, oracle_vit,
+                           spawn_pool)
 
 pytestmark = pytest.mark.gpu
 
@@ -61,7 +62,7 @@ def test_workload_full_size(pace, pool, name):
         oracle_sizes.append((ref["H_out"], ref["W_out"]))
         n = ref["N"]
         assert s["n_patches"] == n and s["k_tail"] == ref["k_tail"]
-        assert_scores_close(d[p0:p0 + n], ref["d"], atol_frac=2e-3, atol=1e-5, what=f"{name}[{b}] d_i")
+        assert_distances_close(d[p0:p0 + n], ref["d"], what=f"{name}[{b}] d_i")
         for k in ("phi", "d_top", "rho_d", "rho", "r"):
             assert abs(s[k] - ref[k]) <= 2e-3 * max(abs(ref[k]), 1e-3) + 2e-6, (name, b, k, s[k], ref[k])
         for side, key, exp in ((img.shape[0], "h_out", ref["H_out"]), (img.shape[1], "w_out", ref["W_out"])):
