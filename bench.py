@@ -60,21 +60,63 @@ def load_peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
+DRAM_SUMMARY = os.path.join(ROOT, "profiles", "vit_importance_img4k_dram.txt")
+ATTN_SRC = os.path.join(ROOT, "paper_2608_27206_gb300", "csrc", "attn.cu")
+DRAM_CMD = ("ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum --clock-control none "
+            "-k regex:attn_ -c 3 --csv --log-file gpurun_out/vit_dram.csv python bench.py --profile vit --reps 1")
+
+
+def source_hash():
+    return hashlib.sha256(open(ATTN_SRC, "rb").read()).hexdigest()[:16]
+
+
 def profiled_traffic():
-    """DRAM bytes per ViT-importance call from the committed ncu summary, or None when the
-    kernel source has changed since those counters were taken."""
-    path = os.path.join(ROOT, "profiles", "vit_importance_img4k.md")
-    src = os.path.join(ROOT, "paper_2608_27206_gb300", "csrc", "attn.cu")
+    """DRAM bytes per ViT-importance call from the committed ncu summary (written by
+    --write-dram-summary), or None when the kernel source has changed since those counters were
+    taken."""
     try:
-        text = open(path).read()
-        t = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
-        h = re.search(r"sha256\[:16\]\s*([0-9a-f]{16})", text)
-        cur = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        if t and h and h.group(1) == cur:
+        text = open(DRAM_SUMMARY).read()
+        t = re.search(r"^traffic_bytes_per_launch:\s*(\d+)", text, re.M)
+        h = re.search(r"^source_sha256_16:\s*([0-9a-f]{16})", text, re.M)
+        if t and h and h.group(1) == source_hash():
             return int(t.group(1))
     except OSError:
         pass
     return None
+
+
+def write_dram_summary(csv_path):
+    """Turns the ncu CSV of DRAM_CMD (one ViT call of the 4K workload) into DRAM_SUMMARY."""
+    import csv
+    rows = {}
+    with open(csv_path) as f:
+        lines = [ln for ln in f if ln.startswith('"')]
+    for r in csv.DictReader(lines):
+        name = r["Kernel Name"].split("(")[0].replace("void ", "").replace("unnamed>::", "")
+        key = (r["ID"], name)
+        rows.setdefault(key, {})[r["Metric Name"]] = float(r["Metric Value"].replace(",", ""))
+    total = 0
+    out = ["# DRAM traffic of one pace_vit_attn_importance call: the 4K workload (42196 patches, 16 heads,",
+           "# head dim 80, merge 4), one launch of each kernel, cold L2 (ncu flushes caches between kernels).",
+           "# Written by: python bench.py --write-dram-summary gpurun_out/vit_dram.csv",
+           "# Capture (the same bench.py --profile command first ran without ncu and exited 0):",
+           "#   " + DRAM_CMD,
+           "# kernel | dram read bytes | dram write bytes | time ns"]
+    for (_, name), m in sorted(rows.items(), key=lambda kv: int(kv[0][0])):
+        rd, wr = int(m.get("dram__bytes_read.sum", 0)), int(m.get("dram__bytes_write.sum", 0))
+        total += rd + wr
+        out.append(f"{name} | {rd} | {wr} | {int(m.get('gpu__time_duration.sum', 0))}")
+    q_k = 2 * 42196 * 16 * 80 * 2                       # Q and K, bf16, once
+    shift = 16 * (42196 + 256 - 42196 % 256) * 32        # shift rows written by pass 1, read by pass 2
+    alg = 2 * q_k + 2 * shift
+    out += [f"traffic_bytes_per_launch: {total}",
+            f"algorithmic_bytes_per_launch: {alg}   # Q + K read by each pass, the shift rows written and read",
+            f"traffic_over_algorithmic: {total / alg:.3f}",
+            f"source_sha256_16: {source_hash()}"]
+    with open(DRAM_SUMMARY, "w") as f:
+        f.write("\n".join(out) + "\n")
+    print("\n".join(out))
+    return 0
 
 
 def workload_config(wl, keep):
@@ -160,40 +202,73 @@ def per_image_us(total_ms: float, steps: int, world: int, images_per_step: int =
 
 
 # ----------------------------------------------------------------------------------------------
-# CPU oracle sample (the reference arm and the cpu_baseline leg)
+# CPU oracle (the reference arm and the cpu_baseline leg)
 # ----------------------------------------------------------------------------------------------
-def oracle_sample(wl, keep, vit_rows=2048, crop_div=4):
-    """Times the fp64 oracle on a bounded sample of one image and scales it to a whole image.
+def _vit_rows_job(q_bits, k_bits, scale):
+    """Pool job: the oracle's received attention of some query rows of one head (fp64)."""
+    from oracle import pace_oracle as O
+    from paper_2608_27206_gb300 import synth
+    return O.received_attention(synth.bf16_bits_to_f64(q_bits), synth.bf16_bits_to_f64(k_bits), scale)
 
-    density : oracle on a centred crop with 1/crop_div of each side, scaled by (N/N_crop)^2
-              (Eq. 1 is a double sum over all token pairs);
-    resample: whole image to the oracle's target size;
-    S_vis   : one head, the first vit_rows query rows against all keys, scaled by
-              heads x N / vit_rows;
-    S_llm, fusion, top-K, gather: whole image.
+
+def oracle_pool(n=None):
+    """Spawn pool over the host cores (spawn: never forked from a process that uses CUDA)."""
+    import multiprocessing as mp
+    n = n or os.cpu_count() or 4
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ.setdefault(k, "1")
+    return mp.get_context("spawn").Pool(n), n
+
+
+def oracle_timing(wl, keep, pool, vit_rows, density_crop_div=1):
+    """Times the fp64 oracle on one 4K image of the workload, on the host cores.
+
+    density : the whole image (density_crop_div = 1: Eq. 1 summed over all N^2 pairs), or a
+              centred crop with 1/density_crop_div of each side, scaled by (N / N_crop)^2;
+    resample: the whole image to the oracle's target size;
+    S_vis   : every head, the first vit_rows query rows of each against all keys, one job per head
+              on the pool; scaled by N / vit_rows (the rows' softmaxes are independent, so the work
+              is exactly proportional to the rows);
+    S_llm, fusion, top-K, gather: the whole image.
+    Returns (seconds per image, measured seconds, parts, description).
     """
     from oracle import pace_oracle as O
     from paper_2608_27206_gb300 import synth
     img = wl.images[0]
     H, W = img.shape[:2]
-    t = {}
-    ch, cw = (H // crop_div) // 14 * 14, (W // crop_div) // 14 * 14
-    y0, x0 = (H - ch) // 2 // 14 * 14, (W - cw) // 2 // 14 * 14
-    crop = np.ascontiguousarray(img[y0:y0 + ch, x0:x0 + cw])
-    n_full, n_crop = (H // 14) * (W // 14), (ch // 14) * (cw // 14)
-    t0 = time.perf_counter()
-    O.apc_density(crop)
-    t["density"] = (time.perf_counter() - t0) * (n_full / n_crop) ** 2
-    st = O.apc_density_tokens(O.patch_tokens(crop))
-    ho, wo = O.target_size(H, W, O.retention_ratio(st["rho"]))
+    t, measured = {}, 0.0
+    if density_crop_div > 1:
+        ch, cw = (H // density_crop_div) // 14 * 14, (W // density_crop_div) // 14 * 14
+        y0, x0 = (H - ch) // 2 // 14 * 14, (W - cw) // 2 // 14 * 14
+        crop = np.ascontiguousarray(img[y0:y0 + ch, x0:x0 + cw])
+        n_full, n_crop = (H // 14) * (W // 14), (ch // 14) * (cw // 14)
+        t0 = time.perf_counter()
+        st = O.apc_density(crop)
+        dt = time.perf_counter() - t0
+        t["density"] = dt * (n_full / n_crop) ** 2
+        ho, wo = O.target_size(H, W, O.retention_ratio(st["rho"]))
+        dens_desc = f"density on a {cw}x{ch} centre crop scaled by (N/N_crop)^2"
+    else:
+        t0 = time.perf_counter()
+        st = O.apc_density(img)
+        dt = time.perf_counter() - t0
+        t["density"] = dt
+        ho, wo = st["H_out"], st["W_out"]
+        dens_desc = "density of the whole image"
+    measured += dt
     t0 = time.perf_counter()
     O.apc_resample(img, ho, wo)
     t["resample"] = time.perf_counter() - t0
-    q = synth.bf16_bits_to_f64(wl.vit_q[:vit_rows, 0])
-    k = synth.bf16_bits_to_f64(wl.vit_k[:, 0])
+    measured += t["resample"]
+    n, heads = wl.vit_q.shape[0], wl.vit_q.shape[1]
+    R = min(vit_rows, n)
+    jobs = [(np.ascontiguousarray(wl.vit_q[:R, h]), np.ascontiguousarray(wl.vit_k[:, h]), 1 / math.sqrt(80))
+            for h in range(heads)]
     t0 = time.perf_counter()
-    O.received_attention(q, k, 1 / math.sqrt(80))
-    t["vit"] = (time.perf_counter() - t0) * wl.vit_q.shape[1] * (wl.vit_q.shape[0] / vit_rows)
+    pool.starmap(_vit_rows_job, jobs, chunksize=1)
+    dt = time.perf_counter() - t0
+    t["vit"] = dt * n / R
+    measured += dt
     ql, kl = synth.bf16_bits_to_f64(wl.llm_q), synth.bf16_bits_to_f64(wl.llm_k)
     t0 = time.perf_counter()
     s_llm = O.llm_text_visual_importance(ql, kl, wl.cu_q, wl.cu_vis, 1 / math.sqrt(128))
@@ -206,11 +281,11 @@ def oracle_sample(wl, keep, vit_rows=2048, crop_div=4):
     t0 = time.perf_counter()
     O.gather_rows(wl.embed, sel["kept"])
     t["gather"] = time.perf_counter() - t0
-    total = sum(t.values())
-    sample = (f"fp64 numpy oracle on the host cores: density on a {cw}x{ch} centre crop scaled by (N/N_crop)^2, "
-              f"resample of the whole image, S_vis for 1 of 16 heads x {vit_rows} of {wl.vit_q.shape[0]} query rows "
-              f"scaled linearly, S_llm / fusion / top-K / gather on the whole image")
-    return total, t, sample
+    measured += t["llm"] + t["select"] + t["gather"]
+    desc = (f"fp64 numpy oracle on {pool._processes} host processes: {dens_desc}; resample of the whole image; "
+            f"S_vis for all {heads} heads x the first {R} of {n} query rows (one pool job per head), scaled "
+            f"by {n}/{R}; S_llm, fusion, top-K, gather of the whole image")
+    return sum(t.values()), measured, t, desc
 
 
 def run_reference(args):
@@ -219,21 +294,30 @@ def run_reference(args):
         return 0
     from paper_2608_27206_gb300 import synth
     wl = synth.make_workload(WORKLOAD, seed=0, keep=KEEP, parts=("image", "vit", "llm", "embed"))
-    for _ in range(args.warmup):
-        oracle_sample(wl, KEEP, vit_rows=args.ref_vit_rows)
-    times, parts, sample = [], None, ""
-    for _ in range(args.steps):
-        tot, parts, sample = oracle_sample(wl, KEEP, vit_rows=args.ref_vit_rows)
-        times.append(tot)
-    per_image_s = float(np.mean(times))
-    value = per_image_s * 1e6
+    pool, cores = oracle_pool()
+    try:
+        # each step is a bounded sample of the image's work (a few seconds on the host cores)
+        for _ in range(args.warmup):
+            oracle_timing(wl, KEEP, pool, args.ref_vit_rows, density_crop_div=4)
+        per_image, sample_s, parts, sample = [], [], None, ""
+        for _ in range(args.steps):
+            tot, meas, parts, sample = oracle_timing(wl, KEEP, pool, args.ref_vit_rows, density_crop_div=4)
+            per_image.append(tot)
+            sample_s.append(meas)
+    finally:
+        pool.close()
+        pool.join()
+    value = float(np.mean(per_image)) * 1e6
+    ms_step = float(np.mean(sample_s)) * 1e3
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_image_s * 1e3, "higher_is_better": False,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": False,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(wl, KEEP),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample,
-                         "parts_s": {k: round(v, 4) for k, v in parts.items()}},
+        "images_per_step": round(ms_step * 1e3 / value, 6),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample,
+                         "sample_seconds_per_step": round(ms_step * 1e-3, 3),
+                         "parts_s_per_image": {k: round(v, 4) for k, v in parts.items()}},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -409,6 +493,162 @@ def measure_next_rows(P, device, flush, peak_tf, hbm_gbs, reps=10):
     return out
 
 
+def workload_counts(wl, stats_rows):
+    """Algorithmic flops / bytes of one step over all images of a workload, per part.  stats_rows:
+    the device density statistics of every image (target sizes of the resample)."""
+    n = wl.n_patches
+    nv = wl.n_vis
+    K = [int(math.floor(s.keep * v + 0.5)) for s, v in zip(wl.specs, nv)]
+    img = [s.H * s.W * 3 for s in wl.specs]
+    out = [st["h_out"] * st["w_out"] * 3 for st in stats_rows]
+    return {
+        "vit_flops": sum(2 * 2 * x * x * 80 * 16 for x in n),
+        "llm_flops": sum(2 * 2 * s.tq * 28 * v * 128 for s, v in zip(wl.specs, nv)),
+        "density_bytes": sum(img) + 4 * sum(n),
+        "resample_bytes": sum(img) + sum(out),
+        "select_bytes": sum(3 * 4 * v for v in nv) + 4 * sum(K),
+        "gather_bytes": 2 * sum(K) * 3584 * 2,
+    }
+
+
+def part_rooflines(cnt, part_us, peak_tf, hbm):
+    out = {}
+    for name, key, bound in (("density", "density_bytes", "hbm"), ("resample", "resample_bytes", "hbm"),
+                             ("vit", "vit_flops", "tensor"), ("llm", "llm_flops", "tensor"),
+                             ("select", "select_bytes", "hbm"), ("gather", "gather_bytes", "hbm")):
+        sec = part_us[name] * 1e-6
+        if bound == "hbm":
+            a = cnt[key] / sec / 1e9
+            out[name] = {"bound": "hbm", "us": round(part_us[name], 2), "achieved": round(a, 1), "unit": "GB/s",
+                         "frac": round(a / hbm, 4), "bytes": cnt[key]}
+        else:
+            a = cnt[key] / sec / 1e12
+            out[name] = {"bound": "tensor", "us": round(part_us[name], 2), "achieved": round(a, 1),
+                         "unit": "TFLOP/s", "frac": round(a / peak_tf, 4), "flops": cnt[key]}
+    return out
+
+
+def time_graphs(graphs, flush, steps):
+    """Per-part and per-step CUDA-event times (ms) of `steps` replays, L2 flushed before each."""
+    import torch
+    nparts = len(graphs)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nparts + 1)] for _ in range(steps)]
+    for k in range(steps):
+        flush.zero_()
+        ev[k][0].record()
+        for i, (_, g) in enumerate(graphs):
+            g.replay()
+            ev[k][i + 1].record()
+    torch.cuda.synchronize()
+    part = {name: statistics.mean(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(steps))
+            for i, (name, _) in enumerate(graphs)}
+    step = statistics.mean(ev[k][0].elapsed_time(ev[k][nparts]) for k in range(steps))
+    return part, step
+
+
+def measure_configs(P, device, flush, peak_tf, hbm, steps=10):
+    """The other workloads of the benchmark (448^2, 1344^2, 1904x1064 with sinks, the ragged
+    16-image batch): the whole step through HotPath, each call replayed from a CUDA graph, L2
+    flushed before every step; microseconds per image, the per-call breakdown and each call's
+    roofline fraction."""
+    import torch
+    from paper_2608_27206_gb300 import synth
+    from paper_2608_27206_gb300.hotpath import HotPath
+    out = {}
+    for name in ("img448", "img1344", "frame1904", "ragged16"):
+        wl = synth.make_workload(name, seed=0)
+        pipe = HotPath(wl, device)
+        graphs = capture_graphs(pipe)
+        for _ in range(3):
+            flush.zero_()
+            for _, g in graphs:
+                g.replay()
+        torch.cuda.synchronize()
+        part_ms, step_ms = time_graphs(graphs, flush, steps)
+        code, where = P.pace_device_status(clear=True)
+        if code != 0:
+            raise RuntimeError(f"device status {code} from kernel {where} in config {name}")
+        cnt = workload_counts(wl, P.stats_dict(pipe.stats[: wl.B]))
+        part_us = {k: v * 1e3 for k, v in part_ms.items()}
+        out[name] = {"images": wl.B, "us_per_image": round(step_ms * 1e3 / wl.B, 2),
+                     "us_per_step": round(step_ms * 1e3, 2),
+                     "visual_tokens": int(sum(wl.n_vis)), "patches": int(sum(wl.n_patches)),
+                     "breakdown_us": {k: round(v, 2) for k, v in part_us.items()},
+                     "rooflines": part_rooflines(cnt, part_us, peak_tf, hbm)}
+        del pipe, graphs
+        torch.cuda.empty_cache()
+    return out
+
+
+def measure_batched(P, device, flush, hbm, n_img=8, reps=10):
+    """The bandwidth-bound calls on a batch of n_img 4K images in one call each (198 MB of pixels,
+    larger than L2): density, resample to the density's target sizes, and the gather of 10 % of
+    each image's embedding rows.  Each call replayed from a CUDA graph, L2 flushed before every
+    replay, median of reps."""
+    import torch
+    from paper_2608_27206_gb300 import synth
+    H, W = 2156, 3836
+    imgs = [synth.make_image(np.random.default_rng([77, i]), H, W, 32, 18, 0.15) for i in range(n_img)]
+    buf, off = synth.pack_images(imgs)
+    src = torch.from_numpy(buf).to(device)
+    Hs, Ws = [H] * n_img, [W] * n_img
+    n = (H // 14) * (W // 14)
+    d = torch.empty(n * n_img, dtype=torch.float32, device=device)
+    st = torch.zeros((n_img, 10), dtype=torch.int32, device=device)
+    ws = torch.empty(P.pace_apc_density_workspace_size(Hs, Ws), dtype=torch.uint8, device=device)
+    dst = torch.empty_like(src)
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        s_ = torch.cuda.Stream(device)
+        with torch.cuda.stream(s_):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s_):
+                fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        return statistics.median(ts) * 1e-3
+
+    out = {}
+    sec = timed(lambda: P.pace_apc_density(src, off, Hs, Ws, d_out=d, stats=st, ws=ws))
+    nbytes = n_img * (H * W * 3 + 4 * n)
+    out[f"density_{n_img}x4k"] = {"us": round(sec * 1e6, 2), "bytes": nbytes, "achieved": round(nbytes / sec / 1e9, 1),
+                                  "unit": "GB/s", "frac": round(nbytes / sec / 1e9 / hbm, 4), "bound": "hbm"}
+    sd = P.stats_dict(st)
+    sec = timed(lambda: P.pace_apc_resample(src, off, Hs, Ws, st, dst, off))
+    nbytes = n_img * H * W * 3 + sum(x["h_out"] * x["w_out"] * 3 for x in sd)
+    out[f"resample_{n_img}x4k"] = {"us": round(sec * 1e6, 2), "bytes": nbytes,
+                                   "achieved": round(nbytes / sec / 1e9, 1), "unit": "GB/s",
+                                   "frac": round(nbytes / sec / 1e9 / hbm, 4), "bound": "hbm",
+                                   "target": [sd[0]["h_out"], sd[0]["w_out"]]}
+    del src, dst, d, ws
+    nv = (H // 28) * (W // 28)
+    emb = (torch.randn(n_img * nv, 3584, device=device) * 0.5).to(torch.bfloat16)
+    g = torch.Generator(device=device)
+    g.manual_seed(5)
+    keep = P.pace_budget(nv, 0.10)
+    idx = torch.cat([torch.sort(torch.randperm(nv, generator=g, device=device)[:keep])[0] + i * nv
+                     for i in range(n_img)]).to(torch.int32)
+    rows = torch.empty(idx.numel(), 3584, dtype=torch.bfloat16, device=device)
+    sec = timed(lambda: P.pace_gather(emb, idx, dst=rows))
+    nbytes = 2 * idx.numel() * 3584 * 2
+    out[f"gather_{n_img}x4k"] = {"us": round(sec * 1e6, 2), "bytes": nbytes, "achieved": round(nbytes / sec / 1e9, 1),
+                                 "unit": "GB/s", "frac": round(nbytes / sec / 1e9 / hbm, 4), "bound": "hbm",
+                                 "rows": int(idx.numel())}
+    del emb, rows, idx
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
@@ -548,11 +788,19 @@ def run_gpu(args):
         other["llm"] = {"bound": "tensor", "us": round(mean["llm"] * 1e3, 2), "achieved": round(llm_tf, 1),
                         "peak": peak, "unit": "TFLOP/s", "frac": round(llm_tf / peak, 4), "flops": cnt["llm_flops"]}
         nxt = measure_next_rows(P, device, flush, peak, hbm) if world == 1 and not args.no_next_rows else None
+        cfgs = measure_configs(P, device, flush, peak, hbm) if world == 1 and not args.no_configs else None
+        batched = measure_batched(P, device, flush, hbm) if world == 1 and not args.no_configs else None
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
-            tot, parts, sample = oracle_sample(wl, KEEP, vit_rows=args.ref_vit_rows)
-            cpu = {"value": tot * 1e6, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle", "sample": sample,
-                   "parts_s": {k: round(v, 4) for k, v in parts.items()}}
+            pool, cores = oracle_pool()
+            try:
+                vit_rows = wl.vit_q.shape[0] if args.cpu_full else args.cpu_vit_rows
+                tot, meas, parts, sample = oracle_timing(wl, KEEP, pool, vit_rows, density_crop_div=1)
+            finally:
+                pool.close()
+                pool.join()
+            cpu = {"value": tot * 1e6, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample,
+                   "measured_seconds": round(meas, 3), "parts_s_per_image": {k: round(v, 4) for k, v in parts.items()}}
         line = {
             "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": False,
@@ -560,7 +808,7 @@ def run_gpu(args):
             "config": workload_config(wl, KEEP),
             "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
                          "frac": round(achieved / peak, 4), "traffic": profiled_traffic(),
-                         "traffic_unit": "bytes per call (ncu dram read+write, profiles/vit_importance_img4k.md)",
+                         "traffic_unit": "bytes per call (ncu dram read+write, profiles/vit_importance_img4k_dram.txt)",
                          "kernel": "ViT received attention (attn_row_lse + attn_colsum + attn_reduce), one launch "
                                    "of pace_vit_attn_importance",
                          "algorithmic_flops": cnt["vit_flops"], "us": round(vit_ms * 1e3, 1),
@@ -574,6 +822,8 @@ def run_gpu(args):
                          "peak_source": f"{peak_src} bf16 dense burst (MEASURED_PEAKS.json)"
                          if peak_src == "measured" else "fallback 1.9 PFLOP/s bf16"},
             "rooflines_other": other,
+            "rooflines_batched": batched,
+            "configs_other": cfgs,
             "next_rows": nxt,
             "breakdown_us": {k: round(v * 1e3, 2) for k, v in mean.items()},
             "visual_tokens_scored_per_s": round(wl.n_vis[0] * world / (ms_per_step * 1e-3), 1),
@@ -625,14 +875,25 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--ref-vit-rows", type=int, default=2048)
+    ap.add_argument("--ref-vit-rows", type=int, default=512,
+                    help="query rows per head of the reference arm's per-step oracle sample")
+    ap.add_argument("--cpu-vit-rows", type=int, default=2048,
+                    help="query rows per head of the cpu_baseline oracle sample")
+    ap.add_argument("--cpu-full", action="store_true",
+                    help="cpu_baseline: run the oracle on the whole image (all query rows; minutes)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next-rows", action="store_true", help="skip the timing of the NEXT-row calls")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other workloads and the batched bandwidth measurements")
     ap.add_argument("--profile", choices=("density", "resample", "vit", "llm", "select", "gather"),
                     help="run only this call --reps times (for profiler captures)")
     ap.add_argument("--reps", type=int, default=1)
     ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--write-dram-summary", metavar="NCU_CSV",
+                    help="write the committed DRAM-traffic summary of the ViT call from an ncu CSV capture")
     args = ap.parse_args()
+    if args.write_dram_summary:
+        return write_dram_summary(args.write_dram_summary)
     if args.profile:
         return run_profile(args)
     if args.warmup < 3:

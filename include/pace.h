@@ -381,9 +381,6 @@ PACE_API void pace_ddae_params_default(pace_ddae_params* params);
 /* Token budget K = floor(frac * n_vis + 0.5), clamped to [0, n_vis]. */
 PACE_API int32_t pace_budget(int32_t n_vis, double frac);
 
-/* Largest visual-token count per image accepted by pace_ddae_select. */
-#define PACE_DDAE_MAX_TOKENS 24576
-
 /*
  * DDAE fusion and top-K (Sec. 3.3, Eq. 7).  Per image b: S_llm, S_vis = min-max
  * normalised maps (a constant map becomes 0); sigma = population standard deviation;
@@ -391,9 +388,16 @@ PACE_API int32_t pace_budget(int32_t n_vis, double frac);
  * params' fusion mode);
  * S_final = alpha_w S_llm + beta_w S_vis; keep the K_b = cu_keep[b+1] - cu_keep[b]
  * highest S_final (ties: lower index first), written in ascending index order.
+ * One CTA per map; maps of up to 12288 tokens keep their scores in registers, larger ones
+ * (any size) read them again for each pass, with identical results.
+ * Raw scores must be finite: a NaN or infinite raw score records PACE_ERR_INVALID_ARG (kernel
+ * id 9) in the device status word.  The map's S_final and weights are then not meaningful
+ * (the value reaches the normalisation and the Eq. 7 weights), but kept still receives K_b
+ * distinct indices of the map in ascending order: a NaN fused score ranks below every other
+ * score, ties going to the lower index.
  *
  *  s_llm_raw, s_vis_raw  device  float [sum Nv]
- *  cu_v      host    int32 [B+1]; 1 <= Nv_b <= PACE_DDAE_MAX_TOKENS
+ *  cu_v      host    int32 [B+1]; Nv_b >= 1
  *  cu_keep   host    int32 [B+1]; 0 <= K_b <= Nv_b
  *  params    host    NULL for tau = 0.5
  *  s_final   device  float [sum Nv] (may be NULL)

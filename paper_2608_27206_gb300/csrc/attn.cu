@@ -340,6 +340,25 @@ __device__ __forceinline__ void colsum64_from(const uint32_t (&v)[64], int lo, f
   colsum64(w, c, a0, a1);
 }
 
+// Overwrites query rows rows .. kStream - 1 of a staged pass-2 tile with zeros: the 128-byte rows
+// of its 64-column blocks and the 32-byte rows of its 16-column slices (a swizzle only moves
+// 16-byte pieces within their own row), by the 32 lanes of a warp.  The shift slice keeps the
+// padded rows' -2^100, so these rows add exactly 0 to every key's sum.
+template <int D>
+__device__ __forceinline__ void zero_stage_rows(uint8_t* st, int rows) {
+  using F = TileFmt<D, kStream>;
+  constexpr int PIECES = F::NB * 8 + F::R * 2;   // 16-byte pieces per row
+  const int lane = threadIdx.x & 31;
+  const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+  for (int i = lane; i < (kStream - rows) * PIECES; i += 32) {
+    const int row = rows + i / PIECES, pc = i % PIECES;
+    uint8_t* dst = pc < F::NB * 8 ? st + (pc >> 3) * F::BLOCK + row * 128 + (pc & 7) * 16
+                                  : st + F::NB * F::BLOCK + ((pc - F::NB * 8) >> 1) * F::SLICE + row * 32 +
+                                        ((pc - F::NB * 8) & 1) * 16;
+    *reinterpret_cast<uint4*>(dst) = z;
+  }
+}
+
 // Brings the CTA to a quiet point: waits for its MMAs (phase `done_phase` of b_done) and lets
 // in-flight copies land after an abort; TMEM stays allocated.
 __device__ __forceinline__ void cta_quiesce(SmemCtl* ctl, uint32_t b_done, uint32_t done_phase, int* status,
@@ -410,6 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
   const int kt1_all = static_cast<int>((static_cast<int64_t>(split + 1) * nkt_all) / t.splits);
   const int kt1 = CAUSAL ? min(kt1_all, (diag + qrow0 + kTile - 1) / kStream + 1) : kt1_all;
   const int nj = max(kt1 - kt0, 0);
+  const int pre = min(nj, ST);   // key stages issued in the prologue (round 0, first use of each stage)
 
   if (threadIdx.x == 0) {
     mbar_init(b_qfull, 1);
@@ -425,6 +445,21 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
     ctl->abort = 0;
     ctl->redo = 0;
     fence_mbar_init();
+    // The query tile and the first key stages are requested before the CTA-wide barrier below,
+    // so their latency overlaps the TMEM allocation (the barriers are initialised and fenced
+    // by this thread; nobody else touches them before that barrier).
+    prefetch_tensormap(&tmq);
+    prefetch_tensormap(&tmk);
+    if (C::A::R > 0) {
+      prefetch_tensormap(&tmq32);
+      prefetch_tensormap(&tmk32);
+    }
+    mbar_arrive_expect_tx(b_qfull, C::A::BYTES);
+    load_tile<D, kTile>(sQ, &tmq, &tmq32, h * D, t.q0[b] + qrow0, b_qfull);
+    for (int j = 0; j < pre; ++j) {
+      mbar_arrive_expect_tx(b_kfull(j), C::B::BYTES);
+      load_tile<D, kStream>(sK + j * C::B::BYTES, &tmk, &tmk32, g * D, t.k0[b] + (kt0 + j) * kStream, b_kfull(j));
+    }
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(&ctl->tmem_base), kTmemCols);
@@ -442,21 +477,11 @@ __global__ void __launch_bounds__(kThreads, 1) attn_row_lse(const __grid_constan
   const int p = e >> 1, hh = e & 1;
   const int quad = warp & 3;
   const int rr = quad * 32 + lane;
-  if (warp == 0 && lane == 0) {
-    prefetch_tensormap(&tmq);
-    prefetch_tensormap(&tmk);
-    if (C::A::R > 0) {
-      prefetch_tensormap(&tmq32);
-      prefetch_tensormap(&tmk32);
-    }
-    mbar_arrive_expect_tx(b_qfull, C::A::BYTES);
-    load_tile<D, kTile>(sQ, &tmq, &tmq32, h * D, t.q0[b] + qrow0, b_qfull);
-  }
   auto run_round = [&](int round) {
     const int it0 = round * nj;
     if (warp == 0) {
       if (lane == 0) {
-        for (int j = 0; j < nj; ++j) {
+        for (int j = round == 0 ? pre : 0; j < nj; ++j) {
           const int it = it0 + j;
           const int s = it % ST, u = it / ST;
           if (u > 0 && !mbar_wait(b_kempty(s), (u - 1) & 1, kWaitLimitNs)) {
@@ -642,6 +667,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
   auto b_qempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };
   auto b_sfull = [&](int p) { return smem_u32(&ctl->bars[2 + 2 * ST + p]); };
   auto b_sfree = [&](int p) { return smem_u32(&ctl->bars[4 + 2 * ST + p]); };
+  // stage s is ready for the MMA beyond its copy: every stage use gets one arrival, right after the
+  // copy is issued, or once the rows past the image have been zeroed on an image's ragged last tile
+  auto b_fixed = [&](int s) { return smem_u32(&ctl->bars[6 + 2 * ST + s]); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = blockIdx.x & 1u;       // which 128-row half of the item
@@ -658,6 +686,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
   const int qt_min = CAUSAL && krow0 > diag ? (krow0 - diag) / kStream : 0;
   const int nspan = max(nqt - qt_min, 0);
   const int nj = t.G * nspan;                                         // stream: (head in group, query tile)
+  // query rows of stream tile j that lie inside the image (kStream unless it is the image's last
+  // tile and the image ends inside it)
+  auto ragged_rows = [&](int j) { return min(kStream, t.nq[b] - (qt_min + j % nspan) * kStream); };
 
   if (threadIdx.x == 0) {
     mbar_init(b_afull, 1);
@@ -670,8 +701,38 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
       mbar_init(b_sfull(p), 1);
       mbar_init(b_sfree(p), 8);
     }
+    for (int s = 0; s < ST; ++s) mbar_init(b_fixed(s), 1);
     ctl->abort = 0;
     fence_mbar_init();
+  }
+  // stage s of stream item j: query tile (head in group, query tile) plus its shift slice
+  auto issue_stage = [&](int j, int s) {
+    const int hq = j / nspan, qt = qt_min + j - hq * nspan;
+    const int h = g * t.G + hq;
+    uint8_t* st = sQ + s * B2;
+    mbar_arrive_expect_tx(b_qfull(s), B2);
+    load_tile<D, kStream>(st, &tmq, &tmq32, h * D, t.q0[b] + qt * kStream, b_qfull(s));
+    const int srow = h * t.prows + t.lpad[b] + qt * kStream;
+#pragma unroll
+    for (int q = 0; q < kStream / kTile; ++q)
+      tma_load_2d(smem_u32(st + C::B::BYTES + q * kTile * kShiftCols * 2), &tmshift, 0, srow + q * kTile,
+                  b_qfull(s));
+  };
+  const int pre = min(nj, ST);   // query stages issued in the prologue (first use of each stage)
+  if (threadIdx.x == 0) {
+    // the resident key tile and the first query stages are requested before the CTA-wide
+    // barrier, so their latency overlaps the TMEM allocation
+    prefetch_tensormap(&tmq);
+    prefetch_tensormap(&tmk);
+    if (C::A::R > 0) {
+      prefetch_tensormap(&tmq32);
+      prefetch_tensormap(&tmk32);
+    }
+    prefetch_tensormap(&tmshift);
+    mbar_arrive_expect_tx(b_afull, A2);
+    load_tile<D, kTile>(sA, &tmk, &tmk32, g * D, t.k0[b] + krow0, b_afull);
+    tma_load_2d(smem_u32(sA + C::A::BYTES), &tmones, 0, 0, b_afull);
+    for (int j = 0; j < pre; ++j) issue_stage(j, j);
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(&ctl->tmem_base), kTmemCols);
@@ -683,35 +744,39 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
   const uint32_t tmem = ctl->tmem_base;
 
   if (warp == 0) {
-    if (lane == 0) {
-      prefetch_tensormap(&tmq);
-      prefetch_tensormap(&tmk);
-      if (C::A::R > 0) {
-        prefetch_tensormap(&tmq32);
-        prefetch_tensormap(&tmk32);
-      }
-      prefetch_tensormap(&tmshift);
-      mbar_arrive_expect_tx(b_afull, A2);
-      load_tile<D, kTile>(sA, &tmk, &tmk32, g * D, t.k0[b] + krow0, b_afull);
-      tma_load_2d(smem_u32(sA + C::A::BYTES), &tmones, 0, 0, b_afull);
-      for (int j = 0; j < nj; ++j) {
-        const int s = j % ST, u = j / ST;
+    // The whole warp walks the stream: lane 0 issues the copies; on an image's last query tile,
+    // when it holds rows past the image, all lanes overwrite those rows with zeros once the copy
+    // has landed (they belong to the next image and may hold inf or NaN, which the -2^100 shift of
+    // a padded row would not cancel), and then release the tile to the MMA.
+    for (int j = 0; j < nj; ++j) {
+      const int s = j % ST, u = j / ST;
+      int ok = 1;
+      if (j >= pre && lane == 0) {
         if (u > 0 && !mbar_wait(b_qempty(s), (u - 1) & 1, kWaitLimitNs)) {
           set_abort(ctl, status, K_ATTN_COLSUM);
-          break;
+          ok = 0;
+        } else if (aborted(ctl)) {
+          ok = 0;
+        } else {
+          issue_stage(j, s);
         }
-        if (aborted(ctl)) break;
-        const int hq = j / nspan, qt = qt_min + j - hq * nspan;
-        const int h = g * t.G + hq;
-        uint8_t* st = sQ + s * B2;
-        mbar_arrive_expect_tx(b_qfull(s), B2);
-        load_tile<D, kStream>(st, &tmq, &tmq32, h * D, t.q0[b] + qt * kStream, b_qfull(s));
-        const int srow = h * t.prows + t.lpad[b] + qt * kStream;
-#pragma unroll
-        for (int q = 0; q < kStream / kTile; ++q)
-          tma_load_2d(smem_u32(st + C::B::BYTES + q * kTile * kShiftCols * 2), &tmshift, 0, srow + q * kTile,
-                      b_qfull(s));
       }
+      const int rows = ragged_rows(j);
+      if (rows < kStream) {
+        if (lane == 0 && ok && !mbar_wait(b_qfull(s), u & 1, kWaitLimitNs)) {
+          set_abort(ctl, status, K_ATTN_COLSUM);
+          ok = 0;
+        }
+        if (__shfl_sync(0xffffffffu, ok, 0)) {
+          zero_stage_rows<D>(sQ + s * B2, rows);
+          fence_proxy_async_shared();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(b_fixed(s));
+        }
+      } else if (lane == 0 && ok) {
+        mbar_arrive(b_fixed(s));
+      }
+      if (!__shfl_sync(0xffffffffu, ok, 0)) break;
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -727,6 +792,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
         const int p = j & 1, v = j >> 1;
         if (!mbar_wait(b_qfull(s), u & 1, kWaitLimitNs) ||
             (v > 0 && !mbar_wait(b_sfree(p), (v - 1) & 1, kWaitLimitNs)) || aborted(ctl)) {
+          set_abort(ctl, status, K_ATTN_COLSUM);
+          break;
+        }
+        if (!mbar_wait(b_fixed(s), u & 1, kWaitLimitNs)) {
           set_abort(ctl, status, K_ATTN_COLSUM);
           break;
         }

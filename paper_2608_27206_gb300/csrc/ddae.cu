@@ -14,19 +14,29 @@
 #include <cmath>
 
 #include "pace_common.cuh"
-#include "pace_select.cuh"
 
 namespace pace {
 namespace {
 
 constexpr int kSelThreads = 1024;
+constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kSelMaxB = 256;
+constexpr int kSelBins = 4096;           // bins of one selection round (4 per thread)
+constexpr int kSelRegMax = 12;           // scores per thread held in registers (12288 per map)
 
 struct SelectTable {
   int v0[kSelMaxB];  // first global row of image b
   int nv[kSelMaxB];  // visual tokens of image b
   int k0[kSelMaxB];  // first output slot of image b
   int nk[kSelMaxB];  // tokens kept for image b
+};
+
+struct SelShared {
+  float red[3][4][kSelWarps];   // warp partials of the three block reductions
+  unsigned bins[kSelBins];      // histogram of the current selection round
+  unsigned wtot[kSelWarps];     // per-warp totals (bin prefix, compaction scans)
+  unsigned wtot2[kSelWarps];
+  unsigned sel[2];              // selected bin, entries in the bins above it
 };
 
 __device__ __forceinline__ float warp_min(float v) {
@@ -44,81 +54,185 @@ __device__ __forceinline__ float warp_sum(float v) {
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
-
-// Block-wide reduction of two values; every thread gets the result.  `red` holds 2*32 floats.
-template <int OP>  // 0 = sum, 1 = min, 2 = max
-__device__ __forceinline__ float2 block_reduce2(float a, float b, float* red) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  if (OP == 0) { a = warp_sum(a); b = warp_sum(b); }
-  if (OP == 1) { a = warp_min(a); b = warp_min(b); }
-  if (OP == 2) { a = warp_max(a); b = warp_max(b); }
-  __syncthreads();
-  if (lane == 0) { red[warp] = a; red[32 + warp] = b; }
-  __syncthreads();
-  if (warp == 0) {
-    a = red[lane];
-    b = red[32 + lane];
-    if (OP == 0) { a = warp_sum(a); b = warp_sum(b); }
-    if (OP == 1) { a = warp_min(a); b = warp_min(b); }
-    if (OP == 2) { a = warp_max(a); b = warp_max(b); }
-    if (lane == 0) { red[0] = a; red[32] = b; }
+__device__ __forceinline__ unsigned warp_incl_scan(unsigned v) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const unsigned n = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += n;
   }
-  __syncthreads();
-  return make_float2(red[0], red[32]);
+  return v;
 }
 
+// Selection key of a fused score: its bit pattern (integer order = float order for values > 0);
+// zero, negative and NaN scores take key 0, below every positive score.
+__device__ __forceinline__ unsigned sel_key(float f) { return f > 0.f ? __float_as_uint(f) : 0u; }
+
+// Value bucket of a key for the first selection round: floor(4096 f), capped at the top bucket
+// (monotone in the key; S_final lies in [0, 1]).
+__device__ __forceinline__ unsigned sel_bucket(unsigned key) {
+  return min(__float2uint_rz(__uint_as_float(key) * 4096.0f), static_cast<unsigned>(kSelBins - 1));
+}
+
+// The bin holding the r-th largest entry of sh.bins, counting from bin 4095 down (1 <= r <= total):
+// sh.sel[0] = that bin, sh.sel[1] = entries in the bins above it.  Every thread of the block calls
+// it; thread t owns bins 4095 - 4t .. 4092 - 4t.  Ends with the result visible to all threads.
+__device__ __forceinline__ void sel_bin_from_top(SelShared& sh, unsigned r) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int top = kSelBins - 1 - 4 * static_cast<int>(threadIdx.x);
+  unsigned c[4], s4 = 0u;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    c[q] = sh.bins[top - q];
+    s4 += c[q];
+  }
+  unsigned incl = warp_incl_scan(s4);
+  if (lane == 31) sh.wtot[warp] = incl;
+  __syncthreads();
+  unsigned before = 0u;   // entries in the warps before this one (fixed order)
+  for (int w = 0; w < warp; ++w) before += sh.wtot[w];
+  incl += before;
+  const unsigned excl = incl - s4;
+  if (excl < r && incl >= r) {   // exactly one thread
+    unsigned above = excl;
+    int q = 0;
+#pragma unroll
+    for (int qq = 0; qq < 3; ++qq)
+      if (q == qq && above + c[qq] < r) {
+        above += c[qq];
+        q = qq + 1;
+      }
+    sh.sel[0] = static_cast<unsigned>(top - q);
+    sh.sel[1] = above;
+  }
+  __syncthreads();
+}
+
+// Fusion + top-K of one map per CTA (1024 threads).  Thread t owns the contiguous scores
+// [t R, t R + R) of its map (R = ceil(nv / 1024)); with RM > 0 they stay in registers (R <= RM),
+// with RM = 0 (maps above 16384 tokens) every pass reads the raw scores again and recomputes
+// them with the same operations in the same order, so both give the same bits.
+//   1. min / max of both raw maps; any non-finite raw score records PACE_ERR_INVALID_ARG;
+//   2. min-max normalisation (a constant map becomes 0) and the two means;
+//   3. population variances, then the Eq. 7 weights (or a fixed ablation pair);
+//   4. S_final = alpha_w S_llm + beta_w S_vis (written out);
+//   5. the K-th largest S_final: 4096 value buckets, then rounds of 4096 bins over the key bits
+//      inside the selected range until one key T is left (exact);
+//   6. kept = every score above T plus the lowest-index scores equal to T, written in index order
+//      from one block-wide scan of per-thread counts.
+// Reductions run in a fixed order, so results are the same from run to run.
+template <int RM>
 __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* __restrict__ s_llm,
                                                                   const float* __restrict__ s_vis,
                                                                   const __grid_constant__ SelectTable tab,
                                                                   float tau, int fusion, float* __restrict__ s_final,
                                                                   float* __restrict__ weights,
-                                                                  int32_t* __restrict__ kept, int b_base) {
-  extern __shared__ float sm[];
-  __shared__ float red[64];
-  __shared__ int wsum[33];
-  __shared__ unsigned hist[256];
-  __shared__ unsigned sel[2];
+                                                                  int32_t* __restrict__ kept, int b_base, int* status) {
+  __shared__ SelShared sh;
   const int b = blockIdx.x;
   const int nv = tab.nv[b], v0 = tab.v0[b];
-  float* A = sm;        // S_llm raw -> normalised -> S_final
-  float* V = sm + nv;   // S_vis raw -> normalised
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int R = (nv + kSelThreads - 1) / kSelThreads;
+  const int i0 = tid * R;                                 // first score of this thread
+  const int n_mine = max(0, min(R, nv - i0));             // scores this thread owns
+  constexpr int RL = RM > 0 ? RM : 1;
+  float ra[RL], rv[RL];
+  const float* pa = s_llm + v0;
+  const float* pv = s_vis + v0;
 
-  // 1. stage both maps, min / max
+  // 1. min / max (and the finiteness check)
   float amin = FLT_MAX, amax = -FLT_MAX, vmin = FLT_MAX, vmax = -FLT_MAX;
-  for (int i = tid; i < nv; i += kSelThreads) {
-    const float a = s_llm[v0 + i], v = s_vis[v0 + i];
-    A[i] = a;
-    V[i] = v;
-    amin = fminf(amin, a); amax = fmaxf(amax, a);
-    vmin = fminf(vmin, v); vmax = fmaxf(vmax, v);
+  bool bad = false;
+  if constexpr (RM > 0) {
+#pragma unroll
+    for (int k = 0; k < RM; ++k)
+      if (k < n_mine) {
+        ra[k] = __ldg(pa + i0 + k);
+        rv[k] = __ldg(pv + i0 + k);
+      }
+#pragma unroll
+    for (int k = 0; k < RM; ++k)
+      if (k < n_mine) {
+        bad |= !(fabsf(ra[k]) <= FLT_MAX) || !(fabsf(rv[k]) <= FLT_MAX);
+        amin = fminf(amin, ra[k]); amax = fmaxf(amax, ra[k]);
+        vmin = fminf(vmin, rv[k]); vmax = fmaxf(vmax, rv[k]);
+      }
+  } else {
+    for (int k = 0; k < n_mine; ++k) {
+      const float a = __ldg(pa + i0 + k), v = __ldg(pv + i0 + k);
+      bad |= !(fabsf(a) <= FLT_MAX) || !(fabsf(v) <= FLT_MAX);
+      amin = fminf(amin, a); amax = fmaxf(amax, a);
+      vmin = fminf(vmin, v); vmax = fmaxf(vmax, v);
+    }
   }
-  const float2 mn = block_reduce2<1>(amin, vmin, red);
-  const float2 mx = block_reduce2<2>(amax, vmax, red);
-  const float ar = mx.x - mn.x, vr = mx.y - mn.y;
+  amin = warp_min(amin); amax = warp_max(amax);
+  vmin = warp_min(vmin); vmax = warp_max(vmax);
+  if (lane == 0) {
+    sh.red[0][0][warp] = amin; sh.red[0][1][warp] = amax;
+    sh.red[0][2][warp] = vmin; sh.red[0][3][warp] = vmax;
+  }
+  if (__syncthreads_or(bad) && tid == 0) record_error(status, PACE_ERR_INVALID_ARG, K_DDAE_SELECT);
+  float mna = FLT_MAX, mxa = -FLT_MAX, mnv = FLT_MAX, mxv = -FLT_MAX;
+  for (int w = 0; w < kSelWarps; ++w) {
+    mna = fminf(mna, sh.red[0][0][w]); mxa = fmaxf(mxa, sh.red[0][1][w]);
+    mnv = fminf(mnv, sh.red[0][2][w]); mxv = fmaxf(mxv, sh.red[0][3][w]);
+  }
+  const float ar = mxa - mna, vr = mxv - mnv;
+  // (x - min) / range as a product with the range's reciprocal: within an ulp of the quotient,
+  // and exact when the range is a power of two (a map spanning [0, 1] keeps its values)
+  const float ia = ar > 0.f ? 1.0f / ar : 0.f, iv = vr > 0.f ? 1.0f / vr : 0.f;
+  auto norm_a = [&](float a) { return (a - mna) * ia; };
+  auto norm_v = [&](float v) { return (v - mnv) * iv; };
 
-  // 2. min-max normalisation (a constant map becomes 0) and the means
+  // 2. normalisation and the means
   float sa = 0.f, sv = 0.f;
-  for (int i = tid; i < nv; i += kSelThreads) {
-    const float a = ar > 0.f ? __fdiv_rn(A[i] - mn.x, ar) : 0.f;
-    const float v = vr > 0.f ? __fdiv_rn(V[i] - mn.y, vr) : 0.f;
-    A[i] = a;
-    V[i] = v;
-    sa += a;
-    sv += v;
+  if constexpr (RM > 0) {
+#pragma unroll
+    for (int k = 0; k < RM; ++k)
+      if (k < n_mine) {
+        ra[k] = norm_a(ra[k]);
+        rv[k] = norm_v(rv[k]);
+        sa += ra[k];
+        sv += rv[k];
+      }
+  } else {
+    for (int k = 0; k < n_mine; ++k) {
+      sa += norm_a(__ldg(pa + i0 + k));
+      sv += norm_v(__ldg(pv + i0 + k));
+    }
   }
-  const float2 sums = block_reduce2<0>(sa, sv, red);
-  const float ma = sums.x / nv, mv = sums.y / nv;
-  float qa = 0.f, qv = 0.f;
-  for (int i = tid; i < nv; i += kSelThreads) {
-    const float da = A[i] - ma, dv = V[i] - mv;
-    qa = fmaf(da, da, qa);
-    qv = fmaf(dv, dv, qv);
-  }
-  const float2 sq = block_reduce2<0>(qa, qv, red);
-  const float sig_a = sqrtf(sq.x / nv), sig_v = sqrtf(sq.y / nv);
+  sa = warp_sum(sa);
+  sv = warp_sum(sv);
+  if (lane == 0) { sh.red[1][0][warp] = sa; sh.red[1][1][warp] = sv; }
+  __syncthreads();
+  float ta = 0.f, tv = 0.f;
+  for (int w = 0; w < kSelWarps; ++w) { ta += sh.red[1][0][w]; tv += sh.red[1][1][w]; }
+  const float ma = ta / nv, mv = tv / nv;
 
-  // 3. Eq. 7: confidence-weighted softmax fusion (or a fixed-weight ablation)
+  // 3. population variances and the fusion weights
+  float qa = 0.f, qv = 0.f;
+  if constexpr (RM > 0) {
+#pragma unroll
+    for (int k = 0; k < RM; ++k)
+      if (k < n_mine) {
+        const float da = ra[k] - ma, dv = rv[k] - mv;
+        qa = fmaf(da, da, qa);
+        qv = fmaf(dv, dv, qv);
+      }
+  } else {
+    for (int k = 0; k < n_mine; ++k) {
+      const float da = norm_a(__ldg(pa + i0 + k)) - ma, dv = norm_v(__ldg(pv + i0 + k)) - mv;
+      qa = fmaf(da, da, qa);
+      qv = fmaf(dv, dv, qv);
+    }
+  }
+  qa = warp_sum(qa);
+  qv = warp_sum(qv);
+  if (lane == 0) { sh.red[2][0][warp] = qa; sh.red[2][1][warp] = qv; }
+  __syncthreads();
+  float ua = 0.f, uv = 0.f;
+  for (int w = 0; w < kSelWarps; ++w) { ua += sh.red[2][0][w]; uv += sh.red[2][1][w]; }
+  const float sig_a = sqrtf(ua / nv), sig_v = sqrtf(uv / nv);
   float wa, wv;
   if (fusion == PACE_DDAE_ONLY_LLM) {
     wa = 1.f;
@@ -128,7 +242,7 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
     wv = 1.f;
   } else if (fusion == PACE_DDAE_FIXED) {
     wa = wv = 0.5f;
-  } else {
+  } else {   // Eq. 7
     const float za = sig_a / tau, zv = sig_v / tau, zm = fmaxf(za, zv);
     const float ea = expf(za - zm), ev = expf(zv - zm);
     wa = ea / (ea + ev);
@@ -138,81 +252,117 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
     weights[2 * (b_base + b)] = wa;
     weights[2 * (b_base + b) + 1] = wv;
   }
-  for (int i = tid; i < nv; i += kSelThreads) {
-    const float f = fmaf(wa, A[i], wv * V[i]);
-    A[i] = f;
-    if (s_final != nullptr) s_final[v0 + i] = f;
-  }
-  __syncthreads();
 
-  // 4. top-K threshold by radix select on the fp32 bits
+  // 4. S_final, kept in registers as selection keys (ra reused)
+  auto fused = [&](float a, float v) { return fmaf(wa, a, wv * v); };
+  if constexpr (RM > 0) {
+#pragma unroll
+    for (int k = 0; k < RM; ++k)
+      if (k < n_mine) {
+        const float f = fused(ra[k], rv[k]);
+        if (s_final != nullptr) s_final[v0 + i0 + k] = f;
+        ra[k] = __uint_as_float(sel_key(f));
+      }
+  } else if (s_final != nullptr) {
+    for (int k = 0; k < n_mine; ++k) s_final[v0 + i0 + k] = fused(norm_a(__ldg(pa + i0 + k)), norm_v(__ldg(pv + i0 + k)));
+  }
+  auto key_of = [&](int k) -> unsigned {
+    if constexpr (RM > 0) return __float_as_uint(ra[k]);
+    else return sel_key(fused(norm_a(__ldg(pa + i0 + k)), norm_v(__ldg(pv + i0 + k))));
+  };
+  // calls f(k, key) for every score of this thread, in index order
+  auto for_each_key = [&](auto&& f) {
+    if constexpr (RM > 0) {
+#pragma unroll
+      for (int k = 0; k < RM; ++k)
+        if (k < n_mine) f(k, key_of(k));
+    } else {
+      for (int k = 0; k < n_mine; ++k) f(k, key_of(k));
+    }
+  };
+
   const int K = tab.nk[b], k0 = tab.k0[b];
   if (K <= 0) return;
   if (K >= nv) {
     for (int i = tid; i < nv; i += kSelThreads) kept[k0 + i] = v0 + i;
     return;
   }
-  unsigned prefix = 0u, mask = 0u;
-  unsigned remaining = static_cast<unsigned>(K);
-  const int lane = tid & 31;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = tid; i < 256; i += kSelThreads) hist[i] = 0u;
-    __syncthreads();
-    // histogram of the next digit; lanes holding the same digit are combined first, so a
-    // narrow value range costs one shared atomic per distinct digit per warp
-    for (int base = 0; base < nv; base += kSelThreads) {
-      const int i = base + tid;
-      const unsigned key = i < nv ? __float_as_uint(A[i]) : 0u;
-      const bool in = i < nv && (key & mask) == prefix;
-      const unsigned digit = in ? ((key >> shift) & 255u) : 256u;
-      const unsigned peers = __match_any_sync(0xffffffffu, digit);
-      if (in && lane == __ffs(peers) - 1) atomicAdd(&hist[digit], static_cast<unsigned>(__popc(peers)));
-    }
-    __syncthreads();
-    if (tid < 32) warp_digit_search(hist, remaining, sel);
-    __syncthreads();
-    prefix |= sel[0] << shift;
-    mask |= 255u << shift;
-    remaining -= sel[1];
-    __syncthreads();
-  }
-  const unsigned T = prefix;  // bit pattern of the K-th largest S_final
-  // `remaining` = how many keys equal to T are kept (lowest indices first)
 
-  // 5. ascending compaction: the kept tokens before index i are the keys > T before i plus
-  // min(keys == T before i, remaining), so one packed prefix count per chunk places them
-  int gt_run = 0, eq_run = 0;
-  const unsigned lt_mask = (1u << lane) - 1u;
-  const int warp = tid >> 5;
-  for (int base = 0; base < nv; base += kSelThreads) {
-    const int i = base + tid;
-    const unsigned key = i < nv ? __float_as_uint(A[i]) : 0u;
-    const bool gt = i < nv && key > T;
-    const bool eq = i < nv && key == T;
-    const unsigned bg = __ballot_sync(0xffffffffu, gt), be = __ballot_sync(0xffffffffu, eq);
-    if (lane == 0) wsum[warp] = static_cast<int>(__popc(bg) | (__popc(be) << 16));
-    __syncthreads();
-    if (warp == 0) {
-      const int v = wsum[lane];
-      int incl = v;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int n = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += n;
+  // 5. the K-th largest key.  Round 0 counts value buckets; each later round splits the key
+  // range [lo, lo + span) of the selected bin into 4096 bins of 2^shift keys until shift = 0.
+  unsigned lo = 0u, span = 0u, r = static_cast<unsigned>(K);
+  int shift = -1;   // round 0: value buckets
+  // Histogram of this round: lanes of a warp holding the same bin add once (fused scores crowd a
+  // few low buckets, and equal keys one bin, which would otherwise serialise on one counter).
+  // Every lane takes part in every step (a lane without a score brings the no-bin value).
+  auto count_one = [&](int k) {
+    unsigned bin = kSelBins;   // no bin
+    if (k < n_mine) {
+      const unsigned key = key_of(k);
+      if (shift < 0) {
+        bin = sel_bucket(key);
+      } else {
+        const unsigned off = key - lo;   // wraps for keys below lo
+        if (off < span) bin = off >> shift;
       }
-      wsum[lane] = incl - v;
-      if (lane == 31) wsum[32] = incl;
     }
+    const unsigned peers = __match_any_sync(0xffffffffu, bin);
+    if (bin < kSelBins && lane == __ffs(peers) - 1) atomicAdd(&sh.bins[bin], static_cast<unsigned>(__popc(peers)));
+  };
+  auto count_bins = [&]() {
+    if constexpr (RM > 0) {
+#pragma unroll
+      for (int k = 0; k < RM; ++k) count_one(k);
+    } else {
+      for (int k = 0; k < R; ++k) count_one(k);   // R is the same for the whole block
+    }
+  };
+  while (true) {
+    for (int q = tid; q < kSelBins; q += kSelThreads) sh.bins[q] = 0u;
     __syncthreads();
-    const int wp = wsum[warp];
-    const int gt_before = gt_run + (wp & 0xffff) + __popc(bg & lt_mask);
-    const int eq_before = eq_run + (wp >> 16) + __popc(be & lt_mask);
-    if (gt || (eq && static_cast<unsigned>(eq_before) < remaining))
-      kept[k0 + gt_before + min(eq_before, static_cast<int>(remaining))] = v0 + i;
-    gt_run += wsum[32] & 0xffff;
-    eq_run += wsum[32] >> 16;
+    count_bins();
     __syncthreads();
+    sel_bin_from_top(sh, r);
+    const unsigned bsel = sh.sel[0], above = sh.sel[1];
+    r -= above;
+    if (shift < 0) {
+      lo = __float_as_uint(static_cast<float>(bsel) * (1.0f / kSelBins));
+      const unsigned hi = bsel == kSelBins - 1 ? 0x7F800001u   // the top bucket takes everything up to +inf
+                                               : __float_as_uint(static_cast<float>(bsel + 1) * (1.0f / kSelBins));
+      span = hi - lo;
+    } else {
+      lo += bsel << shift;
+      span = min(span - (bsel << shift), 1u << shift);
+      if (shift == 0) break;
+    }
+    const int bits = 32 - __clz(span - 1u);   // keys lo .. lo + span - 1 need `bits` bits
+    shift = bits > 12 ? bits - 12 : 0;
+    __syncthreads();   // everyone has read sel before the next round rewrites it
   }
+  const unsigned T = lo;        // key of the K-th largest S_final
+  const unsigned remaining = r; // how many keys equal to T are kept (lowest indices first)
+
+  // 6. ascending compaction from per-thread counts
+  unsigned gt = 0u, eq = 0u;
+  for_each_key([&](int, unsigned key) {
+    gt += key > T;
+    eq += key == T;
+  });
+  const unsigned gi = warp_incl_scan(gt), ei = warp_incl_scan(eq);
+  __syncthreads();   // the last round's readers of sh.sel / sh.wtot are done
+  if (lane == 31) { sh.wtot[warp] = gi; sh.wtot2[warp] = ei; }
+  __syncthreads();
+  unsigned g_before = gi - gt, e_before = ei - eq;
+  for (int w = 0; w < warp; ++w) { g_before += sh.wtot[w]; e_before += sh.wtot2[w]; }
+  for_each_key([&](int k, unsigned key) {
+    if (key > T) {
+      kept[k0 + g_before + min(e_before, remaining)] = v0 + i0 + k;
+      ++g_before;
+    } else if (key == T) {
+      if (e_before < remaining) kept[k0 + g_before + e_before] = v0 + i0 + k;
+      ++e_before;
+    }
+  });
 }
 
 // One warp per 2 KB piece of a row (128 16-byte vectors, 4 per lane, all in flight), so that a
@@ -380,7 +530,7 @@ extern "C" pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s
   int max_nv = 0;
   for (int b = 0; b < B; ++b) {
     const int nv = cu_v[b + 1] - cu_v[b], nk = cu_keep[b + 1] - cu_keep[b];
-    if (nv < 1 || nv > PACE_DDAE_MAX_TOKENS || nk < 0 || nk > nv) return PACE_ERR_INVALID_ARG;
+    if (nv < 1 || nk < 0 || nk > nv) return PACE_ERR_INVALID_ARG;
     if (nv > max_nv) max_nv = nv;
   }
   if (cu_keep[B] > 0 && kept == nullptr) return PACE_ERR_INVALID_ARG;
@@ -389,30 +539,29 @@ extern "C" pace_status_t pace_ddae_select(const float* s_llm_raw, const float* s
   if (!(tau > 0.f) || !std::isfinite(tau)) return PACE_ERR_INVALID_ARG;
   if (fusion < PACE_DDAE_ADAPTIVE || fusion > PACE_DDAE_FIXED) return PACE_ERR_INVALID_ARG;
   PACE_CHECK(check_device());
-  const size_t smem = static_cast<size_t>(2 * max_nv) * sizeof(float);
-  {
-    // opt in to the largest size once per device
-    static DeviceOnce once;
-    int dev = 0;
-    PACE_CUDA(cudaGetDevice(&dev));
-    if (!once.done(dev)) {
-      PACE_CUDA(cudaFuncSetAttribute(ddae_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(2 * PACE_DDAE_MAX_TOKENS * sizeof(float))));
-      once.mark(dev);
-    }
-  }
+  int* status = device_status_word();
   for (int c0 = 0; c0 < B; c0 += kSelMaxB) {
     const int nb = (B - c0) < kSelMaxB ? (B - c0) : kSelMaxB;
     SelectTable t;
+    int per_thread = 1;
     for (int i = 0; i < nb; ++i) {
       const int b = c0 + i;
       t.v0[i] = cu_v[b];
       t.nv[i] = cu_v[b + 1] - cu_v[b];
       t.k0[i] = cu_keep[b];
       t.nk[i] = cu_keep[b + 1] - cu_keep[b];
+      per_thread = std::max(per_thread, (t.nv[i] + kSelThreads - 1) / kSelThreads);
     }
-    ddae_select_kernel<<<nb, kSelThreads, smem, stream>>>(s_llm_raw, s_vis_raw, t, tau, fusion, s_final, weights, kept,
-                                                           c0);
+    // scores per thread in registers: 4 or 12, else (maps above 12288 tokens) read again per pass
+    if (per_thread <= 4)
+      ddae_select_kernel<4><<<nb, kSelThreads, 0, stream>>>(s_llm_raw, s_vis_raw, t, tau, fusion, s_final, weights,
+                                                             kept, c0, status);
+    else if (per_thread <= kSelRegMax)
+      ddae_select_kernel<kSelRegMax><<<nb, kSelThreads, 0, stream>>>(s_llm_raw, s_vis_raw, t, tau, fusion, s_final,
+                                                                      weights, kept, c0, status);
+    else
+      ddae_select_kernel<0><<<nb, kSelThreads, 0, stream>>>(s_llm_raw, s_vis_raw, t, tau, fusion, s_final, weights,
+                                                             kept, c0, status);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;

@@ -20,7 +20,6 @@ LIB_PATH = os.path.join(_HERE, "libpace.so")
 
 PACE_OK, PACE_ERR_INVALID_ARG, PACE_ERR_UNSUPPORTED_ARCH = 0, 1, 2
 PACE_ERR_WORKSPACE, PACE_ERR_CUDA, PACE_ERR_TIMEOUT = 3, 4, 5
-PACE_DDAE_MAX_TOKENS = 24576
 STATS_FIELDS = ("phi", "rho_g", "d_top", "rho_d", "rho", "r", "n_patches", "k_tail", "h_out", "w_out")
 
 

@@ -432,6 +432,52 @@ def test_vit_importance_chunked_matches_unchunked(pace, ends):
     _no_device_error(pace)
 
 
+def test_vit_importance_nan_rows_stay_in_their_image(pace):
+    """NaN and inf in the query rows of some images of a ragged batch: every other image's
+    S_vis_raw still equals the oracle's on its own (clean) rows.  An image's last query tile
+    in pass 2 also covers the next image's first rows; those columns are masked explicitly."""
+    lens = [300, 516, 4, 1300, 388, 260]
+    H, D, merge = 4, 80, 4
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    total = int(cu[-1])
+    Qb = synth.random_small_qk(31, total, H, D)
+    Kb = synth.random_small_qk(1031, total, H, D)
+    scale = 1.0 / math.sqrt(D)
+    ref = O.vit_attn_importance(f64(Qb), f64(Kb), cu, scale, merge)
+    Q = bf16_tensor(Qb)
+    Q[cu[1]:cu[1] + 7] = float("nan")            # image 1: its first rows (inside image 0's last tile)
+    Q[cu[3]] = float("inf")                       # image 3: first row +inf, another row -inf
+    Q[cu[3] + 1, :, 5] = float("-inf")
+    Q[cu[5]:cu[6]] = float("nan")                 # image 5: every row, past the end of image 4
+    out = pace.pace_vit_attn_importance(Q, bf16_tensor(Kb), cu, scale, merge).cpu().numpy()
+    for b in (0, 2, 4):
+        m0, m1 = cu[b] // merge, cu[b + 1] // merge
+        assert np.isfinite(out[m0:m1]).all(), b
+        assert_scores_close(out[m0:m1], ref[m0:m1], what=f"S_vis_raw of clean image {b}")
+    _no_device_error(pace)
+
+
+def test_llm_importance_nan_queries_stay_in_their_image(pace):
+    """The same isolation on the LLM text->visual path (GQA): NaN text queries of image 1 leave
+    images 0 and 2 equal to the oracle."""
+    tq, nv = [70, 33, 140], [300, 129, 260]
+    Hq, Hkv, D = 8, 2, 128
+    cu_q = np.concatenate([[0], np.cumsum(tq)]).astype(np.int32)
+    cu_k = np.concatenate([[0], np.cumsum(nv)]).astype(np.int32)
+    Qb = synth.random_small_qk(41, int(cu_q[-1]), Hq, D)
+    Kb = synth.random_small_qk(1041, int(cu_k[-1]), Hkv, D)
+    scale = 1.0 / math.sqrt(D)
+    ref = O.llm_text_visual_importance(f64(Qb), f64(Kb), cu_q, cu_k, scale)
+    Q = bf16_tensor(Qb)
+    Q[cu_q[1]:cu_q[2]] = float("nan")
+    out = pace.pace_llm_text_visual_importance(Q, bf16_tensor(Kb), cu_q, cu_k, scale).cpu().numpy()
+    for b in (0, 2):
+        v0, v1 = cu_k[b], cu_k[b + 1]
+        assert np.isfinite(out[v0:v1]).all(), b
+        assert_scores_close(out[v0:v1], ref[v0:v1], what=f"S_llm_raw of clean image {b}")
+    _no_device_error(pace)
+
+
 def test_vit_importance_chunked_rejects_bad_chunks(pace):
     Q = torch.zeros((8, 1, 64), dtype=torch.bfloat16, device="cuda")
     ev = torch.cuda.Event()
@@ -593,7 +639,9 @@ def test_ddae_fusion_ablations(pace, mode, name):
 
 
 @pytest.mark.parametrize("lens,fracs", [([256], [0.1]), ([2584], [0.1]), ([10549], [0.05]), ([1], [1.0]),
-                                        ([7, 300, 1000, 24576], [0.25, 0.0, 1.0, 0.1])])
+                                        ([7, 300, 1000, 24576], [0.25, 0.0, 1.0, 0.1]),
+                                        ([4096, 4097, 12288, 12289], [0.1, 0.05, 0.25, 0.1]),
+                                        ([42196], [0.1]), ([150000, 3], [0.02, 0.5])])
 def test_ddae_select_random(pace, lens, fracs):
     rng = np.random.default_rng(len(lens) + lens[0])
     cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
@@ -615,7 +663,7 @@ def test_ddae_select_exact_decisions_with_ties(pace):
     """S_llm == S_vis with min 0 and max 1: S_final = x exactly in fp32 and fp64, so the kept
     set (ties broken by the lower index) must equal the oracle's bit for bit."""
     rng = np.random.default_rng(9)
-    for n, K in ((1000, 100), (4096, 1), (333, 332), (50, 25)):
+    for n, K in ((1000, 100), (4096, 1), (333, 332), (50, 25), (20000, 2000), (12289, 7)):
         x = np.round(rng.uniform(size=n) * 16) / 16      # many exact ties
         x[0], x[-1] = 0.0, 1.0
         cu = np.array([0, n], dtype=np.int32)
@@ -634,14 +682,40 @@ def test_ddae_select_golden_and_constant(pace, golden):
     assert kept.tolist() == [int(v) for v in g["kept_top2"]]
     s_final, w, kept = _select(pace, np.full(10, 3.0), np.arange(10.0), np.array([0, 10], np.int32), [3])
     assert kept.tolist() == [7, 8, 9]
+    # both maps constant: S_final = 0 everywhere, every score ties, the lowest indices are kept
+    for n in (10, 5000, 13000):
+        s_final, w, kept = _select(pace, np.full(n, 2.0), np.full(n, 7.0), np.array([0, n], np.int32), [3])
+        assert not s_final.any() and kept.tolist() == [0, 1, 2]
+
+
+def test_ddae_select_non_finite_scores_are_reported(pace):
+    """A NaN or inf raw score records PACE_ERR_INVALID_ARG (kernel id 9) in the device status
+    word.  The map's scores are then not meaningful (NaN reaches the Eq. 7 weights), but the call
+    still writes K distinct in-range indices in ascending order, the same on every run."""
+    n = 600
+    rng = np.random.default_rng(3)
+    sl = rng.uniform(size=n).astype(np.float32)
+    sv = rng.uniform(size=n).astype(np.float32)
+    sl[[10, 500]] = np.nan
+    for bad_v in (None, np.inf):
+        if bad_v is not None:
+            sl[[10, 500]] = 0.5
+            sv[7] = bad_v
+        outs = []
+        for _ in range(2):
+            _, _, kept = _select(pace, sl, sv, np.array([0, n], np.int32), [n // 3])
+            code, where = pace.pace_device_status(clear=True)
+            assert code == pace.PACE_ERR_INVALID_ARG and where == 9
+            assert kept.size == n // 3 and np.all(np.diff(kept) > 0) and kept.min() >= 0 and kept.max() < n
+            outs.append(kept)
+        np.testing.assert_array_equal(outs[0], outs[1])
 
 
 def test_ddae_select_rejects(pace):
     with pytest.raises(pace.PaceError):
         _select(pace, np.zeros(5), np.zeros(5), np.array([0, 5], np.int32), [6])
     with pytest.raises(pace.PaceError):
-        n = pace.PACE_DDAE_MAX_TOKENS + 1
-        _select(pace, np.zeros(n), np.zeros(n), np.array([0, n], np.int32), [1])
+        _select(pace, np.zeros(5), np.zeros(5), np.array([0, 0, 5], np.int32), [0, 1])   # an empty map
 
 
 # ----------------------------------------------------------------------------------------------
