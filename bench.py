@@ -61,6 +61,8 @@ def load_peaks():
 
 
 DRAM_SUMMARY = os.path.join(ROOT, "profiles", "vit_importance_img4k_dram.txt")
+# NVIDIA's dense (no 2:4 sparsity) bf16 tensor figure for one GB300, TFLOP/s
+DATASHEET_BF16_TFLOPS = 2250.0
 ATTN_SRC = os.path.join(ROOT, "paper_2608_27206_gb300", "csrc", "attn.cu")
 DRAM_CMD = ("ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum --clock-control none "
             "-k regex:attn_ -c 3 --csv --log-file gpurun_out/vit_dram.csv python bench.py --profile vit --reps 1")
@@ -814,6 +816,10 @@ def run_gpu(args):
                          "algorithmic_flops": cnt["vit_flops"], "us": round(vit_ms * 1e3, 1),
                          # one pass of QK^T is the "useful" work; the second pass recomputes it
                          "useful_one_pass_frac": round(achieved / 2 / peak, 4),
+                         # the same achieved rate against NVIDIA's published dense bf16 figure
+                         "datasheet_peak": DATASHEET_BF16_TFLOPS,
+                         "frac_of_datasheet": round(achieved / DATASHEET_BF16_TFLOPS, 4),
+                         "useful_one_pass_frac_of_datasheet": round(achieved / 2 / DATASHEET_BF16_TFLOPS, 4),
                          # every score costs one exp2 per pass (N^2 H per pass)
                          "mufu_ex2_per_s": round(cnt["vit_ex2"] / (vit_ms * 1e-3), 1),
                          "mufu_frac": round(cnt["vit_ex2"] / (vit_ms * 1e-3) / mufu_peak, 4)

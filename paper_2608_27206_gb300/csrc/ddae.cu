@@ -1,11 +1,11 @@
 // DDAE fusion + top-K selection (Sec. 3.3, Eq. 7) and the gather of kept rows.
 //
-// pace_ddae_select: one CTA of 1024 threads per image.  Both raw maps are staged in
-// shared memory; min/max, mean and the population variance are block reductions in a
-// fixed order (bit-stable run to run); the K-th largest S_final is found by an MSB-first
-// 8-bit radix select on the fp32 bit patterns (S_final >= 0, so integer order equals
-// float order), and the kept set is compacted in ascending index order with warp
-// ballots, the lower index winning among equal scores.
+// pace_ddae_select: one CTA of 1024 threads per image.  Thread t owns scores t, t + 1024, ..
+// (every warp access to the maps is one coalesced row of 32 scores); min/max, mean and the
+// population variance are block reductions in a fixed order (bit-stable run to run); the K-th
+// largest S_final is found by histogram rounds over the fp32 bit patterns (S_final >= 0, so
+// integer order equals float order), and the kept set is compacted in ascending index order
+// with warp ballots, the lower index winning among equal scores.
 //
 // pace_gather: one warp per kept row, 16-byte vector loads and stores.
 #include <algorithm>
@@ -20,9 +20,12 @@ namespace {
 
 constexpr int kSelThreads = 1024;
 constexpr int kSelWarps = kSelThreads / 32;
+static_assert(kSelWarps == 32, "block reductions take one warp partial per lane");
 constexpr int kSelMaxB = 256;
 constexpr int kSelBins = 4096;           // bins of one selection round (4 per thread)
 constexpr int kSelRegMax = 12;           // scores per thread held in registers (12288 per map)
+constexpr int kSelCompK = 16;            // score rows (of 1024) per compaction chunk
+constexpr int kSelCand = kSelThreads;    // largest value bucket ranked directly (one score per thread)
 
 struct SelectTable {
   int v0[kSelMaxB];  // first global row of image b
@@ -32,11 +35,20 @@ struct SelectTable {
 };
 
 struct SelShared {
-  float red[3][4][kSelWarps];   // warp partials of the three block reductions
+  float red[8][kSelWarps];      // warp partials of the block reduction (min, max and two moments per map)
   unsigned bins[kSelBins];      // histogram of the current selection round
-  unsigned wtot[kSelWarps];     // per-warp totals (bin prefix, compaction scans)
-  unsigned wtot2[kSelWarps];
+  unsigned wtot[kSelWarps];     // per-warp totals (bin prefix)
   unsigned sel[2];              // selected bin, entries in the bins above it
+  unsigned cand[kSelCand];      // keys of the selected value bucket
+  int cidx[kSelCand];           // and their indices in the map
+  unsigned ncand;
+  // compaction: per (score row k, warp) ballots of the keys above / equal to the threshold, the
+  // exclusive prefix of their counts along the row (above in the low, equal in the high 16
+  // bits), and the row totals
+  unsigned mgt[kSelCompK][kSelWarps];
+  unsigned meq[kSelCompK][kSelWarps];
+  unsigned pre[kSelCompK][kSelWarps];
+  unsigned rtot[kSelCompK];
 };
 
 __device__ __forceinline__ float warp_min(float v) {
@@ -89,9 +101,8 @@ __device__ __forceinline__ void sel_bin_from_top(SelShared& sh, unsigned r) {
   unsigned incl = warp_incl_scan(s4);
   if (lane == 31) sh.wtot[warp] = incl;
   __syncthreads();
-  unsigned before = 0u;   // entries in the warps before this one (fixed order)
-  for (int w = 0; w < warp; ++w) before += sh.wtot[w];
-  incl += before;
+  // entries in the warps before this one
+  incl += __reduce_add_sync(0xffffffffu, lane < warp ? sh.wtot[lane] : 0u);
   const unsigned excl = incl - s4;
   if (excl < r && incl >= r) {   // exactly one thread
     unsigned above = excl;
@@ -108,18 +119,26 @@ __device__ __forceinline__ void sel_bin_from_top(SelShared& sh, unsigned r) {
   __syncthreads();
 }
 
-// Fusion + top-K of one map per CTA (1024 threads).  Thread t owns the contiguous scores
-// [t R, t R + R) of its map (R = ceil(nv / 1024)); with RM > 0 they stay in registers (R <= RM),
-// with RM = 0 (maps above 16384 tokens) every pass reads the raw scores again and recomputes
-// them with the same operations in the same order, so both give the same bits.
-//   1. min / max of both raw maps; any non-finite raw score records PACE_ERR_INVALID_ARG;
-//   2. min-max normalisation (a constant map becomes 0) and the two means;
-//   3. population variances, then the Eq. 7 weights (or a fixed ablation pair);
-//   4. S_final = alpha_w S_llm + beta_w S_vis (written out);
-//   5. the K-th largest S_final: 4096 value buckets, then rounds of 4096 bins over the key bits
-//      inside the selected range until one key T is left (exact);
-//   6. kept = every score above T plus the lowest-index scores equal to T, written in index order
-//      from one block-wide scan of per-thread counts.
+// Fusion + top-K of one map per CTA (1024 threads).  Thread t owns the scores i = k * 1024 + t,
+// k = 0 .. R - 1 (R = ceil(nv / 1024)); with RM > 0 they stay in registers (R <= RM), with
+// RM = 0 (maps above 12288 tokens) every pass reads the raw scores again and recomputes them
+// with the same operations in the same order, so both give the same bits.
+//   1. one block reduction of both raw maps: min, max, and the sums of x - c and (x - c)^2 with c
+//      the map's first score (the shifted-data form of the variance); any non-finite raw score
+//      records PACE_ERR_INVALID_ARG;
+//   2. min-max normalisation is affine (a constant map becomes 0), so the normalised maps'
+//      population variances follow from those sums;
+//   3. the Eq. 7 weights (or a fixed ablation pair);
+//   4. S_final = alpha_w norm(S_llm) + beta_w norm(S_vis) (written out);
+//   5. the K-th largest S_final: 4096 value buckets; if the selected bucket holds at most 1024
+//      scores, their keys are gathered and ranked directly, else rounds of 4096 bins over the key
+//      bits inside the selected range run until one key T is left (exact either way);
+//      for maps of up to 16384 scores with such a bucket, the pass that gathers the bucket also
+//      records which scores lie above it, and each bucket score places itself by its own rank,
+//      so 6. starts from those records;
+//   6. kept = every score above T plus the lowest-index scores equal to T, written in index order:
+//      score i sits at place (k, warp, lane) of that order, so the per (k, warp) ballot counts,
+//      scanned along each row and summed over the rows before, give every kept score its slot.
 // Reductions run in a fixed order, so results are the same from run to run.
 template <int RM>
 __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* __restrict__ s_llm,
@@ -132,107 +151,70 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
   const int b = blockIdx.x;
   const int nv = tab.nv[b], v0 = tab.v0[b];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int R = (nv + kSelThreads - 1) / kSelThreads;
-  const int i0 = tid * R;                                 // first score of this thread
-  const int n_mine = max(0, min(R, nv - i0));             // scores this thread owns
+  const int R = (nv + kSelThreads - 1) / kSelThreads;   // the same for the whole block
+  auto idx = [&](int k) { return k * kSelThreads + tid; };
+  auto has = [&](int k) { return idx(k) < nv; };
   constexpr int RL = RM > 0 ? RM : 1;
   float ra[RL], rv[RL];
   const float* pa = s_llm + v0;
   const float* pv = s_vis + v0;
 
-  // 1. min / max (and the finiteness check)
+  // 1. min / max and shifted moments (and the finiteness check); the first round's bins are
+  // cleared on the way
+  const float ca = __ldg(pa), cv = __ldg(pv);
+  for (int q = tid; q < kSelBins; q += kSelThreads) sh.bins[q] = 0u;
+  if (tid == 0) sh.ncand = 0u;
   float amin = FLT_MAX, amax = -FLT_MAX, vmin = FLT_MAX, vmax = -FLT_MAX;
+  float s1a = 0.f, s2a = 0.f, s1v = 0.f, s2v = 0.f;
   bool bad = false;
+  auto take = [&](float a, float v) {
+    bad |= !(fabsf(a) <= FLT_MAX) || !(fabsf(v) <= FLT_MAX);
+    amin = fminf(amin, a); amax = fmaxf(amax, a);
+    vmin = fminf(vmin, v); vmax = fmaxf(vmax, v);
+    const float da = a - ca, dv = v - cv;
+    s1a += da; s2a = fmaf(da, da, s2a);
+    s1v += dv; s2v = fmaf(dv, dv, s2v);
+  };
   if constexpr (RM > 0) {
 #pragma unroll
     for (int k = 0; k < RM; ++k)
-      if (k < n_mine) {
-        ra[k] = __ldg(pa + i0 + k);
-        rv[k] = __ldg(pv + i0 + k);
+      if (has(k)) {
+        ra[k] = __ldg(pa + idx(k));
+        rv[k] = __ldg(pv + idx(k));
       }
 #pragma unroll
     for (int k = 0; k < RM; ++k)
-      if (k < n_mine) {
-        bad |= !(fabsf(ra[k]) <= FLT_MAX) || !(fabsf(rv[k]) <= FLT_MAX);
-        amin = fminf(amin, ra[k]); amax = fmaxf(amax, ra[k]);
-        vmin = fminf(vmin, rv[k]); vmax = fmaxf(vmax, rv[k]);
-      }
+      if (has(k)) take(ra[k], rv[k]);
   } else {
-    for (int k = 0; k < n_mine; ++k) {
-      const float a = __ldg(pa + i0 + k), v = __ldg(pv + i0 + k);
-      bad |= !(fabsf(a) <= FLT_MAX) || !(fabsf(v) <= FLT_MAX);
-      amin = fminf(amin, a); amax = fmaxf(amax, a);
-      vmin = fminf(vmin, v); vmax = fmaxf(vmax, v);
-    }
+    for (int k = 0; k < R; ++k)
+      if (has(k)) take(__ldg(pa + idx(k)), __ldg(pv + idx(k)));
   }
   amin = warp_min(amin); amax = warp_max(amax);
   vmin = warp_min(vmin); vmax = warp_max(vmax);
+  s1a = warp_sum(s1a); s2a = warp_sum(s2a);
+  s1v = warp_sum(s1v); s2v = warp_sum(s2v);
   if (lane == 0) {
-    sh.red[0][0][warp] = amin; sh.red[0][1][warp] = amax;
-    sh.red[0][2][warp] = vmin; sh.red[0][3][warp] = vmax;
+    sh.red[0][warp] = amin; sh.red[1][warp] = amax; sh.red[2][warp] = vmin; sh.red[3][warp] = vmax;
+    sh.red[4][warp] = s1a; sh.red[5][warp] = s2a; sh.red[6][warp] = s1v; sh.red[7][warp] = s2v;
   }
   if (__syncthreads_or(bad) && tid == 0) record_error(status, PACE_ERR_INVALID_ARG, K_DDAE_SELECT);
-  float mna = FLT_MAX, mxa = -FLT_MAX, mnv = FLT_MAX, mxv = -FLT_MAX;
-  for (int w = 0; w < kSelWarps; ++w) {
-    mna = fminf(mna, sh.red[0][0][w]); mxa = fmaxf(mxa, sh.red[0][1][w]);
-    mnv = fminf(mnv, sh.red[0][2][w]); mxv = fmaxf(mxv, sh.red[0][3][w]);
-  }
+  // lane l takes warp l's partials; the butterflies leave the block's values in every lane
+  const float mna = warp_min(sh.red[0][lane]), mxa = warp_max(sh.red[1][lane]);
+  const float mnv = warp_min(sh.red[2][lane]), mxv = warp_max(sh.red[3][lane]);
+  const float t1a = warp_sum(sh.red[4][lane]), t2a = warp_sum(sh.red[5][lane]);
+  const float t1v = warp_sum(sh.red[6][lane]), t2v = warp_sum(sh.red[7][lane]);
   const float ar = mxa - mna, vr = mxv - mnv;
   // (x - min) / range as a product with the range's reciprocal: within an ulp of the quotient,
   // and exact when the range is a power of two (a map spanning [0, 1] keeps its values)
   const float ia = ar > 0.f ? 1.0f / ar : 0.f, iv = vr > 0.f ? 1.0f / vr : 0.f;
-  auto norm_a = [&](float a) { return (a - mna) * ia; };
-  auto norm_v = [&](float v) { return (v - mnv) * iv; };
 
-  // 2. normalisation and the means
-  float sa = 0.f, sv = 0.f;
-  if constexpr (RM > 0) {
-#pragma unroll
-    for (int k = 0; k < RM; ++k)
-      if (k < n_mine) {
-        ra[k] = norm_a(ra[k]);
-        rv[k] = norm_v(rv[k]);
-        sa += ra[k];
-        sv += rv[k];
-      }
-  } else {
-    for (int k = 0; k < n_mine; ++k) {
-      sa += norm_a(__ldg(pa + i0 + k));
-      sv += norm_v(__ldg(pv + i0 + k));
-    }
-  }
-  sa = warp_sum(sa);
-  sv = warp_sum(sv);
-  if (lane == 0) { sh.red[1][0][warp] = sa; sh.red[1][1][warp] = sv; }
-  __syncthreads();
-  float ta = 0.f, tv = 0.f;
-  for (int w = 0; w < kSelWarps; ++w) { ta += sh.red[1][0][w]; tv += sh.red[1][1][w]; }
-  const float ma = ta / nv, mv = tv / nv;
-
-  // 3. population variances and the fusion weights
-  float qa = 0.f, qv = 0.f;
-  if constexpr (RM > 0) {
-#pragma unroll
-    for (int k = 0; k < RM; ++k)
-      if (k < n_mine) {
-        const float da = ra[k] - ma, dv = rv[k] - mv;
-        qa = fmaf(da, da, qa);
-        qv = fmaf(dv, dv, qv);
-      }
-  } else {
-    for (int k = 0; k < n_mine; ++k) {
-      const float da = norm_a(__ldg(pa + i0 + k)) - ma, dv = norm_v(__ldg(pv + i0 + k)) - mv;
-      qa = fmaf(da, da, qa);
-      qv = fmaf(dv, dv, qv);
-    }
-  }
-  qa = warp_sum(qa);
-  qv = warp_sum(qv);
-  if (lane == 0) { sh.red[2][0][warp] = qa; sh.red[2][1][warp] = qv; }
-  __syncthreads();
-  float ua = 0.f, uv = 0.f;
-  for (int w = 0; w < kSelWarps; ++w) { ua += sh.red[2][0][w]; uv += sh.red[2][1][w]; }
-  const float sig_a = sqrtf(ua / nv), sig_v = sqrtf(uv / nv);
+  // 2-3. the normalised maps' population variances: (x - min) / range has the variance of x
+  // divided by range^2, and var x = E[(x - c)^2] - (E[x - c])^2
+  const float inv_n = 1.0f / static_cast<float>(nv);
+  const float m1a = t1a * inv_n, m1v = t1v * inv_n;
+  const float var_a = fmaxf(fmaf(-m1a, m1a, t2a * inv_n), 0.f) * ia * ia;
+  const float var_v = fmaxf(fmaf(-m1v, m1v, t2v * inv_n), 0.f) * iv * iv;
+  const float sig_a = sqrtf(var_a), sig_v = sqrtf(var_v);
   float wa, wv;
   if (fusion == PACE_DDAE_ONLY_LLM) {
     wa = 1.f;
@@ -243,61 +225,106 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
   } else if (fusion == PACE_DDAE_FIXED) {
     wa = wv = 0.5f;
   } else {   // Eq. 7
-    const float za = sig_a / tau, zv = sig_v / tau, zm = fmaxf(za, zv);
-    const float ea = expf(za - zm), ev = expf(zv - zm);
-    wa = ea / (ea + ev);
-    wv = ev / (ea + ev);
+    // (every thread evaluates these; the fast intrinsics are within a few ulp)
+    const float za = __fdividef(sig_a, tau), zv = __fdividef(sig_v, tau), zm = fmaxf(za, zv);
+    const float ea = __expf(za - zm), ev = __expf(zv - zm);
+    const float inv = __fdividef(1.0f, ea + ev);
+    wa = ea * inv;
+    wv = ev * inv;
   }
   if (tid == 0 && weights != nullptr) {
     weights[2 * (b_base + b)] = wa;
     weights[2 * (b_base + b) + 1] = wv;
   }
 
-  // 4. S_final, kept in registers as selection keys (ra reused)
-  auto fused = [&](float a, float v) { return fmaf(wa, a, wv * v); };
+  // 4. S_final (in registers, ra reused, when RM > 0: written out by the first counting pass
+  // below, or before an early return; otherwise written here)
+  // alpha_w (a - min_a) / range_a + beta_w (v - min_v) / range_v with each map's weight and
+  // reciprocal range folded into one coefficient
+  const float cfa = wa * ia, cfv = wv * iv;
+  auto fused = [&](float a, float v) { return fmaf(cfa, a - mna, cfv * (v - mnv)); };
   if constexpr (RM > 0) {
 #pragma unroll
     for (int k = 0; k < RM; ++k)
-      if (k < n_mine) {
-        const float f = fused(ra[k], rv[k]);
-        if (s_final != nullptr) s_final[v0 + i0 + k] = f;
-        ra[k] = __uint_as_float(sel_key(f));
-      }
+      if (has(k)) ra[k] = fused(ra[k], rv[k]);
   } else if (s_final != nullptr) {
-    for (int k = 0; k < n_mine; ++k) s_final[v0 + i0 + k] = fused(norm_a(__ldg(pa + i0 + k)), norm_v(__ldg(pv + i0 + k)));
+    for (int k = 0; k < R; ++k)
+      if (has(k)) s_final[v0 + idx(k)] = fused(__ldg(pa + idx(k)), __ldg(pv + idx(k)));
   }
-  auto key_of = [&](int k) -> unsigned {
-    if constexpr (RM > 0) return __float_as_uint(ra[k]);
-    else return sel_key(fused(norm_a(__ldg(pa + i0 + k)), norm_v(__ldg(pv + i0 + k))));
+  auto store_final = [&](int k) {
+    if constexpr (RM > 0)
+      if (s_final != nullptr && has(k)) s_final[v0 + idx(k)] = ra[k];
   };
-  // calls f(k, key) for every score of this thread, in index order
-  auto for_each_key = [&](auto&& f) {
+  // key of this thread's score k (0 where it has none: below every positive score)
+  auto key_of = [&](int k) -> unsigned {
+    if (!has(k)) return 0u;
+    if constexpr (RM > 0) return sel_key(ra[k]);
+    else return sel_key(fused(__ldg(pa + idx(k)), __ldg(pv + idx(k))));
+  };
+  // calls f(k) for k = kb .. ke - 1 (the same k for every thread at each call)
+  auto for_rows = [&](int kb, int ke, auto&& f) {
     if constexpr (RM > 0) {
 #pragma unroll
       for (int k = 0; k < RM; ++k)
-        if (k < n_mine) f(k, key_of(k));
+        if (k >= kb && k < ke) f(k);
     } else {
-      for (int k = 0; k < n_mine; ++k) f(k, key_of(k));
+      for (int k = kb; k < ke; ++k) f(k);
     }
   };
 
   const int K = tab.nk[b], k0 = tab.k0[b];
-  if (K <= 0) return;
-  if (K >= nv) {
-    for (int i = tid; i < nv; i += kSelThreads) kept[k0 + i] = v0 + i;
+  if (K <= 0 || K >= nv) {
+    for_rows(0, R, store_final);
+    if (K > 0)
+      for (int i = tid; i < nv; i += kSelThreads) kept[k0 + i] = v0 + i;
     return;
   }
+
+  // Writes the kept indices of score rows kb .. ke - 1 from the ballots in sh.mgt / sh.meq (row
+  // k - kb, warp w: the lanes whose score k * 1024 + 32 w + lane is above / equal to T): an
+  // exclusive scan along each row (warp k - kb of the block), then thread (k - kb, w) adds the rows
+  // before and places the set bits of its two ballots.  gbase / ebase count the keys above / equal
+  // to T in the rows before kb; the counts after ke are returned.  Every row total fits 16 bits.
+  auto compact_rows = [&](int kb, int ke, unsigned remaining, unsigned gbase, unsigned ebase) {
+    const int nr = ke - kb;
+    if (warp < nr) {
+      const unsigned v = __popc(sh.mgt[warp][lane]) | (__popc(sh.meq[warp][lane]) << 16);
+      const unsigned incl = warp_incl_scan(v);
+      sh.pre[warp][lane] = incl - v;
+      if (lane == 31) sh.rtot[warp] = incl;
+    }
+    __syncthreads();
+    if (tid < nr * kSelWarps) {
+      const int kr = tid >> 5, wp = tid & 31;
+      unsigned pw = sh.pre[kr][wp];
+      for (int q = 0; q < kr; ++q) pw += sh.rtot[q];
+      const unsigned g0 = gbase + (pw & 0xFFFFu), e0 = ebase + (pw >> 16);
+      const unsigned gm = sh.mgt[kr][wp], em = sh.meq[kr][wp];
+      const int first = (kb + kr) * kSelThreads + wp * 32;
+      for (unsigned m = gm | em; m != 0u; m &= m - 1u) {
+        const int bit = __ffs(m) - 1;
+        const unsigned lt = (1u << bit) - 1u;
+        const unsigned gb = g0 + __popc(gm & lt), eb = e0 + __popc(em & lt);
+        if ((gm >> bit) & 1u) __stcg(kept + k0 + gb + min(eb, remaining), v0 + first + bit);
+        else if (eb < remaining) __stcg(kept + k0 + gb + eb, v0 + first + bit);
+      }
+    }
+    unsigned tot = 0u;
+    for (int q = 0; q < nr; ++q) tot += sh.rtot[q];
+    return make_uint2(gbase + (tot & 0xFFFFu), ebase + (tot >> 16));
+  };
 
   // 5. the K-th largest key.  Round 0 counts value buckets; each later round splits the key
   // range [lo, lo + span) of the selected bin into 4096 bins of 2^shift keys until shift = 0.
   unsigned lo = 0u, span = 0u, r = static_cast<unsigned>(K);
   int shift = -1;   // round 0: value buckets
-  // Histogram of this round: lanes of a warp holding the same bin add once (fused scores crowd a
-  // few low buckets, and equal keys one bin, which would otherwise serialise on one counter).
-  // Every lane takes part in every step (a lane without a score brings the no-bin value).
+  // Histogram of this round.  A warp whose 32 scores share one bin (a flat stretch of the map, or
+  // ties) adds once; otherwise each lane adds for itself and the rare same-bin lanes are
+  // serialised by the shared-memory atomics.
   auto count_one = [&](int k) {
+    if (shift < 0) store_final(k);
     unsigned bin = kSelBins;   // no bin
-    if (k < n_mine) {
+    if (has(k)) {
       const unsigned key = key_of(k);
       if (shift < 0) {
         bin = sel_bucket(key);
@@ -306,21 +333,19 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
         if (off < span) bin = off >> shift;
       }
     }
-    const unsigned peers = __match_any_sync(0xffffffffu, bin);
-    if (bin < kSelBins && lane == __ffs(peers) - 1) atomicAdd(&sh.bins[bin], static_cast<unsigned>(__popc(peers)));
-  };
-  auto count_bins = [&]() {
-    if constexpr (RM > 0) {
-#pragma unroll
-      for (int k = 0; k < RM; ++k) count_one(k);
-    } else {
-      for (int k = 0; k < R; ++k) count_one(k);   // R is the same for the whole block
+    const unsigned b0 = __shfl_sync(0xffffffffu, bin, 0);
+    if (__all_sync(0xffffffffu, bin == b0)) {
+      if (lane == 0 && b0 < kSelBins) atomicAdd(&sh.bins[b0], 32u);
+    } else if (bin < kSelBins) {
+      atomicAdd(&sh.bins[bin], 1u);
     }
   };
   while (true) {
-    for (int q = tid; q < kSelBins; q += kSelThreads) sh.bins[q] = 0u;
-    __syncthreads();
-    count_bins();
+    if (shift >= 0) {   // round 0 counts into the bins cleared at the start
+      for (int q = tid; q < kSelBins; q += kSelThreads) sh.bins[q] = 0u;
+      __syncthreads();
+    }
+    for_rows(0, R, count_one);
     __syncthreads();
     sel_bin_from_top(sh, r);
     const unsigned bsel = sh.sel[0], above = sh.sel[1];
@@ -330,6 +355,79 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
       const unsigned hi = bsel == kSelBins - 1 ? 0x7F800001u   // the top bucket takes everything up to +inf
                                                : __float_as_uint(static_cast<float>(bsel + 1) * (1.0f / kSelBins));
       span = hi - lo;
+      const unsigned c = sh.bins[bsel];   // scores in the selected bucket (block-uniform)
+      if (c <= static_cast<unsigned>(kSelCand) && R <= kSelCompK) {
+        // kept masks per (row, warp): the scores above the bucket now, the bucket's own below
+        for_rows(0, R, [&](int k) {
+          const unsigned key = key_of(k);
+          const unsigned off = key - lo;
+          const bool in = has(k) && off < span;
+          const unsigned um = __ballot_sync(0xffffffffu, has(k) && key >= lo && off >= span);
+          if (lane == 0) {
+            sh.mgt[k][warp] = um;
+            sh.meq[k][warp] = 0u;
+          }
+          if (in) {
+            const unsigned pos = atomicAdd(&sh.ncand, 1u);
+            sh.cand[pos] = key;
+            sh.cidx[pos] = idx(k);
+          }
+        });
+        __syncthreads();
+        // a bucket score x with fewer than r bucket scores >= x lies above T; with fewer than r
+        // above it but at least r at or above it, x = T (and r - #above of them are kept)
+        if (tid < static_cast<int>(c)) {
+          const unsigned mine = sh.cand[tid];
+          unsigned gt = 0u, ge = 0u;
+          for (unsigned j = 0; j < c; ++j) {
+            const unsigned o = sh.cand[j];
+            gt += o > mine;
+            ge += o >= mine;
+          }
+          const int i = sh.cidx[tid];
+          const unsigned bit = 1u << (i & 31);
+          if (ge < r) {
+            atomicOr(&sh.mgt[i >> 10][(i >> 5) & 31], bit);
+          } else if (gt < r) {
+            atomicOr(&sh.meq[i >> 10][(i >> 5) & 31], bit);
+            sh.sel[1] = r - gt;   // the same value from every score equal to T
+          }
+        }
+        __syncthreads();
+        compact_rows(0, R, sh.sel[1], 0u, 0u);
+        return;
+      }
+      if (c <= static_cast<unsigned>(kSelCand)) {
+        // gather their keys (in any order) and rank them: the r-th largest is the key with fewer
+        // than r keys above it and at least r at or above it
+        for_rows(0, R, [&](int k) {
+          const unsigned key = key_of(k);
+          const bool in = has(k) && key - lo < span;
+          const unsigned m = __ballot_sync(0xffffffffu, in);
+          unsigned base = 0u;
+          if (lane == 0 && m != 0u) base = atomicAdd(&sh.ncand, static_cast<unsigned>(__popc(m)));
+          base = __shfl_sync(0xffffffffu, base, 0);
+          if (in) sh.cand[base + __popc(m & ((1u << lane) - 1u))] = key;
+        });
+        __syncthreads();
+        if (tid < static_cast<int>(c)) {
+          const unsigned mine = sh.cand[tid];
+          unsigned gt = 0u, ge = 0u;
+          for (unsigned j = 0; j < c; ++j) {
+            const unsigned o = sh.cand[j];
+            gt += o > mine;
+            ge += o >= mine;
+          }
+          if (gt < r && ge >= r) {   // every thread holding the threshold key writes the same pair
+            sh.sel[0] = mine;
+            sh.sel[1] = r - gt;
+          }
+        }
+        __syncthreads();
+        lo = sh.sel[0];
+        r = sh.sel[1];
+        break;
+      }
     } else {
       lo += bsel << shift;
       span = min(span - (bsel << shift), 1u << shift);
@@ -342,27 +440,24 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
   const unsigned T = lo;        // key of the K-th largest S_final
   const unsigned remaining = r; // how many keys equal to T are kept (lowest indices first)
 
-  // 6. ascending compaction from per-thread counts
-  unsigned gt = 0u, eq = 0u;
-  for_each_key([&](int, unsigned key) {
-    gt += key > T;
-    eq += key == T;
-  });
-  const unsigned gi = warp_incl_scan(gt), ei = warp_incl_scan(eq);
-  __syncthreads();   // the last round's readers of sh.sel / sh.wtot are done
-  if (lane == 31) { sh.wtot[warp] = gi; sh.wtot2[warp] = ei; }
-  __syncthreads();
-  unsigned g_before = gi - gt, e_before = ei - eq;
-  for (int w = 0; w < warp; ++w) { g_before += sh.wtot[w]; e_before += sh.wtot2[w]; }
-  for_each_key([&](int k, unsigned key) {
-    if (key > T) {
-      kept[k0 + g_before + min(e_before, remaining)] = v0 + i0 + k;
-      ++g_before;
-    } else if (key == T) {
-      if (e_before < remaining) kept[k0 + g_before + e_before] = v0 + i0 + k;
-      ++e_before;
-    }
-  });
+  // 6. compaction in index order, kSelCompK score rows at a time
+  unsigned gbase = 0u, ebase = 0u;   // keys above / equal to T in the rows before
+  for (int kb = 0; kb < R; kb += kSelCompK) {
+    const int ke = min(R, kb + kSelCompK);
+    __syncthreads();   // the previous readers of sh.sel / sh.mgt are done
+    for_rows(kb, ke, [&](int k) {
+      const unsigned key = key_of(k);
+      const unsigned gm = __ballot_sync(0xffffffffu, key > T), em = __ballot_sync(0xffffffffu, key == T && has(k));
+      if (lane == 0) {
+        sh.mgt[k - kb][warp] = gm;
+        sh.meq[k - kb][warp] = em;
+      }
+    });
+    __syncthreads();
+    const uint2 tot = compact_rows(kb, ke, remaining, gbase, ebase);
+    gbase = tot.x;
+    ebase = tot.y;
+  }
 }
 
 // One warp per 2 KB piece of a row (128 16-byte vectors, 4 per lane, all in flight), so that a
