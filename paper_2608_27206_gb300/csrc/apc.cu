@@ -11,8 +11,9 @@
 //   apc_pass2  same strips: c = sums / N, phi = |c|^2, c_hat = c / |c| (recomputed per
 //              CTA from the 589 integers), then d_i = |t_i - c_hat| computed directly from
 //              the staged pixels (no 2 - 2cos cancellation).
-//   apc_tail   one CTA per image: radix select of the k_tail-th largest d_i (fp32 bits),
-//              tail mean, rho_d, rho, r and the target size.
+//   apc_tail   one CTA per image: select of the k_tail-th largest d_i (value buckets, then the
+//              selected bucket's members ranked directly or by offset rounds over their fp32
+//              bits), tail mean, rho_d, rho, r and the target size.
 // Resize: apc_resample, four CTAs per SM walking the 16 x 32 output tiles of the batch; for
 // downscales up to 2.75x per side the input window is staged in shared memory and filtered
 // there with precomputed weights, steeper downscales take a generic path with per-tap weights.
@@ -81,6 +82,12 @@ __device__ __forceinline__ int find_image(const ApcTable& t, int unit) {
 // Asynchronous 4-byte global -> shared copies (no register round trip, all in flight at once).
 __device__ __forceinline__ void cp_async4(void* dst, const void* src) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+               "l"(src)
+               : "memory");
+}
+// 16-byte copy, both addresses 16-byte aligned (cached in L2 only).
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
                "l"(src)
                : "memory");
 }
@@ -581,8 +588,13 @@ constexpr int kTailSmemMax = 48 * 1024;   // d values staged in shared memory (f
 constexpr int kTailBins = 4096;            // level-1 buckets of the tail select
 constexpr int kTailBins2 = 1024;           // level-2 offset bins over a compacted bucket
 
-// Bucket of a distance d >= 0: floor(2048 d), capped at the top bucket (monotone in d).
-__device__ __forceinline__ int tail_bucket(float v) { return min(static_cast<int>(v * 2048.0f), kTailBins - 1); }
+// Bucket of a distance d >= 0: floor(2048 d), capped at the top bucket (monotone in d; NaN goes to
+// bucket 0).  Full-rate arithmetic only (no float-to-integer conversion): once clamped to
+// [0, 4095], 2048 d + 2^23 rounded toward zero holds floor(2048 d) in its low mantissa bits.
+__device__ __forceinline__ int tail_bucket(float v) {
+  const float x = fminf(fmaxf(v * 2048.0f, 0.0f), static_cast<float>(kTailBins - 1));
+  return __float_as_int(__fadd_rz(x, 8388608.0f)) - 0x4B000000;
+}
 
 // Called by all 1024 threads: the bin holding the r-th largest entry, counting from bin NBINS - 1
 // down (1 <= r <= total): sel[0] = that bin, sel[1] = entries in the bins above it.  wsum: 32 words.
@@ -635,7 +647,7 @@ __device__ __forceinline__ void select_from_top(const unsigned* bins, unsigned r
 
 __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTable t, const float* __restrict__ d,
                                                  TailParams prm, pace_apc_stats* __restrict__ stats) {
-  extern __shared__ float sd[];
+  extern __shared__ __align__(16) float sd[];
   __shared__ unsigned bins[kTailBins];
   __shared__ unsigned hist2[kTailBins2];
   __shared__ unsigned sel[2];
@@ -653,8 +665,16 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
   // shared-memory atomics, which the float's top bits (a few exponents) would not.  The
   // distances are staged in shared memory on the way, when they fit.
   if (N <= kTailSmemMax) {
-    for (int i = threadIdx.x; i < N; i += blockDim.x) cp_async4(sd + i, db + i);
-    db = sd;
+    // 16-byte copies for the 16-byte-aligned interior of db, 4-byte ones for the ends; the staged
+    // copy starts at db's offset within 16 bytes, so each interior copy is aligned at both ends
+    const int mis = static_cast<int>((reinterpret_cast<uintptr_t>(db) >> 2) & 3u);
+    float* s0 = sd + mis;
+    const int head = min(N, (4 - mis) & 3);
+    const int nvec = (N - head) >> 2;
+    for (int i = threadIdx.x; i < head; i += blockDim.x) cp_async4(s0 + i, db + i);
+    for (int v = threadIdx.x; v < nvec; v += blockDim.x) cp_async16(s0 + head + 4 * v, db + head + 4 * v);
+    for (int i = head + 4 * nvec + threadIdx.x; i < N; i += blockDim.x) cp_async4(s0 + i, db + i);
+    db = s0;
   }
   for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
   cp_async_wait_all();
@@ -681,47 +701,63 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
     __syncthreads();   // everyone has read sel and bins[tb]
     if (threadIdx.x == 0) ncomp = 0u;
     __syncthreads();
-    for (int base = 0; base < N; base += blockDim.x) {   // uniform trip count: __ballot_sync below
-      const int i = base + static_cast<int>(threadIdx.x);
-      const float v = i < N ? db[i] : 0.f;
-      const int bk = i < N ? tail_bucket(v) : -1;
+#pragma unroll 4
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {   // the members are few: one slot each
+      const float v = db[i];
+      const int bk = tail_bucket(v);
       if (bk > tb) {
         s += v;
         ++cnt;
-      }
-      const bool in = bk == tb;
-      const unsigned members = __ballot_sync(0xffffffffu, in);
-      if (members != 0u) {
-        const int leader = __ffs(members) - 1;
-        unsigned slot = 0u;
-        if (lane_id == leader) slot = atomicAdd(&ncomp, static_cast<unsigned>(__popc(members)));
-        slot = __shfl_sync(0xffffffffu, slot, leader);
-        if (in) bins[slot + __popc(members & ((1u << lane_id) - 1u))] = __float_as_uint(v);
+      } else if (bk == tb) {
+        bins[atomicAdd(&ncomp, 1u)] = __float_as_uint(v);
       }
     }
     __syncthreads();
-    while (true) {
-      const int bits = 32 - __clz(span - 1u);
-      const int shift = bits > 10 ? bits - 10 : 0;
-      for (int i = threadIdx.x; i < kTailBins2; i += blockDim.x) hist2[i] = 0u;
-      __syncthreads();
-      for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
-        const unsigned off = bins[i] - lo;   // wraps for keys below lo
-        if (off < span) atomicAdd(&hist2[off >> shift], 1u);
+    if (cb <= blockDim.x) {
+      // one member per thread, ranked against the whole list: a member with fewer than
+      // `remaining` members at or above it lies above the k-th largest (and is summed); with fewer
+      // than `remaining` above it but at least that many at or above it, it is the k-th largest
+      if (threadIdx.x < cb) {
+        const unsigned mine = bins[threadIdx.x];
+        unsigned gt = 0u, ge = 0u;
+        for (unsigned j = 0; j < cb; ++j) {
+          const unsigned o = bins[j];
+          gt += o > mine;
+          ge += o >= mine;
+        }
+        if (ge < remaining) {
+          s_fix += fix32(__uint_as_float(mine));
+          ++cnt;
+        } else if (gt < remaining) {
+          sel[0] = mine;   // the same key from every member equal to it
+        }
       }
       __syncthreads();
-      select_from_top<kTailBins2>(hist2, remaining, sel, cred);
-      lo += sel[0] << shift;
-      remaining -= sel[1];
-      if (shift == 0) break;
-      span = min(span - (sel[0] << shift), 1u << shift);
-    }
-    prefix = lo;
-    for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
-      const unsigned key = bins[i];
-      if (key > prefix) {
-        s_fix += fix32(__uint_as_float(key));
-        ++cnt;
+      prefix = sel[0];
+    } else {
+      while (true) {
+        const int bits = 32 - __clz(span - 1u);
+        const int shift = bits > 10 ? bits - 10 : 0;
+        for (int i = threadIdx.x; i < kTailBins2; i += blockDim.x) hist2[i] = 0u;
+        __syncthreads();
+        for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
+          const unsigned off = bins[i] - lo;   // wraps for keys below lo
+          if (off < span) atomicAdd(&hist2[off >> shift], 1u);
+        }
+        __syncthreads();
+        select_from_top<kTailBins2>(hist2, remaining, sel, cred);
+        lo += sel[0] << shift;
+        remaining -= sel[1];
+        if (shift == 0) break;
+        span = min(span - (sel[0] << shift), 1u << shift);
+      }
+      prefix = lo;
+      for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
+        const unsigned key = bins[i];
+        if (key > prefix) {
+          s_fix += fix32(__uint_as_float(key));
+          ++cnt;
+        }
       }
     }
   } else {
@@ -1391,7 +1427,8 @@ unsigned strip_grid(int units) {
 size_t tail_smem(const ApcTable& t) {
   int n = 0;
   for (int i = 0; i < t.nb; ++i) n = std::max(n, t.n[i]);
-  return n <= kTailSmemMax ? static_cast<size_t>(n) * sizeof(float) : 0;
+  // + 16 bytes: the staged copy keeps the distances' offset within 16 bytes
+  return n <= kTailSmemMax ? static_cast<size_t>(n) * sizeof(float) + 16 : 0;
 }
 
 pace_status_t tail_smem_attr() {
@@ -1400,7 +1437,7 @@ pace_status_t tail_smem_attr() {
   PACE_CUDA(cudaGetDevice(&dev));
   if (!once.done(dev)) {
     PACE_CUDA(cudaFuncSetAttribute(apc_tail, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                   static_cast<int>(kTailSmemMax * sizeof(float))));
+                                   static_cast<int>(kTailSmemMax * sizeof(float) + 16)));
     once.mark(dev);
   }
   return PACE_OK;
