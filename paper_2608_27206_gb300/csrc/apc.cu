@@ -717,14 +717,10 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
       // one member per thread, ranked against the whole list: a member with fewer than
       // `remaining` members at or above it lies above the k-th largest (and is summed); with fewer
       // than `remaining` above it but at least that many at or above it, it is the k-th largest
-      if (threadIdx.x < cb) {
-        const unsigned mine = bins[threadIdx.x];
-        unsigned gt = 0u, ge = 0u;
-        for (unsigned j = 0; j < cb; ++j) {
-          const unsigned o = bins[j];
-          gt += o > mine;
-          ge += o >= mine;
-        }
+      int mi;
+      unsigned gt, ge;
+      if (rank_in_list(bins, cb, mi, gt, ge)) {
+        const unsigned mine = bins[mi];
         if (ge < remaining) {
           s_fix += fix32(__uint_as_float(mine));
           ++cnt;

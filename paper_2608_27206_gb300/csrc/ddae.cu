@@ -14,6 +14,7 @@
 #include <cmath>
 
 #include "pace_common.cuh"
+#include "pace_select.cuh"
 
 namespace pace {
 namespace {
@@ -80,10 +81,19 @@ __device__ __forceinline__ unsigned warp_incl_scan(unsigned v) {
 // zero, negative and NaN scores take key 0, below every positive score.
 __device__ __forceinline__ unsigned sel_key(float f) { return f > 0.f ? __float_as_uint(f) : 0u; }
 
-// Value bucket of a key for the first selection round: floor(4096 f), capped at the top bucket
-// (monotone in the key; S_final lies in [0, 1]).
+// Bucket of a key for the first selection round: 64 buckets per octave of the score (the exponent
+// and the top 6 mantissa bits), from 2^-63 (bucket 0 takes everything below, key 0 included) to
+// the top bucket, which takes everything from about 1.98 up (S_final lies in [0, 1]).  Monotone in the
+// key, so a bucket is one key range: sel_bucket_lo(b) .. sel_bucket_lo(b + 1) - 1.  Fused scores
+// crowd near 0 when a map has a few large outliers; relative widths keep every bucket short
+// there as well as near 1.
+constexpr unsigned kSelKeyBase = 0x20000000u;   // 2^-63
+constexpr int kSelKeyShift = 17;
 __device__ __forceinline__ unsigned sel_bucket(unsigned key) {
-  return min(__float2uint_rz(__uint_as_float(key) * 4096.0f), static_cast<unsigned>(kSelBins - 1));
+  return key < kSelKeyBase ? 0u : min((key - kSelKeyBase) >> kSelKeyShift, static_cast<unsigned>(kSelBins - 1));
+}
+__device__ __forceinline__ unsigned sel_bucket_lo(unsigned b) {
+  return b == 0u ? 0u : b >= static_cast<unsigned>(kSelBins) ? 0x7F800001u : kSelKeyBase + (b << kSelKeyShift);
 }
 
 // The bin holding the r-th largest entry of sh.bins, counting from bin 4095 down (1 <= r <= total):
@@ -130,9 +140,9 @@ __device__ __forceinline__ void sel_bin_from_top(SelShared& sh, unsigned r) {
 //      population variances follow from those sums;
 //   3. the Eq. 7 weights (or a fixed ablation pair);
 //   4. S_final = alpha_w norm(S_llm) + beta_w norm(S_vis) (written out);
-//   5. the K-th largest S_final: 4096 value buckets; if the selected bucket holds at most 1024
-//      scores, their keys are gathered and ranked directly, else rounds of 4096 bins over the key
-//      bits inside the selected range run until one key T is left (exact either way);
+//   5. the K-th largest S_final: 4096 buckets (64 per octave); if the selected bucket holds at
+//      most 1024 scores, their keys are gathered and ranked directly, else rounds of 4096 bins
+//      over the key bits inside the selected range run until one key T is left (exact either way);
 //      for maps of up to 16384 scores with such a bucket, the pass that gathers the bucket also
 //      records which scores lie above it, and each bucket score places itself by its own rank,
 //      so 6. starts from those records;
@@ -314,10 +324,10 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
     return make_uint2(gbase + (tot & 0xFFFFu), ebase + (tot >> 16));
   };
 
-  // 5. the K-th largest key.  Round 0 counts value buckets; each later round splits the key
+  // 5. the K-th largest key.  Round 0 counts sel_bucket buckets; each later round splits the key
   // range [lo, lo + span) of the selected bin into 4096 bins of 2^shift keys until shift = 0.
   unsigned lo = 0u, span = 0u, r = static_cast<unsigned>(K);
-  int shift = -1;   // round 0: value buckets
+  int shift = -1;   // round 0: sel_bucket
   // Histogram of this round.  A warp whose 32 scores share one bin (a flat stretch of the map, or
   // ties) adds once; otherwise each lane adds for itself and the rare same-bin lanes are
   // serialised by the shared-memory atomics.
@@ -351,10 +361,8 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
     const unsigned bsel = sh.sel[0], above = sh.sel[1];
     r -= above;
     if (shift < 0) {
-      lo = __float_as_uint(static_cast<float>(bsel) * (1.0f / kSelBins));
-      const unsigned hi = bsel == kSelBins - 1 ? 0x7F800001u   // the top bucket takes everything up to +inf
-                                               : __float_as_uint(static_cast<float>(bsel + 1) * (1.0f / kSelBins));
-      span = hi - lo;
+      lo = sel_bucket_lo(bsel);
+      span = sel_bucket_lo(bsel + 1) - lo;   // the top bucket takes everything up to +inf
       const unsigned c = sh.bins[bsel];   // scores in the selected bucket (block-uniform)
       if (c <= static_cast<unsigned>(kSelCand) && R <= kSelCompK) {
         // kept masks per (row, warp): the scores above the bucket now, the bucket's own below
@@ -367,24 +375,24 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
             sh.mgt[k][warp] = um;
             sh.meq[k][warp] = 0u;
           }
-          if (in) {
-            const unsigned pos = atomicAdd(&sh.ncand, 1u);
-            sh.cand[pos] = key;
-            sh.cidx[pos] = idx(k);
+          const unsigned m = __ballot_sync(0xffffffffu, in);
+          if (m != 0u) {   // one slot claim per warp
+            unsigned base = 0u;
+            if (lane == 0) base = atomicAdd(&sh.ncand, static_cast<unsigned>(__popc(m)));
+            base = __shfl_sync(0xffffffffu, base, 0) + __popc(m & ((1u << lane) - 1u));
+            if (in) {
+              sh.cand[base] = key;
+              sh.cidx[base] = idx(k);
+            }
           }
         });
         __syncthreads();
         // a bucket score x with fewer than r bucket scores >= x lies above T; with fewer than r
         // above it but at least r at or above it, x = T (and r - #above of them are kept)
-        if (tid < static_cast<int>(c)) {
-          const unsigned mine = sh.cand[tid];
-          unsigned gt = 0u, ge = 0u;
-          for (unsigned j = 0; j < c; ++j) {
-            const unsigned o = sh.cand[j];
-            gt += o > mine;
-            ge += o >= mine;
-          }
-          const int i = sh.cidx[tid];
+        int ci;
+        unsigned gt, ge;
+        if (rank_in_list(sh.cand, c, ci, gt, ge)) {
+          const int i = sh.cidx[ci];
           const unsigned bit = 1u << (i & 31);
           if (ge < r) {
             atomicOr(&sh.mgt[i >> 10][(i >> 5) & 31], bit);
@@ -410,16 +418,11 @@ __global__ void __launch_bounds__(kSelThreads) ddae_select_kernel(const float* _
           if (in) sh.cand[base + __popc(m & ((1u << lane) - 1u))] = key;
         });
         __syncthreads();
-        if (tid < static_cast<int>(c)) {
-          const unsigned mine = sh.cand[tid];
-          unsigned gt = 0u, ge = 0u;
-          for (unsigned j = 0; j < c; ++j) {
-            const unsigned o = sh.cand[j];
-            gt += o > mine;
-            ge += o >= mine;
-          }
+        int ci;
+        unsigned gt, ge;
+        if (rank_in_list(sh.cand, c, ci, gt, ge)) {
           if (gt < r && ge >= r) {   // every thread holding the threshold key writes the same pair
-            sh.sel[0] = mine;
+            sh.sel[0] = sh.cand[ci];
             sh.sel[1] = r - gt;
           }
         }

@@ -48,4 +48,34 @@ __device__ __forceinline__ void warp_digit_search(const unsigned* hist, unsigned
   }
 }
 
+// Rank of every entry of a short list (c <= blockDim.x = 1024 keys in shared memory): gt = entries
+// above list[i], ge = entries at or above it.  Each entry's count is spread over P threads (P the
+// largest power of two with c P <= 1024, at most 32): thread t takes entry t / P and every P-th
+// comparison, and the P partial counts meet by shuffles inside their aligned group of lanes.
+// Every thread of the block calls it (its control flow is uniform per warp); it returns true on
+// the one thread per entry (part 0) that holds the complete counts.
+__device__ __forceinline__ bool rank_in_list(const unsigned* list, unsigned c, int& i, unsigned& gt, unsigned& ge) {
+  unsigned P = 1u;
+  while (P < 32u && 2u * P * c <= blockDim.x) P <<= 1;
+  const unsigned t = threadIdx.x;
+  gt = ge = 0u;
+  i = static_cast<int>(t / P);
+  if ((t & ~31u) >= c * P) return false;   // the whole warp is past the list
+  const unsigned part = t & (P - 1u);
+  const bool valid = static_cast<unsigned>(i) < c;
+  if (valid) {
+    const unsigned mine = list[i];
+    for (unsigned j = part; j < c; j += P) {
+      const unsigned o = list[j];
+      gt += o > mine;
+      ge += o >= mine;
+    }
+  }
+  for (unsigned o = 1u; o < P; o <<= 1) {
+    gt += __shfl_xor_sync(0xffffffffu, gt, static_cast<int>(o));
+    ge += __shfl_xor_sync(0xffffffffu, ge, static_cast<int>(o));
+  }
+  return valid && part == 0u;
+}
+
 }  // namespace pace
