@@ -128,9 +128,6 @@ __device__ __forceinline__ float warp_sum_f(float v) {
   return v;
 }
 
-// Exact uint8 -> float without the conversion pipe: 2^23 + v has v in its low mantissa bits.
-__device__ __forceinline__ float byte_to_float(uint32_t v) { return __uint_as_float(0x4B000000u | v) - 8388608.0f; }
-
 // The two bytes of a 16-bit pair as floats: byte permutes build 2^23 + b in each word, one packed
 // subtract removes the 2^23.
 __device__ __forceinline__ float2 bytes2_to_float2(uint32_t v) {
@@ -1297,45 +1294,63 @@ __device__ __forceinline__ void resample_tile_fast(const uint8_t* __restrict__ i
     // holds kFCols >= the window of the last column + MAXT pixels)
     const int c = tt / 3, ch = tt - 3 * c;
     const int n = xn[c];
+    // A byte b enters as the float 1 + b / 256 (b in the top 8 mantissa bits of 1.0, one integer
+    // multiply-add), so sum_k w_k (1 + b_k / 256) = W + (sum_k w_k b_k) / 256 with W = sum_k w_k;
+    // the accumulators stay in [1, 2) (fp32 steps of 2^-23, i.e. 3e-5 in pixel units after the
+    // final 256 (acc - W)), and two rows share each packed FMA.
     float w[MAXT];
+    float wsum = 0.f;
 #pragma unroll
-    for (int k = 0; k < MAXT; ++k) w[k] = k < n ? wx[c * kFMaxTaps + k] : 0.f;
+    for (int k = 0; k < MAXT; ++k) {
+      w[k] = k < n ? wx[c * kFMaxTaps + k] : 0.f;
+      wsum += w[k];
+    }
+    const float2 post = make_float2(-256.0f * wsum, -256.0f * wsum);
+    const float2 k256 = make_float2(256.0f, 256.0f);
+    auto unit = [](unsigned b) { return __uint_as_float(b * 32768u + 0x3F800000u); };
     const int base = (xlo[c] - x0) * 3 + ch;
     const int r_end = half ? nin_r : (nin_r + 1) / 2;
     int r = half ? (nin_r + 1) / 2 : 0;
     for (; r + 1 < r_end; r += 2) {   // two rows at a time: twice the independent work in flight
       const unsigned char* px0 = sin + r * kFPitch + shift[r] + base;
       const unsigned char* px1 = sin + (r + 1) * kFPitch + shift[r + 1] + base;
-      float acc0 = 0.f, acc1 = 0.f;
+      float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
-      for (int k = 0; k < MAXT; ++k) {
-        acc0 = fmaf(w[k], byte_to_float(px0[3 * k]), acc0);
-        acc1 = fmaf(w[k], byte_to_float(px1[3 * k]), acc1);
-      }
-      sh[r * kFLine + tt] = acc0;
-      sh[(r + 1) * kFLine + tt] = acc1;
+      for (int k = 0; k < MAXT; ++k)
+        acc = ptx::ffma2(make_float2(w[k], w[k]), make_float2(unit(px0[3 * k]), unit(px1[3 * k])), acc);
+      const float2 h = ptx::ffma2(acc, k256, post);
+      sh[r * kFLine + tt] = h.x;
+      sh[(r + 1) * kFLine + tt] = h.y;
     }
     if (r < r_end) {
       const unsigned char* px = sin + r * kFPitch + shift[r] + base;
       float acc = 0.f;
 #pragma unroll
-      for (int k = 0; k < MAXT; ++k) acc = fmaf(w[k], byte_to_float(px[3 * k]), acc);
-      sh[r * kFLine + tt] = acc;
+      for (int k = 0; k < MAXT; ++k) acc = fmaf(w[k], unit(px[3 * k]), acc);
+      sh[r * kFLine + tt] = fmaf(acc, 256.0f, post.x);
     }
   }
   __syncthreads();
-  if (tt < 3 * ncol) {
-    // vertical pass and the uint8 store (a row of the tile is 3 * ncol consecutive bytes); the
-    // halves take alternate output rows
-    uint8_t* o = out + (static_cast<int64_t>(oy0) * Wo + ox0) * 3 + tt;
-    for (int r = half; r < nrow; r += 2) {
+  // vertical pass and the uint8 store (a row of the tile is 3 * ncol consecutive bytes): thread
+  // (g, p) of 4 x 48 filters line entries 2p and 2p + 1 of output rows g, g + 4, .. with one
+  // 8-byte load and one packed FMA per tap (entry 3 * ncol, past the line when it is odd, holds
+  // whatever the buffer held and is not stored)
+  constexpr int kVPairs = kFLine / 2;
+  static_assert(4 * kVPairs <= kRsThreads, "thread roles of the vertical pass");
+  const int vg = tid / kVPairs, t0 = 2 * (tid - vg * kVPairs);
+  if (vg < 4 && t0 < 3 * ncol) {
+    const bool two = t0 + 1 < 3 * ncol;
+    uint8_t* o = out + (static_cast<int64_t>(oy0) * Wo + ox0) * 3 + t0;
+    for (int r = vg; r < nrow; r += 4) {
       const float* w = wy + r * kFMaxTaps;
-      const float* col = sh + (ylo[r] - y0) * kFLine + tt;
+      const float2* col = reinterpret_cast<const float2*>(sh + (ylo[r] - y0) * kFLine + t0);
       const int n = yn[r];
-      float acc = 0.f;
+      float2 acc = make_float2(0.f, 0.f);
 #pragma unroll 4
-      for (int k = 0; k < n; ++k) acc = fmaf(w[k], col[k * kFLine], acc);
-      o[static_cast<int64_t>(r) * Wo * 3] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc))));
+      for (int k = 0; k < n; ++k) acc = ptx::ffma2(make_float2(w[k], w[k]), col[k * kVPairs], acc);
+      uint8_t* orow = o + static_cast<int64_t>(r) * Wo * 3;
+      orow[0] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc.x))));
+      if (two) orow[1] = static_cast<uint8_t>(min(255, max(0, __float2int_rn(acc.y))));
     }
   }
   __syncthreads();   // the shared buffers are reused by the next tile
