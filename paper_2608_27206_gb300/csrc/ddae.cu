@@ -500,6 +500,37 @@ __global__ void __launch_bounds__(256) gather_rows_v16(const uint4* __restrict__
   }
 }
 
+// Rows of up to 32 U 16-byte vectors: one warp per row, grid-stride over the kept rows; every
+// vector of a row is in flight at once (U per lane), and the warp reads its next row's index
+// before it stores this one, so a row costs one memory round trip.
+template <int U>
+__global__ void __launch_bounds__(128) gather_rows_warp(const uint4* __restrict__ src, int64_t n_src, int row_vec,
+                                                        const int32_t* __restrict__ idx, int64_t n_idx,
+                                                        uint4* __restrict__ dst, int* status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 5;
+  int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  int64_t s_next = r < n_idx ? __ldg(idx + r) : 0;
+  for (; r < n_idx; r += nwarps) {
+    const int64_t s = s_next;
+    if (r + nwarps < n_idx) s_next = __ldg(idx + r + nwarps);
+    uint4* dp = dst + r * row_vec;
+    if (s < 0 || s >= n_src) {
+      for (int c = lane; c < row_vec; c += 32) dp[c] = make_uint4(0u, 0u, 0u, 0u);
+      if (lane == 0) record_error(status, PACE_ERR_INVALID_ARG, K_GATHER);
+      continue;
+    }
+    const uint4* sp = src + s * row_vec;
+    uint4 v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (u * 32 + lane < row_vec) v[u] = __ldcs(sp + u * 32 + lane);
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (u * 32 + lane < row_vec) __stcs(dp + u * 32 + lane, v[u]);
+  }
+}
+
 // Byte-granular fallback for rows that are not 16-byte multiples or not 16-byte aligned.
 __global__ void __launch_bounds__(256) gather_rows_bytes(const uint8_t* __restrict__ src, int64_t n_src,
                                                          int64_t row_bytes, const int32_t* __restrict__ idx,
@@ -681,7 +712,20 @@ extern "C" pace_status_t pace_gather(const void* src, int64_t n_src_rows, int64_
   if (blocks > cap) blocks = cap;
   const bool vec = (row_bytes % 16 == 0) && (reinterpret_cast<uintptr_t>(src) % 16 == 0) &&
                    (reinterpret_cast<uintptr_t>(dst) % 16 == 0);
-  if (vec) {
+  const int64_t row_vec = row_bytes / 16;
+  if (vec && row_vec <= 32 * 16) {
+    // a warp per row: enough resident warps for every SM (about 24 per SM at U = 16), no more
+    // than there are rows
+    // than there are rows; blocks of 4 warps, so that a few thousand rows still reach every SM
+    const int64_t b = std::min<int64_t>((n_idx + 3) / 4, static_cast<int64_t>(sms) * 8);
+    const unsigned g = static_cast<unsigned>(b);
+    const int rv = static_cast<int>(row_vec);
+    const uint4* s4 = static_cast<const uint4*>(src);
+    uint4* d4 = static_cast<uint4*>(dst);
+    if (row_vec <= 32 * 4) gather_rows_warp<4><<<g, 128, 0, stream>>>(s4, n_src_rows, rv, idx, n_idx, d4, status);
+    else if (row_vec <= 32 * 8) gather_rows_warp<8><<<g, 128, 0, stream>>>(s4, n_src_rows, rv, idx, n_idx, d4, status);
+    else gather_rows_warp<16><<<g, 128, 0, stream>>>(s4, n_src_rows, rv, idx, n_idx, d4, status);
+  } else if (vec) {
     const int64_t pieces = (row_bytes / 16 + kGatherPiece - 1) / kGatherPiece;
     blocks = std::min<int64_t>((n_idx * pieces + warps_per_block - 1) / warps_per_block, static_cast<int64_t>(sms) * 8);
     gather_rows_v16<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
