@@ -222,72 +222,98 @@ def oracle_pool(n=None):
     return mp.get_context("spawn").Pool(n), n
 
 
-def oracle_timing(wl, keep, pool, vit_rows, density_crop_div=1):
-    """Times the fp64 oracle on one 4K image of the workload, on the host cores.
+class OracleTimer:
+    """Times the fp64 oracle on one 4K image of the workload, on the host cores, part by part.
 
     density : the whole image (density_crop_div = 1: Eq. 1 summed over all N^2 pairs), or a
               centred crop with 1/density_crop_div of each side, scaled by (N / N_crop)^2;
     resample: the whole image to the oracle's target size;
-    S_vis   : every head, the first vit_rows query rows of each against all keys, one job per head
-              on the pool; scaled by N / vit_rows (the rows' softmaxes are independent, so the work
-              is exactly proportional to the rows);
-    S_llm, fusion, top-K, gather: the whole image.
-    Returns (seconds per image, measured seconds, parts, description).
+    vit     : S_vis of every head, the first vit_rows query rows of each against all keys, one job
+              per head on the pool; scaled by N / vit_rows (the rows' softmaxes are independent, so
+              the work is exactly proportional to the rows);
+    llm     : S_llm of the whole image;
+    select  : fusion + top-K of the whole image, then the gather of the kept embedding rows.
+    time(part) returns {name: seconds per image} and the seconds measured.  density comes before
+    resample (the target size) and llm before select (the S_llm map).
     """
-    from oracle import pace_oracle as O
-    from paper_2608_27206_gb300 import synth
-    img = wl.images[0]
-    H, W = img.shape[:2]
-    t, measured = {}, 0.0
-    if density_crop_div > 1:
-        ch, cw = (H // density_crop_div) // 14 * 14, (W // density_crop_div) // 14 * 14
-        y0, x0 = (H - ch) // 2 // 14 * 14, (W - cw) // 2 // 14 * 14
-        crop = np.ascontiguousarray(img[y0:y0 + ch, x0:x0 + cw])
-        n_full, n_crop = (H // 14) * (W // 14), (ch // 14) * (cw // 14)
+    PARTS = ("density", "resample", "vit", "llm", "select")
+
+    def __init__(self, wl, keep, pool, vit_rows, density_crop_div=1):
+        from oracle import pace_oracle as O
+        from paper_2608_27206_gb300 import synth
+        self.O, self.synth, self.wl, self.keep, self.pool = O, synth, wl, keep, pool
+        self.vit_rows, self.crop_div = vit_rows, density_crop_div
+        self.img = wl.images[0]
+        self.size, self.s_llm = None, None
+
+    def time(self, part):
+        O, wl, img = self.O, self.wl, self.img
+        H, W = img.shape[:2]
+        if part == "density":
+            if self.crop_div > 1:
+                ch, cw = (H // self.crop_div) // 14 * 14, (W // self.crop_div) // 14 * 14
+                y0, x0 = (H - ch) // 2 // 14 * 14, (W - cw) // 2 // 14 * 14
+                crop = np.ascontiguousarray(img[y0:y0 + ch, x0:x0 + cw])
+                n_full, n_crop = (H // 14) * (W // 14), (ch // 14) * (cw // 14)
+                t0 = time.perf_counter()
+                st = O.apc_density(crop)
+                dt = time.perf_counter() - t0
+                self.size = O.target_size(H, W, O.retention_ratio(st["rho"]))
+                return {"density": dt * (n_full / n_crop) ** 2}, dt
+            t0 = time.perf_counter()
+            st = O.apc_density(img)
+            dt = time.perf_counter() - t0
+            self.size = (st["H_out"], st["W_out"])
+            return {"density": dt}, dt
+        if part == "resample":
+            t0 = time.perf_counter()
+            O.apc_resample(img, *self.size)
+            dt = time.perf_counter() - t0
+            return {"resample": dt}, dt
+        if part == "vit":
+            n, heads = wl.vit_q.shape[0], wl.vit_q.shape[1]
+            R = min(self.vit_rows, n)
+            jobs = [(np.ascontiguousarray(wl.vit_q[:R, h]), np.ascontiguousarray(wl.vit_k[:, h]), 1 / math.sqrt(80))
+                    for h in range(heads)]
+            t0 = time.perf_counter()
+            self.pool.starmap(_vit_rows_job, jobs, chunksize=1)
+            dt = time.perf_counter() - t0
+            return {"vit": dt * n / R}, dt
+        if part == "llm":
+            ql, kl = self.synth.bf16_bits_to_f64(wl.llm_q), self.synth.bf16_bits_to_f64(wl.llm_k)
+            t0 = time.perf_counter()
+            self.s_llm = O.llm_text_visual_importance(ql, kl, wl.cu_q, wl.cu_vis, 1 / math.sqrt(128))
+            dt = time.perf_counter() - t0
+            return {"llm": dt}, dt
+        s_vis = np.random.default_rng(0).lognormal(size=wl.n_vis[0])  # stand-in map for timing only
+        K = O.budget(wl.n_vis[0], self.keep)
         t0 = time.perf_counter()
-        st = O.apc_density(crop)
-        dt = time.perf_counter() - t0
-        t["density"] = dt * (n_full / n_crop) ** 2
-        ho, wo = O.target_size(H, W, O.retention_ratio(st["rho"]))
-        dens_desc = f"density on a {cw}x{ch} centre crop scaled by (N/N_crop)^2"
-    else:
-        t0 = time.perf_counter()
-        st = O.apc_density(img)
-        dt = time.perf_counter() - t0
-        t["density"] = dt
-        ho, wo = st["H_out"], st["W_out"]
-        dens_desc = "density of the whole image"
-    measured += dt
-    t0 = time.perf_counter()
-    O.apc_resample(img, ho, wo)
-    t["resample"] = time.perf_counter() - t0
-    measured += t["resample"]
-    n, heads = wl.vit_q.shape[0], wl.vit_q.shape[1]
-    R = min(vit_rows, n)
-    jobs = [(np.ascontiguousarray(wl.vit_q[:R, h]), np.ascontiguousarray(wl.vit_k[:, h]), 1 / math.sqrt(80))
-            for h in range(heads)]
-    t0 = time.perf_counter()
-    pool.starmap(_vit_rows_job, jobs, chunksize=1)
-    dt = time.perf_counter() - t0
-    t["vit"] = dt * n / R
-    measured += dt
-    ql, kl = synth.bf16_bits_to_f64(wl.llm_q), synth.bf16_bits_to_f64(wl.llm_k)
-    t0 = time.perf_counter()
-    s_llm = O.llm_text_visual_importance(ql, kl, wl.cu_q, wl.cu_vis, 1 / math.sqrt(128))
-    t["llm"] = time.perf_counter() - t0
-    s_vis = np.random.default_rng(0).lognormal(size=wl.n_vis[0])  # stand-in map for timing only
-    K = O.budget(wl.n_vis[0], keep)
-    t0 = time.perf_counter()
-    sel = O.ddae_select(s_llm, s_vis, wl.cu_vis, [K])
-    t["select"] = time.perf_counter() - t0
-    t0 = time.perf_counter()
-    O.gather_rows(wl.embed, sel["kept"])
-    t["gather"] = time.perf_counter() - t0
-    measured += t["llm"] + t["select"] + t["gather"]
-    desc = (f"fp64 numpy oracle on {pool._processes} host processes: {dens_desc}; resample of the whole image; "
-            f"S_vis for all {heads} heads x the first {R} of {n} query rows (one pool job per head), scaled "
-            f"by {n}/{R}; S_llm, fusion, top-K, gather of the whole image")
-    return sum(t.values()), measured, t, desc
+        sel = O.ddae_select(self.s_llm, s_vis, wl.cu_vis, [K])
+        t1 = time.perf_counter()
+        O.gather_rows(wl.embed, sel["kept"])
+        t2 = time.perf_counter()
+        return {"select": t1 - t0, "gather": t2 - t1}, t2 - t0
+
+    def description(self):
+        n, heads = self.wl.vit_q.shape[0], self.wl.vit_q.shape[1]
+        R = min(self.vit_rows, n)
+        dens = (f"density on a 1/{self.crop_div}-side centre crop scaled by (N/N_crop)^2" if self.crop_div > 1
+                else "density of the whole image")
+        return (f"fp64 numpy oracle on {self.pool._processes} host processes: {dens}; resample of the whole "
+                f"image; S_vis for all {heads} heads x the first {R} of {n} query rows (one pool job per head), "
+                f"scaled by {n}/{R}; S_llm, fusion, top-K, gather of the whole image")
+
+
+def oracle_timing(wl, keep, pool, vit_rows, density_crop_div=1):
+    """Every part of OracleTimer once, in order.
+    Returns (seconds per image, measured seconds, parts, description)."""
+    timer = OracleTimer(wl, keep, pool, vit_rows, density_crop_div)
+    parts, measured = {}, 0.0
+    for part in OracleTimer.PARTS:
+        t, dt = timer.time(part)
+        parts.update(t)
+        measured += dt
+    return sum(parts.values()), measured, parts, timer.description()
 
 
 def run_reference(args):
@@ -298,19 +324,28 @@ def run_reference(args):
     wl = synth.make_workload(WORKLOAD, seed=0, keep=KEEP, parts=("image", "vit", "llm", "embed"))
     pool, cores = oracle_pool()
     try:
-        # each step is a bounded sample of the image's work (a few seconds on the host cores)
-        for _ in range(args.warmup):
-            oracle_timing(wl, KEEP, pool, args.ref_vit_rows, density_crop_div=4)
-        per_image, sample_s, parts, sample = [], [], None, ""
-        for _ in range(args.steps):
-            tot, meas, parts, sample = oracle_timing(wl, KEEP, pool, args.ref_vit_rows, density_crop_div=4)
-            per_image.append(tot)
-            sample_s.append(meas)
+        # Step s times one part of the image's work (OracleTimer.PARTS in turn, about half a second
+        # at most on the host cores), so --steps K --warmup W stays within a few minutes for any K;
+        # the per-image value is the sum of the parts' mean per-image times.
+        timer = OracleTimer(wl, KEEP, pool, args.ref_vit_rows, density_crop_div=4)
+        parts_all = OracleTimer.PARTS
+        timed, warm, sample_s = {}, {}, []
+        n_all = max(args.warmup + args.steps, len(parts_all))   # every part at least once
+        for s in range(n_all):
+            t, dt = timer.time(parts_all[s % len(parts_all)])
+            dest = timed if args.warmup <= s < args.warmup + args.steps else warm
+            for k, v in t.items():
+                dest.setdefault(k, []).append(v)
+            if args.warmup <= s < args.warmup + args.steps:
+                sample_s.append(dt)
+        parts = {k: float(np.mean(timed.get(k) or warm[k])) for k in set(timed) | set(warm)}
+        sample = (timer.description() + "; one part per step (" + ", ".join(parts_all) +
+                  " in turn), per image = the sum of the parts' means")
     finally:
         pool.close()
         pool.join()
-    value = float(np.mean(per_image)) * 1e6
-    ms_step = float(np.mean(sample_s)) * 1e3
+    value = sum(parts.values()) * 1e6
+    ms_step = float(np.mean(sample_s)) * 1e3 if sample_s else 0.0
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": False,

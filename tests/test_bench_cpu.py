@@ -56,3 +56,62 @@ def test_reference_arm_only_rank0_works(monkeypatch, capsys):
     args = types.SimpleNamespace(gpus=2, steps=1, warmup=3, ref_vit_rows=64)
     assert bench.run_reference(args) == 0
     assert capsys.readouterr().out == ""      # other ranks print nothing and do no work
+
+
+def test_reference_arm_times_one_part_per_step(monkeypatch, capsys):
+    """Rank 0 of the reference arm: step s times part s mod 5 only (a bounded sample per step),
+    the per-image value is the sum of the parts' means over the timed steps, and a run with
+    fewer steps than parts still measures every part once."""
+    import json
+    from paper_2608_27206_gb300 import synth
+
+    calls = []
+
+    class FakeTimer:
+        PARTS = ("density", "resample", "vit", "llm", "select")
+        cost = {"density": 1.0, "resample": 2.0, "vit": 30.0, "llm": 0.5, "select": 0.25}
+
+        def __init__(self, *a, **k):
+            self.n = 0
+
+        def time(self, part):
+            self.n += 1
+            calls.append(part)
+            # per-image seconds drift with the call count, so the mean over timed steps is checked
+            return {part: self.cost[part] + 0.01 * self.n}, 0.1
+
+        def description(self):
+            return "fake"
+
+    class FakePool:
+        def close(self):
+            pass
+
+        def join(self):
+            pass
+
+    monkeypatch.setenv("RANK", "0")
+    monkeypatch.setattr(bench, "OracleTimer", FakeTimer)
+    monkeypatch.setattr(bench, "oracle_pool", lambda n=None: (FakePool(), 4))
+    monkeypatch.setattr(bench, "workload_config", lambda wl, keep: {"workload": "fake"})
+    monkeypatch.setattr(synth, "make_workload", lambda *a, **k: object())
+
+    args = types.SimpleNamespace(gpus=1, steps=10, warmup=2, ref_vit_rows=64)
+    assert bench.run_reference(args) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert calls == [FakeTimer.PARTS[s % 5] for s in range(12)]
+    # timed steps are calls 3..12 (n = 3..12); part p was timed at the n with (n - 1) % 5 == index
+    expect = 0.0
+    for i, p in enumerate(FakeTimer.PARTS):
+        ns = [n for n in range(3, 13) if (n - 1) % 5 == i]
+        expect += sum(FakeTimer.cost[p] + 0.01 * n for n in ns) / len(ns)
+    assert line["impl"] == "reference" and line["steps"] == 10 and line["warmup"] == 2
+    assert line["value"] == pytest.approx(expect * 1e6)
+    assert line["ms_per_step"] == pytest.approx(100.0)
+
+    calls.clear()
+    args = types.SimpleNamespace(gpus=1, steps=1, warmup=0, ref_vit_rows=64)
+    assert bench.run_reference(args) == 0
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert calls == list(FakeTimer.PARTS)          # one timed step, four extra to cover every part
+    assert set(line["cpu_baseline"]["parts_s_per_image"]) == set(FakeTimer.PARTS)
