@@ -11,7 +11,8 @@ arrays shaped like Qwen2.5-VL-7B (3836x2156 image: 42196 patches, ViT Q/K
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
 Prints one JSON line.  `value` is microseconds per image with inputs resident in HBM,
-timed with CUDA events around each step (each libpace call replayed from a CUDA graph),
+timed with CUDA events around each step (the step's libpace calls replayed as three CUDA graphs:
+the calls before the ViT call, the ViT call, the calls after it),
 L2 flushed by a 256 MiB write before every step.  `e2e` is the same metric through the
 Python binding with the inputs copied from pinned host memory and the results copied
 back inside the timed region (two device input slots, so one image's copies run under the
@@ -131,7 +132,10 @@ def workload_config(wl, keep):
         "images_per_step_per_gpu": 1,
         "keep_fraction": keep,
         "l2": "flushed before every timed step by a 256 MiB device write",
-        "timing": "CUDA events on the launching stream around each step; each libpace call replayed from a CUDA graph",
+        "timing": "CUDA events on the launching stream around each step; the step's libpace calls replayed as "
+                  "three CUDA graphs (before the ViT call, the ViT call, after it); the ViT roofline time from "
+                  "events around its graph in the timed region, the other calls' breakdown from their own "
+                  "graphs outside it",
     }
 
 
@@ -383,6 +387,25 @@ def capture_graphs(pipe):
     return graphs
 
 
+def capture_step_graphs(pipe, alone="vit"):
+    """The whole step as three CUDA graphs: the calls before `alone`, `alone` itself, the calls
+    after it (so that the timed region can put CUDA events around that one call)."""
+    import torch
+    names = [n for n, _ in pipe.parts]
+    i = names.index(alone)
+    segs = []
+    for label, sl in (("before", pipe.parts[:i]), (alone, pipe.parts[i:i + 1]), ("after", pipe.parts[i + 1:])):
+        if not sl:
+            continue
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for _, f in sl:
+                f()
+        segs.append((label, g))
+    torch.cuda.synchronize()
+    return segs
+
+
 def algorithmic_counts(wl, keep, r_ratio):
     """Algorithmic flops / bytes per step (one image), per part."""
     n, nv = wl.n_patches[0], wl.n_vis[0]
@@ -565,8 +588,9 @@ def part_rooflines(cnt, part_us, peak_tf, hbm):
     return out
 
 
-def time_graphs(graphs, flush, steps):
-    """Per-part and per-step CUDA-event times (ms) of `steps` replays, L2 flushed before each."""
+def time_parts(graphs, flush, steps):
+    """Per-part CUDA-event times (ms): `steps` replays of the per-call graphs in step order, L2
+    flushed before each step, an event between calls."""
     import torch
     nparts = len(graphs)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nparts + 1)] for _ in range(steps)]
@@ -577,17 +601,31 @@ def time_graphs(graphs, flush, steps):
             g.replay()
             ev[k][i + 1].record()
     torch.cuda.synchronize()
-    part = {name: statistics.mean(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(steps))
+    return {name: statistics.mean(ev[k][i].elapsed_time(ev[k][i + 1]) for k in range(steps))
             for i, (name, _) in enumerate(graphs)}
-    step = statistics.mean(ev[k][0].elapsed_time(ev[k][nparts]) for k in range(steps))
-    return part, step
+
+
+def time_graphs(graphs, step_graphs, flush, steps):
+    """Per-part times (ms) as time_parts, and the step time (ms): `steps` replays of the step's
+    graphs (capture_step_graphs), L2 flushed before each step, CUDA events around the step."""
+    import torch
+    part = time_parts(graphs, flush, steps)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for k in range(steps):
+        flush.zero_()
+        ev[k][0].record()
+        for _, g in step_graphs:
+            g.replay()
+        ev[k][1].record()
+    torch.cuda.synchronize()
+    return part, statistics.mean(a.elapsed_time(b) for a, b in ev)
 
 
 def measure_configs(P, device, flush, peak_tf, hbm, steps=10):
     """The other workloads of the benchmark (448^2, 1344^2, 1904x1064 with sinks, the ragged
-    16-image batch): the whole step through HotPath, each call replayed from a CUDA graph, L2
-    flushed before every step; microseconds per image, the per-call breakdown and each call's
-    roofline fraction."""
+    16-image batch): the whole step through HotPath replayed as one CUDA graph, L2 flushed before
+    every step; microseconds per image, the per-call breakdown (each call replayed from its own
+    graph) and each call's roofline fraction."""
     import torch
     from paper_2608_27206_gb300 import synth
     from paper_2608_27206_gb300.hotpath import HotPath
@@ -596,12 +634,13 @@ def measure_configs(P, device, flush, peak_tf, hbm, steps=10):
         wl = synth.make_workload(name, seed=0)
         pipe = HotPath(wl, device)
         graphs = capture_graphs(pipe)
+        step_graphs = capture_step_graphs(pipe)
         for _ in range(3):
             flush.zero_()
-            for _, g in graphs:
+            for _, g in step_graphs:
                 g.replay()
         torch.cuda.synchronize()
-        part_ms, step_ms = time_graphs(graphs, flush, steps)
+        part_ms, step_ms = time_graphs(graphs, step_graphs, flush, steps)
         code, where = P.pace_device_status(clear=True)
         if code != 0:
             raise RuntimeError(f"device status {code} from kernel {where} in config {name}")
@@ -612,7 +651,7 @@ def measure_configs(P, device, flush, peak_tf, hbm, steps=10):
                      "visual_tokens": int(sum(wl.n_vis)), "patches": int(sum(wl.n_patches)),
                      "breakdown_us": {k: round(v, 2) for k, v in part_us.items()},
                      "rooflines": part_rooflines(cnt, part_us, peak_tf, hbm)}
-        del pipe, graphs
+        del pipe, graphs, step_graphs
         torch.cuda.empty_cache()
     return out
 
@@ -715,17 +754,20 @@ def run_gpu(args):
     torch.cuda.synchronize()
     launches_per_step = P.pace_kernel_launch_count() - c0
     graphs = capture_graphs(pipe)
+    step_graphs = capture_step_graphs(pipe)
     for _ in range(args.warmup):
         flush.zero_()
-        for _, g in graphs:
+        for _, g in step_graphs:
             g.replay()
     torch.cuda.synchronize()
     code, where = P.pace_device_status(clear=True)
     if code != 0:
         raise RuntimeError(f"device status {code} from kernel {where} during warm-up")
 
-    nparts = len(graphs)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nparts + 1)] for _ in range(args.steps)]
+    # timed region: the step as three graphs (the calls before the ViT call, the ViT call, the calls
+    # after it), CUDA events around the step and around the ViT call
+    nseg = len(step_graphs)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nseg + 1)] for _ in range(args.steps)]
     sampler = ClockSampler(torch.cuda.current_device())
     sampler.start()
     if world > 1:
@@ -735,7 +777,7 @@ def run_gpu(args):
     for k in range(args.steps):
         flush.zero_()
         ev[k][0].record()
-        for i, (_, g) in enumerate(graphs):
+        for i, (_, g) in enumerate(step_graphs):
             g.replay()
             ev[k][i + 1].record()
     torch.cuda.synchronize()
@@ -743,12 +785,13 @@ def run_gpu(args):
         dist.barrier()
     t_wall = time.perf_counter() - t_wall0
     clocks = sampler.stop()
-    part_ms = {name: [] for name, _ in graphs}
-    step_ms = []
-    for k in range(args.steps):
-        step_ms.append(ev[k][0].elapsed_time(ev[k][nparts]))
-        for i, (name, _) in enumerate(graphs):
-            part_ms[name].append(ev[k][i].elapsed_time(ev[k][i + 1]))
+    step_ms = [e[0].elapsed_time(e[nseg]) for e in ev]
+    iv = [n for n, _ in step_graphs].index("vit")
+    vit_timed_ms = [e[iv].elapsed_time(e[iv + 1]) for e in ev]
+    # the other calls' breakdown, outside the timed region: each call from its own graph, an event
+    # between calls; the ViT entry is the timed region's own
+    part_ms = {k: [v] for k, v in time_parts(graphs, flush, min(args.steps, 20)).items()}
+    part_ms["vit"] = vit_timed_ms
     total_ms = max_over_ranks(float(sum(step_ms)), world, device)
     ms_per_step = total_ms / args.steps
     value = per_image_us(total_ms, args.steps, world)
