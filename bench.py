@@ -73,19 +73,20 @@ def source_hash():
     return hashlib.sha256(open(ATTN_SRC, "rb").read()).hexdigest()[:16]
 
 
-def profiled_traffic():
+def profiled_traffic(with_algorithmic=False):
     """DRAM bytes per ViT-importance call from the committed ncu summary (written by
     --write-dram-summary), or None when the kernel source has changed since those counters were
-    taken."""
+    taken; with_algorithmic: (traffic, the summary's algorithmic bytes per call) or (None, None)."""
     try:
         text = open(DRAM_SUMMARY).read()
         t = re.search(r"^traffic_bytes_per_launch:\s*(\d+)", text, re.M)
+        a = re.search(r"^algorithmic_bytes_per_launch:\s*(\d+)", text, re.M)
         h = re.search(r"^source_sha256_16:\s*([0-9a-f]{16})", text, re.M)
         if t and h and h.group(1) == source_hash():
-            return int(t.group(1))
+            return (int(t.group(1)), int(a.group(1)) if a else None) if with_algorithmic else int(t.group(1))
     except OSError:
         pass
-    return None
+    return (None, None) if with_algorithmic else None
 
 
 def write_dram_summary(csv_path):
@@ -276,9 +277,10 @@ class OracleTimer:
             return {"resample": dt}, dt
         if part == "vit":
             n, heads = wl.vit_q.shape[0], wl.vit_q.shape[1]
-            R = min(self.vit_rows, n)
-            jobs = [(np.ascontiguousarray(wl.vit_q[:R, h]), np.ascontiguousarray(wl.vit_k[:, h]), 1 / math.sqrt(80))
-                    for h in range(heads)]
+            R = min(self.vit_rows, n) if self.vit_rows > 0 else n
+            # one pool job per (head, block of at most 2048 query rows): a job holds 2048 x N fp64 scores
+            jobs = [(np.ascontiguousarray(wl.vit_q[r0:min(r0 + 2048, R), h]), np.ascontiguousarray(wl.vit_k[:, h]),
+                     1 / math.sqrt(80)) for h in range(heads) for r0 in range(0, R, 2048)]
             t0 = time.perf_counter()
             self.pool.starmap(_vit_rows_job, jobs, chunksize=1)
             dt = time.perf_counter() - t0
@@ -300,12 +302,15 @@ class OracleTimer:
 
     def description(self):
         n, heads = self.wl.vit_q.shape[0], self.wl.vit_q.shape[1]
-        R = min(self.vit_rows, n)
+        R = min(self.vit_rows, n) if self.vit_rows > 0 else n
         dens = (f"density on a 1/{self.crop_div}-side centre crop scaled by (N/N_crop)^2" if self.crop_div > 1
                 else "density of the whole image")
         return (f"fp64 numpy oracle on {self.pool._processes} host processes: {dens}; resample of the whole "
-                f"image; S_vis for all {heads} heads x the first {R} of {n} query rows (one pool job per head), "
-                f"scaled by {n}/{R}; S_llm, fusion, top-K, gather of the whole image")
+                f"image; " + (f"S_vis for all {heads} heads and all {n} query rows (pool jobs of 2048 rows of one "
+                              f"head)" if R == n else
+                              f"S_vis for all {heads} heads x the first {R} of {n} query rows (pool jobs of 2048 "
+                              f"rows of one head), scaled by {n}/{R}") +
+                "; S_llm, fusion, top-K, gather of the whole image")
 
 
 def oracle_timing(wl, keep, pool, vit_rows, density_crop_div=1):
@@ -874,20 +879,22 @@ def run_gpu(args):
         if world == 1 and not args.no_cpu_baseline:
             pool, cores = oracle_pool()
             try:
-                vit_rows = wl.vit_q.shape[0] if args.cpu_full else args.cpu_vit_rows
+                vit_rows = args.cpu_vit_rows
                 tot, meas, parts, sample = oracle_timing(wl, KEEP, pool, vit_rows, density_crop_div=1)
             finally:
                 pool.close()
                 pool.join()
             cpu = {"value": tot * 1e6, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample,
                    "measured_seconds": round(meas, 3), "parts_s_per_image": {k: round(v, 4) for k, v in parts.items()}}
+        vit_traffic, vit_algo = profiled_traffic(with_algorithmic=True)
         line = {
             "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": workload_config(wl, KEEP),
             "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
-                         "frac": round(achieved / peak, 4), "traffic": profiled_traffic(),
+                         "frac": round(achieved / peak, 4), "traffic": vit_traffic,
+                         "traffic_over_algorithmic": round(vit_traffic / vit_algo, 4) if vit_traffic and vit_algo else None,
                          "traffic_unit": "bytes per call (ncu dram read+write, profiles/vit_importance_img4k_dram.txt)",
                          "kernel": "ViT received attention (attn_row_lse + attn_colsum + attn_reduce), one launch "
                                    "of pace_vit_attn_importance",
@@ -961,10 +968,9 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--ref-vit-rows", type=int, default=512,
                     help="query rows per head of the reference arm's per-step oracle sample")
-    ap.add_argument("--cpu-vit-rows", type=int, default=2048,
-                    help="query rows per head of the cpu_baseline oracle sample")
-    ap.add_argument("--cpu-full", action="store_true",
-                    help="cpu_baseline: run the oracle on the whole image (all query rows; minutes)")
+    ap.add_argument("--cpu-vit-rows", type=int, default=0,
+                    help="cpu_baseline: query rows per head of the ViT oracle (0, the default: all of them, "
+                         "the whole image, about 30 s on 16 cores; a positive value takes a sample, scaled)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-next-rows", action="store_true", help="skip the timing of the NEXT-row calls")
     ap.add_argument("--no-configs", action="store_true",
