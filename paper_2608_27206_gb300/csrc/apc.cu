@@ -579,6 +579,7 @@ __global__ void __launch_bounds__(kApcThreads) apc_tok_pass2(const uint32_t* __r
 struct TailParams {
   float alpha, gamma, r_min, r_max;
   int align;
+  int stage;   // distances the launch's dynamic shared memory holds (0: none; set by launch_tail)
 };
 
 constexpr int kTailSmemMax = 48 * 1024;   // d values staged in shared memory (floats)
@@ -661,7 +662,7 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
   // unit vectors; the top bucket also takes anything above).  Value-domain buckets spread the
   // shared-memory atomics, which the float's top bits (a few exponents) would not.  The
   // distances are staged in shared memory on the way, when they fit.
-  if (N <= kTailSmemMax) {
+  if (N <= prm.stage) {
     // 16-byte copies for the 16-byte-aligned interior of db, 4-byte ones for the ends; the staged
     // copy starts at db's offset within 16 bytes, so each interior copy is aligned at both ends
     const int mis = static_cast<int>((reinterpret_cast<uintptr_t>(db) >> 2) & 3u);
@@ -1435,11 +1436,16 @@ unsigned strip_grid(int units) {
   return static_cast<unsigned>(std::max(1, std::min(units, c)));
 }
 
-size_t tail_smem(const ApcTable& t) {
+// Launches apc_tail on one ApcTable: when every image's distances fit kTailSmemMax, the launch
+// stages them in dynamic shared memory sized for the largest (+ 16 bytes: the staged copy keeps
+// the distances' offset within 16 bytes); otherwise no image is staged (tp.stage = 0), so an image
+// that would fit cannot write past a buffer sized for another launch.
+void launch_tail(const ApcTable& t, const float* d, TailParams tp, pace_apc_stats* stats, cudaStream_t stream) {
   int n = 0;
   for (int i = 0; i < t.nb; ++i) n = std::max(n, t.n[i]);
-  // + 16 bytes: the staged copy keeps the distances' offset within 16 bytes
-  return n <= kTailSmemMax ? static_cast<size_t>(n) * sizeof(float) + 16 : 0;
+  tp.stage = n <= kTailSmemMax ? n : 0;
+  const size_t smem = tp.stage > 0 ? static_cast<size_t>(n) * sizeof(float) + 16 : 0;
+  apc_tail<<<t.nb, 1024, smem, stream>>>(t, d, tp, stats);
 }
 
 pace_status_t tail_smem_attr() {
@@ -1532,8 +1538,8 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
     if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats);
     else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats);
     PACE_CHECK(check_launch());
-    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
-    apc_tail<<<nb, 1024, tail_smem(t), stream>>>(t, d, tp, stats);
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
+    launch_tail(t, d, tp, stats, stream);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;
@@ -1701,8 +1707,8 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
   if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats);
   else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats);
   PACE_CHECK(check_launch());
-  TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
-  apc_tail<<<B, 1024, tail_smem(t), stream>>>(t, d_out, tp, stats);
+  TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
+  launch_tail(t, d_out, tp, stats, stream);
   return check_launch();
 }
 
@@ -1816,8 +1822,8 @@ extern "C" pace_status_t pace_apc_density_tokens(const void* T, const int32_t* c
     PACE_CHECK(check_launch());
     apc_tok_pass2<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums, d_out, stats);
     PACE_CHECK(check_launch());
-    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
-    apc_tail<<<nb, 1024, tail_smem(at), stream>>>(at, d_out, tp, stats);
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
+    launch_tail(at, d_out, tp, stats, stream);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;
@@ -1944,8 +1950,8 @@ extern "C" pace_status_t pace_apc_density_pixel(const uint8_t* img, const int64_
     PACE_CHECK(check_launch());
     apc_pix_pass2<<<units, kApcThreads, 0, stream>>>(pt, tokens, sums, d_out, stats);
     PACE_CHECK(check_launch());
-    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
-    apc_tail<<<nb, 1024, tail_smem(at), stream>>>(at, d_out, tp, stats);
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
+    launch_tail(at, d_out, tp, stats, stream);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;

@@ -233,6 +233,24 @@ def test_density_crowded_tail(pace, side, noisy):
     _no_device_error(pace)
 
 
+def test_density_large_and_small_images_in_one_call(pace):
+    """One image of 224 x 224 patches (50176: more distances than the tail stages in shared
+    memory) next to a small one in the same call: every image must come out bit-equal to a call
+    with that image alone, and the small one equal to the oracle."""
+    rng = np.random.default_rng(31)
+    big = synth.make_image(rng, 3136, 3136, 8, 8, 0.3)
+    small = synth.make_image(rng, 448, 616, 4, 4, 0.5)
+    d, st = _density(pace, [small, big])
+    d_small, st_small = _density(pace, [small])
+    d_big, st_big = _density(pace, [big])
+    n_small = (448 // 14) * (616 // 14)
+    np.testing.assert_array_equal(d[:n_small], d_small)
+    np.testing.assert_array_equal(d[n_small:], d_big)
+    assert st[0] == st_small[0] and st[1] == st_big[0]
+    _check_density(d[:n_small], st[:1], [small])
+    _no_device_error(pace)
+
+
 def test_density_rejects_bad_sizes(pace):
     img = np.zeros((30, 28, 3), dtype=np.uint8)
     with pytest.raises(pace.PaceError) as e:
