@@ -66,7 +66,7 @@ DRAM_SUMMARY = os.path.join(ROOT, "profiles", "vit_importance_img4k_dram.txt")
 DATASHEET_BF16_TFLOPS = 2250.0
 ATTN_SRC = os.path.join(ROOT, "paper_2608_27206_gb300", "csrc", "attn.cu")
 DRAM_CMD = ("ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum --clock-control none "
-            "-k regex:attn_ -c 3 --csv --log-file gpurun_out/vit_dram.csv python bench.py --profile vit --reps 1")
+            "-k regex:attn_ -c 3 --csv --log-file vit_dram.csv python bench.py --profile vit --reps 1")
 
 
 def source_hash():
@@ -102,7 +102,7 @@ def write_dram_summary(csv_path):
     total = 0
     out = ["# DRAM traffic of one pace_vit_attn_importance call: the 4K workload (42196 patches, 16 heads,",
            "# head dim 80, merge 4), one launch of each kernel, cold L2 (ncu flushes caches between kernels).",
-           "# Written by: python bench.py --write-dram-summary gpurun_out/vit_dram.csv",
+           "# Written by: python bench.py --write-dram-summary vit_dram.csv",
            "# Capture (the same bench.py --profile command first ran without ncu and exited 0):",
            "#   " + DRAM_CMD,
            "# kernel | dram read bytes | dram write bytes | time ns"]
