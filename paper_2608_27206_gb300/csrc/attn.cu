@@ -667,8 +667,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
   auto b_qempty = [&](int s) { return smem_u32(&ctl->bars[2 + ST + s]); };
   auto b_sfull = [&](int p) { return smem_u32(&ctl->bars[2 + 2 * ST + p]); };
   auto b_sfree = [&](int p) { return smem_u32(&ctl->bars[4 + 2 * ST + p]); };
-  // stage s is ready for the MMA beyond its copy: every stage use gets one arrival, right after the
-  // copy is issued, or once the rows past the image have been zeroed on an image's ragged last tile
+  // stage s holds an image's ragged last query tile with the rows past the image zeroed: one
+  // arrival per ragged use of the stage (the other tiles need only their copy)
   auto b_fixed = [&](int s) { return smem_u32(&ctl->bars[6 + 2 * ST + s]); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -689,6 +689,14 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
   // query rows of stream tile j that lie inside the image (kStream unless it is the image's last
   // tile and the image ends inside it)
   auto ragged_rows = [&](int j) { return min(kStream, t.nq[b] - (qt_min + j % nspan) * kStream); };
+  // the ragged tiles are j = nspan - 1, 2 nspan - 1, .. (when the image ends inside its last query
+  // tile); the phase of b_fixed(j % ST) that ragged tile j completes = how many earlier ragged tiles
+  // used the same stage
+  auto ragged_phase = [&](int j) {
+    int k = 0;
+    for (int j2 = nspan - 1; j2 < j; j2 += nspan) k += (j2 % ST) == (j % ST);
+    return k & 1;
+  };
 
   if (threadIdx.x == 0) {
     mbar_init(b_afull, 1);
@@ -773,8 +781,6 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
           __syncwarp();
           if (lane == 0) mbar_arrive(b_fixed(s));
         }
-      } else if (lane == 0 && ok) {
-        mbar_arrive(b_fixed(s));
       }
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;
     }
@@ -795,7 +801,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
           set_abort(ctl, status, K_ATTN_COLSUM);
           break;
         }
-        if (!mbar_wait(b_fixed(s), u & 1, kWaitLimitNs)) {
+        if (ragged_rows(j) < kStream && !mbar_wait(b_fixed(s), ragged_phase(j), kWaitLimitNs)) {
           set_abort(ctl, status, K_ATTN_COLSUM);
           break;
         }
