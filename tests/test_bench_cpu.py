@@ -115,3 +115,31 @@ def test_reference_arm_times_one_part_per_step(monkeypatch, capsys):
     line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
     assert calls == list(FakeTimer.PARTS)          # one timed step, four extra to cover every part
     assert set(line["cpu_baseline"]["parts_s_per_image"]) == set(FakeTimer.PARTS)
+
+
+def test_oracle_timer_parts_on_a_small_workload():
+    """The per-part oracle timer behind cpu_baseline and the reference arm, on the 448^2
+    workload with a two-process spawn pool: every part reports a time, and a row sample of the
+    ViT map is scaled by N / rows (all rows: no scaling)."""
+    from paper_2608_27206_gb300 import synth
+    wl = synth.make_workload("img448", seed=0)
+    pool, _ = bench.oracle_pool(2)
+    try:
+        full = bench.OracleTimer(wl, 0.1, pool, vit_rows=0)
+        seen = {}
+        for part in bench.OracleTimer.PARTS:
+            t, dt = full.time(part)
+            assert dt >= 0.0 and all(v >= 0.0 for v in t.values())
+            seen.update(t)
+        assert set(seen) == {"density", "resample", "vit", "llm", "select", "gather"}
+        n = wl.vit_q.shape[0]
+        t, dt = full.time("vit")
+        assert t["vit"] == pytest.approx(dt)                     # every row: measured, not scaled
+        part = bench.OracleTimer(wl, 0.1, pool, vit_rows=n // 4)
+        t, dt = part.time("vit")
+        assert t["vit"] == pytest.approx(dt * 4)                 # a quarter of the rows, scaled by 4
+        assert "first %d of %d query rows" % (n // 4, n) in part.description()
+        assert "all %d query rows" % n in full.description()
+    finally:
+        pool.close()
+        pool.join()
