@@ -10,10 +10,14 @@
 //              reduction is exact and independent of the CTA order.
 //   apc_pass2  same strips: c = sums / N, phi = |c|^2, c_hat = c / |c| (recomputed per
 //              CTA from the 589 integers), then d_i = |t_i - c_hat| computed directly from
-//              the staged pixels (no 2 - 2cos cancellation).
-//   apc_tail   one CTA per image: select of the k_tail-th largest d_i (value buckets, then the
-//              selected bucket's members ranked directly or by offset rounds over their fp32
-//              bits), tail mean, rho_d, rho, r and the target size.
+//              the staged pixels (no 2 - 2cos cancellation), counted into the tail's value
+//              buckets (global atomics).
+//   apc_tail_scan  one CTA per 4096 distances of an image: the k_tail-th largest's bucket from
+//              the counts, the distances above it summed (2^-32 fixed point) and the bucket's
+//              members listed; the image's last CTA ranks the members (directly, or by offset
+//              rounds over their fp32 bits) and computes the tail mean, rho_d, rho, r and the
+//              target size.  The token and pixel-statistic densities use apc_tail, the same
+//              select in one CTA per image.
 // Resize: apc_resample, four CTAs per SM walking the 16 x 32 output tiles of the batch; for
 // downscales up to 2.75x per side the input window is staged in shared memory and filtered
 // there with precomputed weights, steeper downscales take a generic path with per-tap weights.
@@ -295,13 +299,47 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restri
   static_assert(kSlots <= 2 * kApcThreads, "column slots");
 }
 
+struct TailParams {
+  float alpha, gamma, r_min, r_max;
+  int align;
+  int stage;   // distances the launch's dynamic shared memory holds (0: none; set by launch_tail)
+};
+
+constexpr int kTailSmemMax = 48 * 1024;   // d values staged in shared memory (floats)
+constexpr int kTailBins = 4096;            // level-1 buckets of the tail select
+constexpr int kTailBins2 = 1024;           // level-2 offset bins over a compacted bucket
+
+// Bucket of a distance d >= 0: floor(2048 d), capped at the top bucket (monotone in d; NaN goes to
+// bucket 0).  Full-rate arithmetic only (no float-to-integer conversion): once clamped to
+// [0, 4095], 2048 d + 2^23 rounded toward zero holds floor(2048 d) in its low mantissa bits.
+__device__ __forceinline__ int tail_bucket(float v) {
+  const float x = fminf(fmaxf(v * 2048.0f, 0.0f), static_cast<float>(kTailBins - 1));
+  return __float_as_int(__fadd_rz(x, 8388608.0f)) - 0x4B000000;
+}
+
+// Scratch of the density tail over several CTAs per image (apc_tail_scan): the counts of the
+// distances per bucket (pass 2 adds them), then the sum and count of the distances above the
+// k-th largest's bucket, the members of that bucket, and how many of the image's CTAs are done.
+constexpr int kTailChunk = 4096;   // distances per CTA of apc_tail_scan
+constexpr int kTailList = 4096;    // members of the selected bucket kept for the last CTA's rank
+struct TailWork {
+  unsigned long long above_fix;    // distances above the bucket, 2^-32 fixed point
+  unsigned above_cnt;
+  unsigned list_n;
+  unsigned done;
+  unsigned pad;
+  unsigned hist[kTailBins];
+  unsigned list[kTailList];
+};
+
 template <bool WIDE>
-__global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restrict__ img,
+__global__ void __launch_bounds__(kApcThreads, 4) apc_pass2(const uint8_t* __restrict__ img,
                                                          const __grid_constant__ ApcTable t, int units,
                                                          const float* __restrict__ inv_norm,
                                                          const unsigned long long* __restrict__ sums,
                                                          float* __restrict__ d_out,
-                                                         pace_apc_stats* __restrict__ stats) {
+                                                         pace_apc_stats* __restrict__ stats,
+                                                         TailWork* __restrict__ work) {
   __shared__ __align__(16) uint8_t s2[2][kPatch * kStripRowBytes];
   __shared__ __align__(8) float chat[kTokDim + 3];
   __shared__ float red[kApcThreads / 32];
@@ -314,6 +352,7 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
   int cur_b = -1;
   bool reload = false;
   float2 chr[kPairIters];   // c_hat of this lane's coordinate pairs, in registers
+  unsigned* hist = nullptr; // the current image's tail bucket counts
   issue_strip<WIDE>(img, t, unit, s2[0]);
   for (int i = 0; unit < units; ++i, unit += gridDim.x) {
     const int next = unit + static_cast<int>(gridDim.x);
@@ -321,6 +360,7 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
     if (q.b != cur_b) {   // c = sums / N, |c|^2 (fixed summation order), c_hat = c / |c|
       cur_b = q.b;
       reload = true;
+      hist = work[t.b_base + q.b].hist;
       const int N = (t.H[q.b] / kPatch) * t.gw[q.b];
       const float inv_n = 1.0f / static_cast<float>(N);
       const unsigned long long* sb = sums + static_cast<int64_t>(t.b_base + q.b) * kTokDim;
@@ -379,7 +419,9 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass2(const uint8_t* __restri
       float acc = warp_sum_f(acc2.x + acc2.y);
       if (lane == 0) {
         const float v = iv - chat[kPatchBytes];
-        d_out[t.patch0[q.b] + q.py * t.gw[q.b] + q.px0 + p] = sqrtf(fmaf(v, v, acc));
+        const float dv = sqrtf(fmaf(v, v, acc));
+        d_out[t.patch0[q.b] + q.py * t.gw[q.b] + q.px0 + p] = dv;
+        atomicAdd(hist + tail_bucket(dv), 1u);   // the tail's bucket counts
       }
     }
     __syncthreads();   // this buffer is refilled two strips on; chat may be rewritten
@@ -576,24 +618,6 @@ __global__ void __launch_bounds__(kApcThreads) apc_tok_pass2(const uint32_t* __r
   }
 }
 
-struct TailParams {
-  float alpha, gamma, r_min, r_max;
-  int align;
-  int stage;   // distances the launch's dynamic shared memory holds (0: none; set by launch_tail)
-};
-
-constexpr int kTailSmemMax = 48 * 1024;   // d values staged in shared memory (floats)
-constexpr int kTailBins = 4096;            // level-1 buckets of the tail select
-constexpr int kTailBins2 = 1024;           // level-2 offset bins over a compacted bucket
-
-// Bucket of a distance d >= 0: floor(2048 d), capped at the top bucket (monotone in d; NaN goes to
-// bucket 0).  Full-rate arithmetic only (no float-to-integer conversion): once clamped to
-// [0, 4095], 2048 d + 2^23 rounded toward zero holds floor(2048 d) in its low mantissa bits.
-__device__ __forceinline__ int tail_bucket(float v) {
-  const float x = fminf(fmaxf(v * 2048.0f, 0.0f), static_cast<float>(kTailBins - 1));
-  return __float_as_int(__fadd_rz(x, 8388608.0f)) - 0x4B000000;
-}
-
 // Called by all 1024 threads: the bin holding the r-th largest entry, counting from bin NBINS - 1
 // down (1 <= r <= total): sel[0] = that bin, sel[1] = entries in the bins above it.  wsum: 32 words.
 template <int NBINS>
@@ -641,6 +665,28 @@ __device__ __forceinline__ void select_from_top(const unsigned* bins, unsigned r
     sel[1] = above;
   }
   __syncthreads();
+}
+
+// Eq. 5-6 and R3-R4 from the tail mean d_top of image b: rho_d, rho, r and the target size.
+__device__ __forceinline__ void tail_finish(const ApcTable& t, int b, const TailParams& prm,
+                                            pace_apc_stats* __restrict__ stats, float rho_g, float d_top) {
+  const float rho_d = fminf(d_top / prm.gamma, 1.0f);
+  const float rho = prm.alpha * rho_g + (1.0f - prm.alpha) * rho_d;
+  const float r = fminf(fmaxf(rho, prm.r_min), prm.r_max);
+  const float sr = sqrtf(fmaxf(r, 0.0f));
+  const int al = prm.align;
+  const int H = t.H[b], W = t.W[b];
+  int ho = al * static_cast<int>(floorf(static_cast<float>(H) * sr / al + 0.5f));
+  int wo = al * static_cast<int>(floorf(static_cast<float>(W) * sr / al + 0.5f));
+  ho = min(H, max(al, ho));
+  wo = min(W, max(al, wo));
+  pace_apc_stats& st = stats[t.b_base + b];
+  st.d_top = d_top;
+  st.rho_d = rho_d;
+  st.rho = rho;
+  st.r = r;
+  st.h_out = ho;
+  st.w_out = wo;
 }
 
 __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTable t, const float* __restrict__ d,
@@ -818,27 +864,216 @@ __global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTabl
     }
     tot += unfix32<false>(f, 1.0f);
     tot += static_cast<float>(k - c) * T;  // the remaining entries all equal T
-    const float d_top = tot / static_cast<float>(k);
-    const float rho_g = stats[t.b_base + b].rho_g;
-    const float rho_d = fminf(d_top / prm.gamma, 1.0f);
-    const float rho = prm.alpha * rho_g + (1.0f - prm.alpha) * rho_d;
-    const float r = fminf(fmaxf(rho, prm.r_min), prm.r_max);
-    const float sr = sqrtf(fmaxf(r, 0.0f));
-    const int al = prm.align;
-    const int H = t.H[b], W = t.W[b];
-    int ho = al * static_cast<int>(floorf(static_cast<float>(H) * sr / al + 0.5f));
-    int wo = al * static_cast<int>(floorf(static_cast<float>(W) * sr / al + 0.5f));
-    ho = min(H, max(al, ho));
-    wo = min(W, max(al, wo));
-    pace_apc_stats& st = stats[t.b_base + b];
-    st.d_top = d_top;
-    st.rho_d = rho_d;
-    st.rho = rho;
-    st.r = r;
-    st.h_out = ho;
-    st.w_out = wo;
+    tail_finish(t, b, prm, stats, stats[t.b_base + b].rho_g, tot / static_cast<float>(k));
   }
 }
+
+// The density tail over several CTAs per image (the pixel density call; pass 2 has counted the
+// distances per bucket).  CTA c of image b takes distances c kTailChunk .. : it selects the k-th
+// largest's bucket from the counts (level 1 of apc_tail), adds the distances above that bucket
+// to the image's total in 2^-32 fixed point (exact, so the order of the CTAs does not matter)
+// and lists the bucket's members.  The image's last CTA to finish narrows the members to the
+// k-th largest distance T (apc_tail's level 2: a direct rank, or offset rounds) and writes the
+// statistics; a bucket too crowded for the list is narrowed over the whole array instead.
+__global__ void __launch_bounds__(1024) apc_tail_scan(const __grid_constant__ ApcTable t, const float* __restrict__ d,
+                                                      TailParams prm, pace_apc_stats* __restrict__ stats,
+                                                      TailWork* __restrict__ work) {
+  __shared__ unsigned bins[kTailBins];
+  __shared__ unsigned hist2[kTailBins2];
+  __shared__ unsigned sel[2];
+  __shared__ unsigned cred[32];
+  __shared__ unsigned long long fred[32];
+  __shared__ int last;
+  const int b = blockIdx.y;
+  const int N = t.n[b];
+  const int nchunk = (N + kTailChunk - 1) / kTailChunk;
+  if (static_cast<int>(blockIdx.x) >= nchunk) return;
+  TailWork* w = work + (t.b_base + b);
+  const float* db = d + t.patch0[b];
+  const unsigned k = static_cast<unsigned>(t.ktail[b]);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // level 1 on the counts (written by the previous kernel: read through L2)
+  for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = __ldcg(&w->hist[i]);
+  __syncthreads();
+  select_from_top<kTailBins>(bins, k, sel, cred);
+  const int tb = static_cast<int>(sel[0]);
+  const unsigned cb = bins[tb];         // entries in the k-th largest's bucket
+  const unsigned above_n = sel[1];      // entries in the buckets above it
+  const bool listed = cb <= kTailList;
+  // this CTA's chunk
+  unsigned long long s_fix = 0ull;
+  unsigned cnt = 0u;
+  bool wrote = false;   // this thread listed a member
+  const int i0 = static_cast<int>(blockIdx.x) * kTailChunk, i1 = min(N, i0 + kTailChunk);
+  for (int base = i0; base < i1; base += blockDim.x) {   // uniform trip count: the ballot below
+    const int i = base + static_cast<int>(threadIdx.x);
+    const float v = i < i1 ? db[i] : 0.f;
+    const int bk = i < i1 ? tail_bucket(v) : -1;
+    if (bk > tb) {
+      s_fix += fix32(v);
+      ++cnt;
+    }
+    const bool member = listed && bk == tb;
+    const unsigned ball = __ballot_sync(0xffffffffu, member);
+    if (ball != 0u) {   // one slot reservation per warp
+      unsigned slot = 0u;
+      if (lane == 0) slot = atomicAdd(&w->list_n, static_cast<unsigned>(__popc(ball)));
+      slot = __shfl_sync(0xffffffffu, slot, 0);
+      if (member) {
+        w->list[slot + __popc(ball & ((1u << lane) - 1u))] = __float_as_uint(v);
+        wrote = true;
+      }
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+    s_fix += __shfl_xor_sync(0xffffffffu, s_fix, o);
+  }
+  if (lane == 0) {
+    cred[warp] = cnt;
+    fred[warp] = s_fix;
+  }
+  if (wrote) __threadfence();   // this thread's list entries, before the CTA reports its chunk done
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned c = 0u;
+    unsigned long long f = 0ull;
+    for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) {
+      c += cred[i];
+      f += fred[i];
+    }
+    atomicAdd(&w->above_fix, f);
+    atomicAdd(&w->above_cnt, c);
+    __threadfence();
+    last = atomicAdd(&w->done, 1u) == static_cast<unsigned>(nchunk - 1);
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  // the image's totals and rho_g, read now so that their latency overlaps level 2
+  unsigned tot_cnt = 0u;
+  unsigned long long tot_fix = 0ull;
+  float rho_g = 0.f;
+  if (threadIdx.x == 0) {
+    tot_cnt = __ldcg(&w->above_cnt);
+    tot_fix = __ldcg(&w->above_fix);
+    rho_g = stats[t.b_base + b].rho_g;
+  }
+  // level 2 (the image's last CTA): T = the k-th largest distance; the members of the bucket
+  // above T are summed in fixed point (c counts every distance above T)
+  unsigned remaining = k - above_n;
+  unsigned lo = __float_as_uint(static_cast<float>(tb) * (1.0f / 2048.0f));
+  unsigned span = (tb == kTailBins - 1 ? 0x7F800001u : __float_as_uint(static_cast<float>(tb + 1) * (1.0f / 2048.0f))) - lo;
+  const unsigned bucket_lo = lo, bucket_span = span;
+  s_fix = 0ull;
+  cnt = 0u;
+  unsigned prefix;
+  __syncthreads();   // everyone has read sel and bins[tb]
+  if (listed) {
+    for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) bins[i] = __ldcg(&w->list[i]);
+    __syncthreads();
+    if (cb <= blockDim.x) {
+      // one member per thread, ranked against the whole list (as apc_tail)
+      int mi;
+      unsigned gt, ge;
+      if (rank_in_list(bins, cb, mi, gt, ge)) {
+        const unsigned mine = bins[mi];
+        if (ge < remaining) {
+          s_fix += fix32(__uint_as_float(mine));
+          ++cnt;
+        } else if (gt < remaining) {
+          sel[0] = mine;   // the same key from every member equal to it
+        }
+      }
+      __syncthreads();
+      prefix = sel[0];
+    } else {
+      while (true) {
+        const int bits = 32 - __clz(span - 1u);
+        const int shift = bits > 10 ? bits - 10 : 0;
+        for (int i = threadIdx.x; i < kTailBins2; i += blockDim.x) hist2[i] = 0u;
+        __syncthreads();
+        for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
+          const unsigned off = bins[i] - lo;   // wraps for keys below lo
+          if (off < span) atomicAdd(&hist2[off >> shift], 1u);
+        }
+        __syncthreads();
+        select_from_top<kTailBins2>(hist2, remaining, sel, cred);
+        lo += sel[0] << shift;
+        remaining -= sel[1];
+        if (shift == 0) break;
+        span = min(span - (sel[0] << shift), 1u << shift);
+      }
+      prefix = lo;
+      for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
+        const unsigned key = bins[i];
+        if (key > prefix) {
+          s_fix += fix32(__uint_as_float(key));
+          ++cnt;
+        }
+      }
+    }
+  } else {
+    // a crowded bucket: its members by key offset from its first key over the whole array,
+    // 4096 offsets (2^shift keys each) at a time, until one key is left (as apc_tail)
+    while (true) {
+      const int bits = 32 - __clz(span - 1u);
+      const int shift = bits > 12 ? bits - 12 : 0;
+      __syncthreads();                               // everyone has read sel and the bins
+      for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
+      __syncthreads();
+      for (int base = 0; base < N; base += blockDim.x) {   // uniform trip count: __match_any_sync below
+        const int i = base + static_cast<int>(threadIdx.x);
+        const unsigned off = i < N ? __float_as_uint(db[i]) - lo : span;   // wraps for keys below lo
+        const bool in = off < span;
+        const unsigned digit = in ? off >> shift : kTailBins;
+        const unsigned members = __ballot_sync(0xffffffffu, in);
+        if (__popc(members) > 4) {
+          const unsigned peers = __match_any_sync(0xffffffffu, digit);
+          if (in && lane == __ffs(peers) - 1) atomicAdd(&bins[digit], static_cast<unsigned>(__popc(peers)));
+        } else if (in) {
+          atomicAdd(&bins[digit], 1u);
+        }
+      }
+      __syncthreads();
+      select_from_top<kTailBins>(bins, remaining, sel, cred);
+      lo += sel[0] << shift;
+      remaining -= sel[1];
+      if (shift == 0) break;
+      span = min(span - (sel[0] << shift), 1u << shift);
+    }
+    prefix = lo;
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {   // the bucket's members above T
+      const unsigned key = __float_as_uint(db[i]);
+      if (key > prefix && key - bucket_lo < bucket_span) {
+        s_fix += fix32(__uint_as_float(key));
+        ++cnt;
+      }
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+    s_fix += __shfl_xor_sync(0xffffffffu, s_fix, o);
+  }
+  __syncthreads();   // the level-2 reads of cred and sel are done
+  if (lane == 0) {
+    cred[warp] = cnt;
+    fred[warp] = s_fix;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned c = tot_cnt;
+    unsigned long long f = tot_fix;
+    for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) {
+      c += cred[i];
+      f += fred[i];
+    }
+    const float T = __uint_as_float(prefix);   // k-th largest d
+    const float tot = unfix32<false>(f, 1.0f) + static_cast<float>(k - c) * T;   // the rest equal T
+    tail_finish(t, b, prm, stats, rho_g, tot / static_cast<float>(k));
+  }
+}
+
 
 // ------------------------------------------------------------------------------------------------
 // pixel-statistic previews (App. "Shallow Feature Preview Ablation"): one small token per patch,
@@ -1403,7 +1638,7 @@ __global__ void __launch_bounds__(kRsThreads) apc_resample(const uint8_t* __rest
 // host side
 // ------------------------------------------------------------------------------------------------
 struct DensityLayout {
-  size_t sums_off, inv_off, d_off, total;
+  size_t sums_off, work_off, zero_bytes, inv_off, d_off, total;   // [0, zero_bytes) is zeroed per call
   int64_t n_total;
 };
 
@@ -1413,7 +1648,9 @@ DensityLayout density_layout(int B, const int32_t* H, const int32_t* W) {
   for (int b = 0; b < B; ++b) n += static_cast<int64_t>(H[b] / kPatch) * (W[b] / kPatch);
   L.n_total = n;
   L.sums_off = 0;
-  L.inv_off = align_up(static_cast<size_t>(B) * kTokDim * sizeof(unsigned long long), 256);
+  L.work_off = align_up(static_cast<size_t>(B) * kTokDim * sizeof(unsigned long long), 256);
+  L.zero_bytes = L.work_off + static_cast<size_t>(B) * sizeof(TailWork);
+  L.inv_off = align_up(L.zero_bytes, 256);
   L.d_off = L.inv_off + align_up(static_cast<size_t>(n) * sizeof(float), 256);
   L.total = L.d_off + align_up(static_cast<size_t>(n) * sizeof(float), 256);
   return L;
@@ -1446,6 +1683,16 @@ void launch_tail(const ApcTable& t, const float* d, TailParams tp, pace_apc_stat
   tp.stage = n <= kTailSmemMax ? n : 0;
   const size_t smem = tp.stage > 0 ? static_cast<size_t>(n) * sizeof(float) + 16 : 0;
   apc_tail<<<t.nb, 1024, smem, stream>>>(t, d, tp, stats);
+}
+
+// Launches apc_tail_scan on one ApcTable: kTailChunk distances per CTA, the largest image's
+// chunks per row of the grid (CTAs past a smaller image's chunks return at once).
+void launch_tail_scan(const ApcTable& t, const float* d, TailParams tp, pace_apc_stats* stats, TailWork* work,
+                      cudaStream_t stream) {
+  int chunks = 1;
+  for (int i = 0; i < t.nb; ++i) chunks = std::max(chunks, (t.n[i] + kTailChunk - 1) / kTailChunk);
+  apc_tail_scan<<<dim3(static_cast<unsigned>(chunks), static_cast<unsigned>(t.nb)), 1024, 0, stream>>>(t, d, tp, stats,
+                                                                                                     work);
 }
 
 pace_status_t tail_smem_attr() {
@@ -1502,9 +1749,10 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
   PACE_CHECK(tail_smem_attr());
   uint8_t* w8 = static_cast<uint8_t*>(ws);
   auto* sums = reinterpret_cast<unsigned long long*>(w8 + L.sums_off);
+  auto* work = reinterpret_cast<TailWork*>(w8 + L.work_off);
   auto* inv = reinterpret_cast<float*>(w8 + L.inv_off);
   float* d = d_out ? d_out : reinterpret_cast<float*>(w8 + L.d_off);
-  PACE_CUDA(cudaMemsetAsync(sums, 0, static_cast<size_t>(B) * kTokDim * sizeof(unsigned long long), stream));
+  PACE_CUDA(cudaMemsetAsync(w8, 0, L.zero_bytes, stream));   // column sums and tail scratch
   int patch0 = 0;
   for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
     const int nb = (B - c0) < kApcMaxB ? (B - c0) : kApcMaxB;
@@ -1535,11 +1783,11 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
     if (wide) apc_pass1<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums);
     else apc_pass1<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums);
     PACE_CHECK(check_launch());
-    if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats);
-    else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats);
+    if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats, work);
+    else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats, work);
     PACE_CHECK(check_launch());
     TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
-    launch_tail(t, d, tp, stats, stream);
+    launch_tail_scan(t, d, tp, stats, work, stream);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;
@@ -1624,7 +1872,9 @@ namespace pace {
 namespace {
 constexpr size_t kStaticSumsBytes =
     static_cast<size_t>(PACE_APC_STATIC_MAX_IMAGES) * kTokDim * sizeof(unsigned long long);
-constexpr size_t kStaticInvOff = (kStaticSumsBytes + 255) / 256 * 256;
+constexpr size_t kStaticWorkOff = (kStaticSumsBytes + 255) / 256 * 256;
+constexpr size_t kStaticZeroBytes = kStaticWorkOff + static_cast<size_t>(PACE_APC_STATIC_MAX_IMAGES) * sizeof(TailWork);
+constexpr size_t kStaticInvOff = (kStaticZeroBytes + 255) / 256 * 256;
 constexpr size_t kStaticBytes = kStaticInvOff + static_cast<size_t>(PACE_APC_STATIC_MAX_PATCHES) * sizeof(float);
 
 static __device__ __align__(256) unsigned char g_apc_static_scratch[kStaticBytes];
@@ -1674,9 +1924,12 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
   unsigned char* scratch = nullptr;
   PACE_CHECK(static_scratch(&scratch));
   auto* sums = reinterpret_cast<unsigned long long*>(scratch);
+  auto* work = reinterpret_cast<TailWork*>(scratch + kStaticWorkOff);
   auto* inv = reinterpret_cast<float*>(scratch + kStaticInvOff);
-  // the array keeps the previous call's contents: the column sums must start from zero
+  // the array keeps the previous call's contents: the column sums and the tail scratch of the
+  // call's images must start from zero
   PACE_CUDA(cudaMemsetAsync(sums, 0, static_cast<size_t>(B) * kTokDim * sizeof(unsigned long long), stream));
+  PACE_CUDA(cudaMemsetAsync(work, 0, static_cast<size_t>(B) * sizeof(TailWork), stream));
   ApcTable t{};
   t.nb = B;
   t.b_base = 0;
@@ -1704,11 +1957,11 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
   if (wide) apc_pass1<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums);
   else apc_pass1<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums);
   PACE_CHECK(check_launch());
-  if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats);
-  else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats);
+  if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats, work);
+  else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats, work);
   PACE_CHECK(check_launch());
   TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
-  launch_tail(t, d_out, tp, stats, stream);
+  launch_tail_scan(t, d_out, tp, stats, work, stream);
   return check_launch();
 }
 
