@@ -46,6 +46,7 @@ WORKLOAD = "img4k"
 KEEP = 0.10
 FLUSH_BYTES = 256 << 20
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+LONG_REGION_S = 1.0   # a timed region at least this long is "a long step" for the roofline peak
 
 
 # ----------------------------------------------------------------------------------------------
@@ -861,6 +862,12 @@ def run_gpu(args):
         sm_mhz = (clocks or {}).get("sm_mhz") or float(peaks.get("sm_max_mhz", 0) or 0)
         mufu_peak = 32.0 * torch.cuda.get_device_properties(0).multi_processor_count * sm_mhz * 1e6 if sm_mhz else None
         peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+        peak_sus = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+        # The ViT call is timed inside the step loop: when that loop runs for seconds (the default
+        # 200 steps), the GPU sits at its power-capped operating point like the sustained GEMM of
+        # MEASURED_PEAKS.json, so that figure is the denominator; shorter runs use the burst one.
+        vit_sustained = t_wall >= LONG_REGION_S
+        vit_peak = peak_sus if vit_sustained else peak
         hbm = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
         mean = {k: statistics.mean(v) for k, v in part_ms.items()}
         other = {}
@@ -892,15 +899,16 @@ def run_gpu(args):
             "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": False,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": workload_config(wl, KEEP),
-            "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
-                         "frac": round(achieved / peak, 4), "traffic": vit_traffic,
+            "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": vit_peak, "unit": "TFLOP/s",
+                         "frac": round(achieved / vit_peak, 4), "traffic": vit_traffic,
+                         "peak_burst": peak, "frac_burst": round(achieved / peak, 4),
                          "traffic_over_algorithmic": round(vit_traffic / vit_algo, 4) if vit_traffic and vit_algo else None,
                          "traffic_unit": "bytes per call (ncu dram read+write, profiles/vit_importance_img4k_dram.txt)",
                          "kernel": "ViT received attention (attn_row_lse + attn_colsum + attn_reduce), one launch "
                                    "of pace_vit_attn_importance",
                          "algorithmic_flops": cnt["vit_flops"], "us": round(vit_ms * 1e3, 1),
                          # one pass of QK^T is the "useful" work; the second pass recomputes it
-                         "useful_one_pass_frac": round(achieved / 2 / peak, 4),
+                         "useful_one_pass_frac": round(achieved / 2 / vit_peak, 4),
                          # the same achieved rate against NVIDIA's published dense bf16 figure
                          "datasheet_peak": DATASHEET_BF16_TFLOPS,
                          "frac_of_datasheet": round(achieved / DATASHEET_BF16_TFLOPS, 4),
@@ -910,8 +918,10 @@ def run_gpu(args):
                          "mufu_frac": round(cnt["vit_ex2"] / (vit_ms * 1e-3) / mufu_peak, 4)
                          if mufu_peak else None,
                          "mufu_peak_ex2_per_s": mufu_peak,
-                         "peak_source": f"{peak_src} bf16 dense burst (MEASURED_PEAKS.json)"
-                         if peak_src == "measured" else "fallback 1.9 PFLOP/s bf16"},
+                         "peak_source": (f"{peak_src} bf16 dense "
+                                         + (f"sustained (the ViT call timed inside {t_wall:.2f} s of back-to-back steps)"
+                                            if vit_sustained else "burst (a short timed region)")
+                                         + (" (MEASURED_PEAKS.json)" if peak_src == "measured" else " (recipe fallback)"))},
             "rooflines_other": other,
             "rooflines_batched": batched,
             "configs_other": cfgs,
