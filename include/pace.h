@@ -140,7 +140,7 @@ PACE_API pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img_o
  * running inside a host framework that owns every allocation, or a latency-critical path
  * where cudaMalloc (which may synchronise the device) is not allowed.  It computes exactly
  * what pace_apc_density computes, with the same kernels, but its scratch lives in one
- * file-scope device array owned by the library (about 330 KB on every GPU that loads the
+ * file-scope device array owned by the library (about 860 KB on every GPU that loads the
  * library, held until the process exits).  It allocates and frees nothing.
  *
  *  - At most PACE_APC_STATIC_MAX_IMAGES images and PACE_APC_STATIC_MAX_PATCHES patches
