@@ -16,8 +16,8 @@
 //              the counts, the distances above it summed (2^-32 fixed point) and the bucket's
 //              members listed; the image's last CTA ranks the members (directly, or by offset
 //              rounds over their fp32 bits) and computes the tail mean, rho_d, rho, r and the
-//              target size.  The token and pixel-statistic densities use apc_tail, the same
-//              select in one CTA per image.
+//              target size.  The token and pixel-statistic densities share it (their pass 2
+//              counts the buckets the same way).
 // Resize: apc_resample, four CTAs per SM walking the 16 x 32 output tiles of the batch; for
 // downscales up to 2.75x per side the input window is staged in shared memory and filtered
 // there with precomputed weights, steeper downscales take a generic path with per-tap weights.
@@ -86,12 +86,6 @@ __device__ __forceinline__ int find_image(const ApcTable& t, int unit) {
 // Asynchronous 4-byte global -> shared copies (no register round trip, all in flight at once).
 __device__ __forceinline__ void cp_async4(void* dst, const void* src) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
-               "l"(src)
-               : "memory");
-}
-// 16-byte copy, both addresses 16-byte aligned (cached in L2 only).
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
                "l"(src)
                : "memory");
 }
@@ -302,12 +296,10 @@ __global__ void __launch_bounds__(kApcThreads) apc_pass1(const uint8_t* __restri
 struct TailParams {
   float alpha, gamma, r_min, r_max;
   int align;
-  int stage;   // distances the launch's dynamic shared memory holds (0: none; set by launch_tail)
 };
 
-constexpr int kTailSmemMax = 48 * 1024;   // d values staged in shared memory (floats)
 constexpr int kTailBins = 4096;            // level-1 buckets of the tail select
-constexpr int kTailBins2 = 1024;           // level-2 offset bins over a compacted bucket
+constexpr int kTailBins2 = 1024;           // level-2 offset bins over a listed bucket
 
 // Bucket of a distance d >= 0: floor(2048 d), capped at the top bucket (monotone in d; NaN goes to
 // bucket 0).  Full-rate arithmetic only (no float-to-integer conversion): once clamped to
@@ -568,7 +560,8 @@ __global__ void __launch_bounds__(kApcThreads) apc_tok_pass2(const uint32_t* __r
                                                              const float* __restrict__ inv_norm,
                                                              const unsigned long long* __restrict__ sums,
                                                              float* __restrict__ d_out,
-                                                             pace_apc_stats* __restrict__ stats) {
+                                                             pace_apc_stats* __restrict__ stats,
+                                                             TailWork* __restrict__ work) {
   __shared__ __align__(16) float chat[kTokMaxD];
   __shared__ float red[kApcThreads / 32];
   const int unit = blockIdx.x;
@@ -614,7 +607,11 @@ __global__ void __launch_bounds__(kApcThreads) apc_tok_pass2(const uint32_t* __r
       acc1 = fmaf(e1, e1, acc1);
     }
     const float acc = warp_sum_f(acc0 + acc1);
-    if (lane == 0) d_out[t.tok0[b] + c0 + p] = sqrtf(acc);
+    if (lane == 0) {
+      const float dv = sqrtf(acc);
+      d_out[t.tok0[b] + c0 + p] = dv;
+      atomicAdd(&work[t.b_base + b].hist[tail_bucket(dv)], 1u);   // the tail's bucket counts
+    }
   }
 }
 
@@ -689,192 +686,16 @@ __device__ __forceinline__ void tail_finish(const ApcTable& t, int b, const Tail
   st.w_out = wo;
 }
 
-__global__ void __launch_bounds__(1024) apc_tail(const __grid_constant__ ApcTable t, const float* __restrict__ d,
-                                                 TailParams prm, pace_apc_stats* __restrict__ stats) {
-  extern __shared__ __align__(16) float sd[];
-  __shared__ unsigned bins[kTailBins];
-  __shared__ unsigned hist2[kTailBins2];
-  __shared__ unsigned sel[2];
-  __shared__ float red[32];
-  __shared__ unsigned cred[32];
-  __shared__ unsigned long long fred[32];
-  __shared__ unsigned ncomp;
-  const int b = blockIdx.x;
-  const int N = t.n[b];
-  const float* db = d + t.patch0[b];
-  const unsigned k = static_cast<unsigned>(t.ktail[b]);
-  const int lane_id = threadIdx.x & 31;
-  // Level 1: the k-th largest distance's bucket among 4096 buckets of width 1/2048 (d <= 2 for
-  // unit vectors; the top bucket also takes anything above).  Value-domain buckets spread the
-  // shared-memory atomics, which the float's top bits (a few exponents) would not.  The
-  // distances are staged in shared memory on the way, when they fit.
-  if (N <= prm.stage) {
-    // 16-byte copies for the 16-byte-aligned interior of db, 4-byte ones for the ends; the staged
-    // copy starts at db's offset within 16 bytes, so each interior copy is aligned at both ends
-    const int mis = static_cast<int>((reinterpret_cast<uintptr_t>(db) >> 2) & 3u);
-    float* s0 = sd + mis;
-    const int head = min(N, (4 - mis) & 3);
-    const int nvec = (N - head) >> 2;
-    for (int i = threadIdx.x; i < head; i += blockDim.x) cp_async4(s0 + i, db + i);
-    for (int v = threadIdx.x; v < nvec; v += blockDim.x) cp_async16(s0 + head + 4 * v, db + head + 4 * v);
-    for (int i = head + 4 * nvec + threadIdx.x; i < N; i += blockDim.x) cp_async4(s0 + i, db + i);
-    db = s0;
-  }
-  for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
-  cp_async_wait_all();
-  __syncthreads();
-#pragma unroll 4
-  for (int i = threadIdx.x; i < N; i += blockDim.x) atomicAdd(&bins[tail_bucket(db[i])], 1u);
-  __syncthreads();
-  select_from_top<kTailBins>(bins, k, sel, cred);
-  const int tb = static_cast<int>(sel[0]);
-  const unsigned cb = bins[tb];   // entries in the k-th largest's bucket
-  unsigned lo = __float_as_uint(static_cast<float>(tb) * (1.0f / 2048.0f));
-  unsigned span = (tb == kTailBins - 1 ? 0x7F800001u : __float_as_uint(static_cast<float>(tb + 1) * (1.0f / 2048.0f))) - lo;
-  unsigned remaining = k - sel[1];
-  float s = 0.f;                    // this thread's share of the entries above the k-th largest
-  unsigned long long s_fix = 0ull;  // ... the bucket members among them, 2^-32 fixed point
-  unsigned cnt = 0u;
-  unsigned prefix;
-  if (cb <= kTailBins) {
-    // Level 2 on a short list.  One pass compacts the bucket's members into `bins` (free after
-    // the level-1 select) and sums the entries of the buckets above it; the members are then
-    // narrowed by key offset from the bucket's first key, 1024 offsets (2^shift keys each) at a
-    // time, until one key is left: the k-th largest distance.  The list order depends on warp
-    // timing, so the members' sum is taken in fixed point (exact, order-independent).
-    __syncthreads();   // everyone has read sel and bins[tb]
-    if (threadIdx.x == 0) ncomp = 0u;
-    __syncthreads();
-#pragma unroll 4
-    for (int i = threadIdx.x; i < N; i += blockDim.x) {   // the members are few: one slot each
-      const float v = db[i];
-      const int bk = tail_bucket(v);
-      if (bk > tb) {
-        s += v;
-        ++cnt;
-      } else if (bk == tb) {
-        bins[atomicAdd(&ncomp, 1u)] = __float_as_uint(v);
-      }
-    }
-    __syncthreads();
-    if (cb <= blockDim.x) {
-      // one member per thread, ranked against the whole list: a member with fewer than
-      // `remaining` members at or above it lies above the k-th largest (and is summed); with fewer
-      // than `remaining` above it but at least that many at or above it, it is the k-th largest
-      int mi;
-      unsigned gt, ge;
-      if (rank_in_list(bins, cb, mi, gt, ge)) {
-        const unsigned mine = bins[mi];
-        if (ge < remaining) {
-          s_fix += fix32(__uint_as_float(mine));
-          ++cnt;
-        } else if (gt < remaining) {
-          sel[0] = mine;   // the same key from every member equal to it
-        }
-      }
-      __syncthreads();
-      prefix = sel[0];
-    } else {
-      while (true) {
-        const int bits = 32 - __clz(span - 1u);
-        const int shift = bits > 10 ? bits - 10 : 0;
-        for (int i = threadIdx.x; i < kTailBins2; i += blockDim.x) hist2[i] = 0u;
-        __syncthreads();
-        for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
-          const unsigned off = bins[i] - lo;   // wraps for keys below lo
-          if (off < span) atomicAdd(&hist2[off >> shift], 1u);
-        }
-        __syncthreads();
-        select_from_top<kTailBins2>(hist2, remaining, sel, cred);
-        lo += sel[0] << shift;
-        remaining -= sel[1];
-        if (shift == 0) break;
-        span = min(span - (sel[0] << shift), 1u << shift);
-      }
-      prefix = lo;
-      for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) {
-        const unsigned key = bins[i];
-        if (key > prefix) {
-          s_fix += fix32(__uint_as_float(key));
-          ++cnt;
-        }
-      }
-    }
-  } else {
-    // Level 2 over the whole array (a crowded bucket): the bucket's members by key offset from
-    // its first key, 4096 offsets (2^shift keys each) at a time, until one key is left.
-    while (true) {
-      const int bits = 32 - __clz(span - 1u);        // keys lo .. lo + span - 1 need `bits` bits
-      const int shift = bits > 12 ? bits - 12 : 0;
-      __syncthreads();                               // everyone has read sel and the bins
-      for (int i = threadIdx.x; i < kTailBins; i += blockDim.x) bins[i] = 0u;
-      __syncthreads();
-      for (int base = 0; base < N; base += blockDim.x) {   // uniform trip count: __match_any_sync below
-        const int i = base + static_cast<int>(threadIdx.x);
-        const unsigned off = i < N ? __float_as_uint(db[i]) - lo : span;   // wraps for keys below lo
-        const bool in = off < span;
-        const unsigned digit = in ? off >> shift : kTailBins;
-        const unsigned members = __ballot_sync(0xffffffffu, in);
-        if (__popc(members) > 4) {
-          // many members in this warp: lanes with the same digit add once (identical distances
-          // would otherwise serialise on one counter)
-          const unsigned peers = __match_any_sync(0xffffffffu, digit);
-          if (in && lane_id == __ffs(peers) - 1) atomicAdd(&bins[digit], static_cast<unsigned>(__popc(peers)));
-        } else if (in) {
-          atomicAdd(&bins[digit], 1u);
-        }
-      }
-      __syncthreads();
-      select_from_top<kTailBins>(bins, remaining, sel, cred);
-      lo += sel[0] << shift;
-      remaining -= sel[1];
-      if (shift == 0) break;
-      span = min(span - (sel[0] << shift), 1u << shift);
-    }
-    prefix = lo;
-    for (int i = threadIdx.x; i < N; i += blockDim.x) {
-      const float v = db[i];
-      if (__float_as_uint(v) > prefix) {
-        s += v;
-        ++cnt;
-      }
-    }
-  }
-  const float T = __uint_as_float(prefix);   // k-th largest d
-  s = warp_sum_f(s);
-  for (int o = 16; o > 0; o >>= 1) {
-    cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
-    s_fix += __shfl_xor_sync(0xffffffffu, s_fix, o);
-  }
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) {
-    red[warp] = s;
-    cred[warp] = cnt;
-    fred[warp] = s_fix;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float tot = 0.f;
-    unsigned c = 0u;
-    unsigned long long f = 0ull;
-    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) {
-      tot += red[w];
-      c += cred[w];
-      f += fred[w];
-    }
-    tot += unfix32<false>(f, 1.0f);
-    tot += static_cast<float>(k - c) * T;  // the remaining entries all equal T
-    tail_finish(t, b, prm, stats, stats[t.b_base + b].rho_g, tot / static_cast<float>(k));
-  }
-}
-
-// The density tail over several CTAs per image (the pixel density call; pass 2 has counted the
-// distances per bucket).  CTA c of image b takes distances c kTailChunk .. : it selects the k-th
-// largest's bucket from the counts (level 1 of apc_tail), adds the distances above that bucket
-// to the image's total in 2^-32 fixed point (exact, so the order of the CTAs does not matter)
-// and lists the bucket's members.  The image's last CTA to finish narrows the members to the
-// k-th largest distance T (apc_tail's level 2: a direct rank, or offset rounds) and writes the
-// statistics; a bucket too crowded for the list is narrowed over the whole array instead.
+// The density tail (Eq. 5: the mean of the k_tail largest d_i, then Eq. 6 and R3-R4), several
+// CTAs per image; pass 2 has counted the distances into 4096 value buckets of width 1/2048 (the
+// top one also takes anything above).  CTA c of image b takes distances c kTailChunk .. : it
+// selects the k-th largest's bucket from the counts (level 1), adds the distances above that
+// bucket to the image's total in 2^-32 fixed point (exact, so the order of the CTAs does not
+// matter) and lists the bucket's members.  The image's last CTA to finish narrows the members to
+// the k-th largest distance T (level 2: each member ranked against the others when there are at
+// most 1024, else rounds of 1024 bins over the key offsets from the bucket's first fp32 key) and
+// writes the statistics; a bucket too crowded for the list is narrowed over the whole array by
+// rounds of 4096 bins.
 __global__ void __launch_bounds__(1024) apc_tail_scan(const __grid_constant__ ApcTable t, const float* __restrict__ d,
                                                       TailParams prm, pace_apc_stats* __restrict__ stats,
                                                       TailWork* __restrict__ work) {
@@ -973,7 +794,9 @@ __global__ void __launch_bounds__(1024) apc_tail_scan(const __grid_constant__ Ap
     for (int i = threadIdx.x; i < static_cast<int>(cb); i += blockDim.x) bins[i] = __ldcg(&w->list[i]);
     __syncthreads();
     if (cb <= blockDim.x) {
-      // one member per thread, ranked against the whole list (as apc_tail)
+      // one member per thread, ranked against the whole list: a member with fewer than
+      // `remaining` members at or above it lies above the k-th largest (and is summed); with fewer
+      // than `remaining` above it but at least that many at or above it, it is the k-th largest
       int mi;
       unsigned gt, ge;
       if (rank_in_list(bins, cb, mi, gt, ge)) {
@@ -1015,7 +838,7 @@ __global__ void __launch_bounds__(1024) apc_tail_scan(const __grid_constant__ Ap
     }
   } else {
     // a crowded bucket: its members by key offset from its first key over the whole array,
-    // 4096 offsets (2^shift keys each) at a time, until one key is left (as apc_tail)
+    // 4096 offsets (2^shift keys each) at a time, until one key is left
     while (true) {
       const int bits = 32 - __clz(span - 1u);
       const int shift = bits > 12 ? bits - 12 : 0;
@@ -1278,7 +1101,8 @@ __global__ void __launch_bounds__(kApcThreads) apc_pix_pass2(const __grid_consta
                                                              const float* __restrict__ tokens,
                                                              const unsigned long long* __restrict__ sums,
                                                              float* __restrict__ d_out,
-                                                             pace_apc_stats* __restrict__ stats) {
+                                                             pace_apc_stats* __restrict__ stats,
+                                                             TailWork* __restrict__ work) {
   const int b = find_pix_image(t, blockIdx.x);
   const int u = blockIdx.x - t.unit_prefix[b];
   const int i = u * kApcThreads + threadIdx.x;
@@ -1308,7 +1132,9 @@ __global__ void __launch_bounds__(kApcThreads) apc_pix_pass2(const __grid_consta
     const float x = v[k] - c[k] * inv_c;
     acc = fmaf(x, x, acc);
   }
-  d_out[t.tok0[b] + i] = sqrtf(acc);
+  const float dv = sqrtf(acc);
+  d_out[t.tok0[b] + i] = dv;
+  atomicAdd(&work[t.b_base + b].hist[tail_bucket(dv)], 1u);   // the tail's bucket counts
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -1656,7 +1482,6 @@ DensityLayout density_layout(int B, const int32_t* H, const int32_t* W) {
   return L;
 }
 
-// Dynamic shared memory of apc_tail: the largest image's distances when they fit.
 // Grid of the strip passes: the CTAs that are resident at once (capped by the strips).
 unsigned strip_grid(int units) {
   static std::atomic<int> cap[64];
@@ -1673,18 +1498,6 @@ unsigned strip_grid(int units) {
   return static_cast<unsigned>(std::max(1, std::min(units, c)));
 }
 
-// Launches apc_tail on one ApcTable: when every image's distances fit kTailSmemMax, the launch
-// stages them in dynamic shared memory sized for the largest (+ 16 bytes: the staged copy keeps
-// the distances' offset within 16 bytes); otherwise no image is staged (tp.stage = 0), so an image
-// that would fit cannot write past a buffer sized for another launch.
-void launch_tail(const ApcTable& t, const float* d, TailParams tp, pace_apc_stats* stats, cudaStream_t stream) {
-  int n = 0;
-  for (int i = 0; i < t.nb; ++i) n = std::max(n, t.n[i]);
-  tp.stage = n <= kTailSmemMax ? n : 0;
-  const size_t smem = tp.stage > 0 ? static_cast<size_t>(n) * sizeof(float) + 16 : 0;
-  apc_tail<<<t.nb, 1024, smem, stream>>>(t, d, tp, stats);
-}
-
 // Launches apc_tail_scan on one ApcTable: kTailChunk distances per CTA, the largest image's
 // chunks per row of the grid (CTAs past a smaller image's chunks return at once).
 void launch_tail_scan(const ApcTable& t, const float* d, TailParams tp, pace_apc_stats* stats, TailWork* work,
@@ -1695,17 +1508,6 @@ void launch_tail_scan(const ApcTable& t, const float* d, TailParams tp, pace_apc
                                                                                                      work);
 }
 
-pace_status_t tail_smem_attr() {
-  static DeviceOnce once;
-  int dev = 0;
-  PACE_CUDA(cudaGetDevice(&dev));
-  if (!once.done(dev)) {
-    PACE_CUDA(cudaFuncSetAttribute(apc_tail, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                   static_cast<int>(kTailSmemMax * sizeof(float) + 16)));
-    once.mark(dev);
-  }
-  return PACE_OK;
-}
 
 pace_status_t check_images(const uint8_t* img, const int64_t* off, const int32_t* H, const int32_t* W, int B) {
   if (B < 0) return PACE_ERR_INVALID_ARG;
@@ -1746,7 +1548,6 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
   const DensityLayout L = density_layout(B, H, W);
   if (ws == nullptr || ws_bytes < L.total || reinterpret_cast<uintptr_t>(ws) % 16) return PACE_ERR_WORKSPACE;
   PACE_CHECK(check_device());
-  PACE_CHECK(tail_smem_attr());
   uint8_t* w8 = static_cast<uint8_t*>(ws);
   auto* sums = reinterpret_cast<unsigned long long*>(w8 + L.sums_off);
   auto* work = reinterpret_cast<TailWork*>(w8 + L.work_off);
@@ -1786,7 +1587,7 @@ extern "C" pace_status_t pace_apc_density(const uint8_t* img, const int64_t* img
     if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats, work);
     else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d, stats, work);
     PACE_CHECK(check_launch());
-    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
     launch_tail_scan(t, d, tp, stats, work, stream);
     PACE_CHECK(check_launch());
   }
@@ -1920,7 +1721,6 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
       !(p.r_min <= p.r_max) || p.align < 1)
     return PACE_ERR_INVALID_ARG;
   PACE_CHECK(check_device());
-  PACE_CHECK(tail_smem_attr());
   unsigned char* scratch = nullptr;
   PACE_CHECK(static_scratch(&scratch));
   auto* sums = reinterpret_cast<unsigned long long*>(scratch);
@@ -1960,7 +1760,7 @@ extern "C" pace_status_t pace_apc_density_static(const uint8_t* img, const int64
   if (wide) apc_pass2<true><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats, work);
   else apc_pass2<false><<<strip_grid(units), kApcThreads, 0, stream>>>(img, t, units, inv, sums, d_out, stats, work);
   PACE_CHECK(check_launch());
-  TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
+  TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
   launch_tail_scan(t, d_out, tp, stats, work, stream);
   return check_launch();
 }
@@ -1998,12 +1798,14 @@ unsigned tok_pass1_grid(int units) {
 }
 
 struct TokLayout {
-  size_t sums_off, inv_off, total;
+  size_t sums_off, work_off, zero_bytes, inv_off, total;   // [0, zero_bytes) is zeroed per call
 };
 TokLayout tok_layout(int B, const int32_t* cu, int D) {
   TokLayout L{};
   L.sums_off = 0;
-  L.inv_off = align_up(static_cast<size_t>(B) * D * sizeof(unsigned long long), 256);
+  L.work_off = align_up(static_cast<size_t>(B) * D * sizeof(unsigned long long), 256);
+  L.zero_bytes = L.work_off + static_cast<size_t>(B) * sizeof(TailWork);
+  L.inv_off = align_up(L.zero_bytes, 256);
   L.total = L.inv_off + align_up(static_cast<size_t>(cu[B]) * sizeof(float), 256);
   return L;
 }
@@ -2036,16 +1838,16 @@ extern "C" pace_status_t pace_apc_density_tokens(const void* T, const int32_t* c
   const TokLayout L = tok_layout(B, cu_tokens, D);
   if (ws == nullptr || ws_bytes < L.total || reinterpret_cast<uintptr_t>(ws) % 16) return PACE_ERR_WORKSPACE;
   PACE_CHECK(check_device());
-  PACE_CHECK(tail_smem_attr());
   uint8_t* w8 = static_cast<uint8_t*>(ws);
   auto* sums = reinterpret_cast<unsigned long long*>(w8 + L.sums_off);
+  auto* work = reinterpret_cast<TailWork*>(w8 + L.work_off);
   auto* inv = reinterpret_cast<float*>(w8 + L.inv_off);
-  PACE_CUDA(cudaMemsetAsync(sums, 0, static_cast<size_t>(B) * D * sizeof(unsigned long long), stream));
+  PACE_CUDA(cudaMemsetAsync(w8, 0, L.zero_bytes, stream));   // column sums and tail scratch
   const uint32_t* T32 = static_cast<const uint32_t*>(T);
   for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
     const int nb = (B - c0) < kApcMaxB ? (B - c0) : kApcMaxB;
     TokTable tt{};
-    ApcTable at{};   // what the shared tail kernel reads: sizes, token ranges, k_tail
+    ApcTable at{};   // what the tail kernel reads: sizes, token ranges, k_tail
     tt.nb = at.nb = nb;
     tt.b_base = at.b_base = c0;
     tt.D = D;
@@ -2073,10 +1875,10 @@ extern "C" pace_status_t pace_apc_density_tokens(const void* T, const int32_t* c
     PACE_CHECK(tok_pass1_attr());
     apc_tok_pass1<<<tok_pass1_grid(units1), kApcThreads, smem1, stream>>>(T32, tt, units1, inv, sums);
     PACE_CHECK(check_launch());
-    apc_tok_pass2<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums, d_out, stats);
+    apc_tok_pass2<<<units, kApcThreads, 0, stream>>>(T32, tt, inv, sums, d_out, stats, work);
     PACE_CHECK(check_launch());
-    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
-    launch_tail(at, d_out, tp, stats, stream);
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
+    launch_tail_scan(at, d_out, tp, stats, work, stream);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;
@@ -2157,7 +1959,8 @@ extern "C" size_t pace_apc_density_pixel_workspace_size(int B, const int32_t* H,
   for (int b = 0; b < B; ++b)
     if (H[b] < kPatch || W[b] < kPatch) return 0;
   return align_up(static_cast<size_t>(total_patches(B, H, W)) * kPixDim * sizeof(float), 256) +
-         align_up(static_cast<size_t>(B) * kPixDim * sizeof(unsigned long long), 256);
+         align_up(static_cast<size_t>(B) * kPixDim * sizeof(unsigned long long), 256) +
+         static_cast<size_t>(B) * sizeof(TailWork);
 }
 
 extern "C" pace_status_t pace_apc_density_pixel(const uint8_t* img, const int64_t* img_off, const int32_t* H,
@@ -2178,10 +1981,11 @@ extern "C" pace_status_t pace_apc_density_pixel(const uint8_t* img, const int64_
       reinterpret_cast<uintptr_t>(ws) % 16)
     return PACE_ERR_WORKSPACE;
   PACE_CHECK(check_device());
-  PACE_CHECK(tail_smem_attr());
   auto* tokens = static_cast<float*>(ws);
   auto* sums = reinterpret_cast<unsigned long long*>(static_cast<uint8_t*>(ws) + tok_bytes);
-  PACE_CUDA(cudaMemsetAsync(sums, 0, static_cast<size_t>(B) * kPixDim * sizeof(unsigned long long), stream));
+  const size_t sums_bytes = align_up(static_cast<size_t>(B) * kPixDim * sizeof(unsigned long long), 256);
+  auto* work = reinterpret_cast<TailWork*>(reinterpret_cast<uint8_t*>(sums) + sums_bytes);
+  PACE_CUDA(cudaMemsetAsync(sums, 0, sums_bytes + static_cast<size_t>(B) * sizeof(TailWork), stream));   // sums, tail scratch
   int patch0 = 0;
   for (int c0 = 0; c0 < B; c0 += kApcMaxB) {
     const int nb = std::min(kApcMaxB, B - c0);
@@ -2201,10 +2005,10 @@ extern "C" pace_status_t pace_apc_density_pixel(const uint8_t* img, const int64_
     const int units = pt.unit_prefix[nb];
     apc_pix_pass1<<<units, kApcThreads, 0, stream>>>(pt, tokens, sums);
     PACE_CHECK(check_launch());
-    apc_pix_pass2<<<units, kApcThreads, 0, stream>>>(pt, tokens, sums, d_out, stats);
+    apc_pix_pass2<<<units, kApcThreads, 0, stream>>>(pt, tokens, sums, d_out, stats, work);
     PACE_CHECK(check_launch());
-    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align, 0};
-    launch_tail(at, d_out, tp, stats, stream);
+    TailParams tp{p.alpha, p.gamma, p.r_min, p.r_max, p.align};
+    launch_tail_scan(at, d_out, tp, stats, work, stream);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;

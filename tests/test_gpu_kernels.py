@@ -215,6 +215,15 @@ def test_density_constant_images(pace):
         assert (s["h_out"], s["w_out"]) == (28, 28)
 
 
+def _background_with_noise(rng, side, noisy):
+    img = np.full((side, side, 3), 120, dtype=np.uint8)
+    g = side // 14
+    for q in rng.choice(g * g, size=int(noisy * g * g), replace=False):
+        y, x = divmod(int(q), g)
+        img[14 * y:14 * y + 14, 14 * x:14 * x + 14] = rng.integers(0, 256, (14, 14, 3), dtype=np.uint8)
+    return img
+
+
 @pytest.mark.parametrize("side,noisy", [(1008, 0.05), (896, 0.03), (896, 0.5)])
 def test_density_crowded_tail(pace, side, noisy):
     """Images whose tail bucket is crowded with identical distances: a constant background with
@@ -223,13 +232,31 @@ def test_density_crowded_tail(pace, side, noisy):
     there (the compacted list, full of equal keys); 896^2 at 50 % has the k-th largest among the
     noise patches."""
     rng = np.random.default_rng(side + int(noisy * 100))
-    img = np.full((side, side, 3), 120, dtype=np.uint8)
-    g = side // 14
-    for q in rng.choice(g * g, size=int(noisy * g * g), replace=False):
-        y, x = divmod(int(q), g)
-        img[14 * y:14 * y + 14, 14 * x:14 * x + 14] = rng.integers(0, 256, (14, 14, 3), dtype=np.uint8)
+    img = _background_with_noise(rng, side, noisy)
     d, st = _density(pace, [img])
     _check_density(d, st, [img])
+    _no_device_error(pace)
+
+
+def test_density_tail_paths_mixed_in_one_call(pace):
+    """The three ways the tail narrows the k-th largest distance, in one call: a crowded bucket
+    (1008^2 at 5 % noise: more equal distances than the member list holds, narrowed over the
+    whole array), a list full of equal keys (896^2 at 3 %: offset rounds over the list) and a
+    short list (a natural image: direct ranking).  The images have 5184, 1056 and 4096 patches,
+    i.e. 2, 1 and 1 CTAs of the tail, so each image's last CTA works beside the others.  Every
+    image must be bit-equal to a call with that image alone, and equal to the oracle."""
+    rng = np.random.default_rng(77)
+    imgs = [_background_with_noise(rng, 1008, 0.05), synth.make_image(rng, 448, 462, 4, 4, 0.5),
+            _background_with_noise(rng, 896, 0.03)]
+    d, st = _density(pace, imgs)
+    p0 = 0
+    for b, im in enumerate(imgs):
+        d1, st1 = _density(pace, [im])
+        n = d1.size
+        np.testing.assert_array_equal(d[p0:p0 + n], d1)
+        assert st[b] == st1[0], b
+        p0 += n
+    _check_density(d, st, imgs)
     _no_device_error(pace)
 
 
