@@ -864,20 +864,34 @@ __global__ void __launch_bounds__(kThreads, 1) attn_colsum(const __grid_constant
   cta_release_tmem(tmem);
 }
 
-// out[m] = sum over groups and the `merge` rows of token m of part[group][row].
+// out[m] = sum over groups and the `merge` rows of token m of part[group][row].  Four lanes per
+// output: lane j sums groups j, j + 4, .. in order, then the four partial sums are added by a
+// fixed shuffle tree (the same bits for any launch), so 4x more loads are in flight than with
+// one thread per output.
+constexpr int kReduceLanes = 4;
 __global__ void __launch_bounds__(256) attn_reduce(const float* __restrict__ part, int groups, int ktot, int merge,
                                                    float* __restrict__ out) {
-  const int m = blockIdx.x * blockDim.x + threadIdx.x;
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int m = tid / kReduceLanes, j = tid % kReduceLanes;
   const int nout = ktot / merge;
-  if (m >= nout) return;
   float s = 0.f;
-  for (int g = 0; g < groups; ++g) {
-    const float* p = part + static_cast<int64_t>(g) * ktot + static_cast<int64_t>(m) * merge;
-    float gs = 0.f;
-    for (int q = 0; q < merge; ++q) gs += p[q];
-    s += gs;
+  if (m < nout) {
+    for (int g = j; g < groups; g += kReduceLanes) {
+      const float* p = part + static_cast<int64_t>(g) * ktot + static_cast<int64_t>(m) * merge;
+      float gs;
+      if (merge == 4 && (ktot & 3) == 0) {   // 16-byte aligned rows of four
+        const float4 v = __ldg(reinterpret_cast<const float4*>(p));
+        gs = (v.x + v.y) + (v.z + v.w);
+      } else {
+        gs = 0.f;
+        for (int q = 0; q < merge; ++q) gs += p[q];
+      }
+      s += gs;
+    }
   }
-  out[m] = s;
+  s += __shfl_xor_sync(0xffffffffu, s, 1);
+  s += __shfl_xor_sync(0xffffffffu, s, 2);
+  if (j == 0 && m < nout) out[m] = s;
 }
 
 // ------------------------------------------------------------------------------------------------
@@ -1141,7 +1155,8 @@ pace_status_t run_importance(const void* Q, const void* K, int64_t qrows, int64_
   }
   const int nout = static_cast<int>(Lay.ktot / merge);
   if (nout > 0) {
-    attn_reduce<<<(nout + 255) / 256, 256, 0, stream>>>(part, Hkv, static_cast<int>(Lay.ktot), merge, out);
+    attn_reduce<<<(nout * kReduceLanes + 255) / 256, 256, 0, stream>>>(part, Hkv, static_cast<int>(Lay.ktot), merge,
+                                                                         out);
     PACE_CHECK(check_launch());
   }
   return PACE_OK;
